@@ -1,0 +1,420 @@
+#!/usr/bin/env python3
+"""TurboAngle KV-cache encode/decode benchmark on GB300 (libtac, sm_103a).
+
+One step = encode every (layer, K/V) block of a synthetic KV cache into packed
+records (tac_encode_multi, one launch) and decode every record back to bf16
+(tac_decode_multi, one launch).  Default workload: the Mistral-7B-shaped cache
+(32 layers x 8 KV heads x 32768 tokens x d 128, bf16; early-boost n = 256 on
+layers 0-3, n = 64 elsewhere; K 8-bit linear / V 4-bit log norms).
+
+value = algorithmic bytes moved per step (bf16 rows in + packed records out for
+encode, records in + bf16 rows out for decode) / step time, summed over ranks.
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tac|reference]
+       [--config mistral7b|llama1b|append|longctx]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads  # noqa: E402
+
+METRIC = "KV encode / decode GB/s (bf16 in/out) on 1 GB300 and % of HBM peak"
+UNIT = "GB/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["tac", "reference"], default="tac")
+    ap.add_argument("--config", default="mistral7b", choices=["mistral7b", "llama1b", "append", "longctx"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-rows", type=int, default=400_000,
+                    help="rows in the bounded oracle sample (CPU baseline / reference arm)")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    Q = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            cmd = ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "100"]
+            if self.uuid:
+                cmd += ["-i", self.uuid]
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+        sm, smax, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                sm.append(float(f[2])); smax.append(float(f[3]))
+                power.append(float(f[4]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[6:10]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "power_w_max": max(power) if power else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# workloads
+# ---------------------------------------------------------------------------
+def record_bytes(d, n, b):
+    import math
+    return d // 2 * int(math.log2(n)) // 8 + d // 2 * b // 8 + 8
+
+
+def config_desc(name):
+    if name == "append":
+        a = workloads.APPEND
+        w = workloads.CONFIGS[a["base"]]
+        return (f"decode-step append: {a['seqs']} seqs x {w.layers} L x 2 (K,V) x {w.heads} KV heads x d {w.d}, "
+                f"1 bf16 token each into paged pools ({a['pool_pages']} pages x {a['page']} tok per (L,kv)), "
+                "codebooks as mistral7b; encode only")
+    w = workloads.CONFIGS[name]
+    sched = "early-boost" if len(set(w.n_k)) > 1 else "uniform"
+    return (f"{name}-shaped KV cache: {w.layers} L x 2 (K,V) x {w.heads} KV heads x {w.tokens} T x d {w.d}, "
+            f"{w.dtype}; {sched} n_K={sorted(set(w.n_k))} n_V={sorted(set(w.n_v))}; "
+            f"K {w.b_k}-bit linear / V {w.b_v}-bit log norms")
+
+
+class Workset:
+    """Device-resident cache, records and decode output of one rank, plus byte accounting."""
+
+    def __init__(self, tac, name, seed, device):
+        import torch
+        self.name = name
+        self.enc_jobs, self.dec_jobs = [], []
+        self.enc_bytes = 0
+        self.dec_bytes = 0
+        self.tokens = 0
+        if name == "append":
+            a = workloads.APPEND
+            w = workloads.CONFIGS[a["base"]]
+            rows = a["seqs"] * w.heads
+            blocks = w.blocks()
+            self.x_all = torch.empty((len(blocks), rows, w.d), dtype=torch.bfloat16, device=device)
+            slots = torch.from_numpy(workloads.append_slots(seed, 0)).to(device)
+            cap = workloads.append_capacity()
+            for bi, (l, kv) in enumerate(blocks):
+                d, n, b, mode = w.codebook(l, kv)
+                cfg = tac.layer_cfg(d, n, b, mode, seed, l, kv)
+                x = workloads.block(w, l, kv, tokens=a["seqs"], seed=seed + 11, device=device)
+                self.x_all[bi].copy_(x.view(w.heads, a["seqs"], d).transpose(0, 1).reshape(rows, d))
+                cache = tac.Cache.empty(cfg, cap, device=device)
+                self.enc_jobs.append(tac.EncodeJob(cfg, self.x_all[bi], cache, slots))
+                self.enc_bytes += rows * (2 * d + record_bytes(d, n, b))
+            self.tokens = a["seqs"]
+            self.y_all = None
+            return
+        w = workloads.CONFIGS[name]
+        blocks = w.blocks()
+        R = w.rows_per_block
+        self.x_all = torch.empty((len(blocks), R, w.d), dtype=torch.bfloat16, device=device)
+        self.y_all = torch.empty_like(self.x_all)
+        for bi, (l, kv) in enumerate(blocks):
+            d, n, b, mode = w.codebook(l, kv)
+            cfg = tac.layer_cfg(d, n, b, mode, seed, l, kv)
+            self.x_all[bi].copy_(workloads.block(w, l, kv, seed=seed, device=device, dtype=torch.bfloat16))
+            cache = tac.Cache.empty(cfg, R, device=device)
+            self.enc_jobs.append(tac.EncodeJob(cfg, self.x_all[bi], cache))
+            self.dec_jobs.append(tac.DecodeJob(cfg, cache, self.y_all[bi]))
+            rb = record_bytes(d, n, b)
+            self.enc_bytes += R * (2 * d + rb)
+            self.dec_bytes += R * (rb + 2 * d)
+        self.tokens = w.tokens
+
+    @property
+    def step_bytes(self):
+        return self.enc_bytes + self.dec_bytes
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle on a bounded sample (cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+def oracle_sample(name, total_rows, seed=0):
+    """A bounded sample of the workload: the first rows of every (layer, K/V) block."""
+    import numpy as np
+    base = workloads.APPEND["base"] if name == "append" else name
+    w = workloads.CONFIGS[base]
+    blocks = w.blocks()
+    per = max(8, total_rows // len(blocks))
+    out = []
+    for (l, kv) in blocks:
+        x = workloads.block(w, l, kv, tokens=-(-per // w.heads), seed=seed)[:per].double().numpy()
+        out.append(((l, kv), np.ascontiguousarray(x)))
+    return w, out
+
+
+def run_oracle(w, sample, threads, do_decode=True):
+    import oracle
+    nbytes = 0
+    t0 = time.perf_counter()
+    for (l, kv), x in sample:
+        d, n, b, mode = w.codebook(l, kv)
+        s = oracle.signs(0, l, kv, d)
+        r = oracle.encode_threads(x, s, n, b, mode, threads)
+        rb = record_bytes(d, n, b)
+        nbytes += x.shape[0] * (2 * d + rb)
+        if do_decode:
+            oracle.decode_threads(r["k"], r["c"], r["hdr"], s, n, b, mode, threads)
+            nbytes += x.shape[0] * (rb + 2 * d)
+    return nbytes, time.perf_counter() - t0
+
+
+def cpu_baseline(args):
+    import oracle
+    oracle.build()
+    threads = os.cpu_count() or 1
+    w, sample = oracle_sample(args.config, args.cpu_rows)
+    rows = sum(x.shape[0] for _, x in sample)
+    nbytes, dt = run_oracle(w, sample, threads, do_decode=args.config != "append")
+    what = "encode" if args.config == "append" else "encode+decode"
+    return {"value": nbytes / dt / 1e9, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{rows} rows ({len(sample)} blocks x {sample[0][1].shape[0]} first rows), {what}, "
+                      f"fp64 dense-Hadamard oracle, {dt:.1f} s wall on {threads} host threads"}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    threads = os.cpu_count() or 1
+    per_step = max(2048, args.cpu_rows // 20)
+    w, sample = oracle_sample(args.config, per_step)
+    rows = sum(x.shape[0] for _, x in sample)
+    do_dec = args.config != "append"
+    for _ in range(args.warmup):
+        run_oracle(w, sample, threads, do_dec)
+    times, nbytes = [], 0
+    for _ in range(args.steps):
+        nb, dt = run_oracle(w, sample, threads, do_dec)
+        times.append(dt)
+        nbytes = nb
+    tot = sum(times)
+    value = nbytes * args.steps / tot / 1e9
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": tot / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": config_desc(args.config), "sample_rows_per_step": rows},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": f"{rows} rows per step (first rows of each of {len(sample)} blocks)"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    import torch
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    from paper_2603_27467_gb300 import build as tb
+    tb.build()
+    import paper_2603_27467_gb300 as tac
+    tac.load()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    ws = Workset(tac, args.config, seed=rank, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+    enc_only = args.config == "append"
+
+    def step():
+        tac.encode_multi(ws.enc_jobs, stream=stream)
+        if not enc_only:
+            tac.decode_multi(ws.dec_jobs, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    barrier()
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    uuid = None
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        uuid = None
+    clk = ClockSampler(uuid)
+    clk.start()
+    time.sleep(0.3)
+    barrier()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(K):
+        ev[i][0].record(stream)
+        tac.encode_multi(ws.enc_jobs, stream=stream)
+        ev[i][1].record(stream)
+        if not enc_only:
+            tac.decode_multi(ws.dec_jobs, stream=stream)
+        ev[i][2].record(stream)
+    t_end.record(stream)
+    barrier()
+    clocks = clk.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    enc_ms = [e[0].elapsed_time(e[1]) for e in ev]
+    dec_ms = [e[1].elapsed_time(e[2]) for e in ev] if not enc_only else [0.0]
+    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms = float(t.item())
+    launches_per_step = (1 if enc_only else 2) * (1 + (len(ws.enc_jobs) - 1) // 96)
+
+    step_bytes = ws.enc_bytes + (0 if enc_only else ws.dec_bytes)
+    value = world * step_bytes * K / (total_ms / 1e3) / 1e9
+    hbm, peak_kind = peaks()
+    enc_avg = statistics.mean(enc_ms)
+    dec_avg = statistics.mean(dec_ms)
+    enc_gbs = ws.enc_bytes / (enc_avg / 1e3) / 1e9
+    dec_gbs = ws.dec_bytes / (dec_avg / 1e3) / 1e9 if not enc_only else None
+    dom = "encode" if enc_only or sum(enc_ms) >= sum(dec_ms) else "decode"
+    dom_gbs = enc_gbs if dom == "encode" else dec_gbs
+    dom_bytes = ws.enc_bytes if dom == "encode" else ws.dec_bytes
+
+    # e2e: same step through the C ABI from pinned host buffers, copies inside the timed region
+    e2e = None
+    if not args.no_e2e and not enc_only:
+        hx = torch.empty(ws.x_all.shape, dtype=ws.x_all.dtype, pin_memory=True)
+        hx.copy_(ws.x_all)
+        hy = torch.empty(ws.y_all.shape, dtype=ws.y_all.dtype, pin_memory=True)
+        with torch.cuda.stream(stream):
+            ws.x_all.copy_(hx, non_blocking=True)
+            step()
+            hy.copy_(ws.y_all, non_blocking=True)
+        barrier()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        with torch.cuda.stream(stream):
+            for _ in range(args.e2e_steps):
+                ws.x_all.copy_(hx, non_blocking=True)
+                step()
+                hy.copy_(ws.y_all, non_blocking=True)
+        e1.record(stream)
+        barrier()
+        et = torch.tensor([e0.elapsed_time(e1)], dtype=torch.float64, device=dev)
+        if world > 1:
+            dist.all_reduce(et, op=dist.ReduceOp.MAX)
+        e2e_ms = float(et.item())
+        e2e = {"value": world * step_bytes * args.e2e_steps / (e2e_ms / 1e3) / 1e9, "unit": UNIT,
+               "h2d_bytes_per_step": hx.numel() * hx.element_size(),
+               "d2h_bytes_per_step": hy.numel() * hy.element_size(),
+               "ms_per_step": e2e_ms / args.e2e_steps}
+        del hx, hy
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args)
+
+    if rank == 0:
+        w = workloads.CONFIGS[workloads.APPEND["base"] if enc_only else args.config]
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": config_desc(args.config), "io_dtype": "bf16",
+                       "bytes_per_step_per_gpu": step_bytes,
+                       "l2": "inputs larger than L2 (no flush needed): "
+                             f"{ws.x_all.numel() * 2 / 1e9:.2f} GB of bf16 rows per step",
+                       "parallelism": f"replicas x{world} (independent caches, no collective)"},
+            "pct_hbm_peak": 100.0 * value / world / hbm,
+            "encode_gbs": enc_gbs, "decode_gbs": dec_gbs,
+            "tokens_per_s": world * ws.tokens * w.layers * K / (total_ms / 1e3),
+            "roofline": {"bound": "hbm", "kernel": f"{dom} (tac_{dom}_multi, one launch)",
+                         "achieved": dom_gbs, "peak": hbm, "unit": "GB/s", "frac": dom_gbs / hbm,
+                         "peak_source": f"{peak_kind} hbm_gbs", "traffic": None,
+                         "algorithmic_bytes_per_launch": dom_bytes},
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * K, "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,177 @@
+/*
+ * tac.h -- C ABI of libtac, a GB300 (sm_103a) implementation of the TurboAngle
+ * KV-cache encode/decode path (arXiv 2603.27467, "TurboAngle: Near-Lossless KV
+ * Cache Compression via Uniform Angle Quantization").
+ *
+ * What the library computes, per head vector x of dimension d (one "row"):
+ *   encode (Alg. 1 with Sec. 3.3):
+ *     y = H D x                 D: random +-1 diagonal, H: normalized Hadamard (Sec. 2)
+ *     r_i = |(y_2i, y_2i+1)|, theta_i = atan2(y_2i+1, y_2i)          (Alg. 1)
+ *     k_i = floor(n theta_i / 2 pi + 1/2) mod n                      (Alg. 1)
+ *     c_i = round((r_i - r_min)/(r_max - r_min) (2^b - 1))           (Eq. 2, linear)
+ *           or Eq. 2 applied to log2 r_i                              (Sec. 3.3, log-space)
+ *     stored: k_i (log2 n bits each), c_i (b bits each), (r_min, r_max) as fp32.
+ *   decode (Sec. 3.1): y^_2i = r^_i cos(2 pi k_i / n), y^_2i+1 = r^_i sin(2 pi k_i / n),
+ *     x^ = D H y^, with r^_i the dequantized norm (r_min + c (r_max - r_min)/(2^b - 1), or
+ *     the same in log2 space).
+ *
+ * Record layout ("three planes", caller-owned device memory, one record slot per row):
+ *   angle plane   slot s at  codes + s * tac_angle_row_bytes(cfg):  d/2 codes of log2(n) bits,
+ *                 one LSB-first bitstream per row (code i occupies bits [i*w, i*w + w)).
+ *   norm plane    slot s at  norms + s * tac_norm_row_bytes(cfg):   d/2 codes of b bits, same order.
+ *   header plane  slot s at  norms + tac_header_offset(cfg, capacity) + 8*s:
+ *                 float r_min, float r_max (little endian).
+ *
+ * Conventions shared by every entry point:
+ *   - All device pointers must be 16-byte aligned; rows are row_stride elements
+ *     apart and row_stride * sizeof(element) must be a multiple of 16.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream), allocate nothing, and never synchronize.
+ *   - Errors: a nonzero tac_status is returned and tac_last_error() gives a message
+ *     (per host thread).  TAC_E_INVAL: a bad argument (nothing launched).
+ *     TAC_E_UNSUPPORTED: a valid but unimplemented shape (nothing launched).
+ *     TAC_E_CUDA: the launch failed (cudaGetLastError after the launch).
+ *   - Inputs must be finite with |x_j| <= 2^56; other values give unspecified codes
+ *     but never out-of-bounds accesses.
+ */
+#ifndef TAC_H_
+#define TAC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* tac_stream_t; /* == cudaStream_t */
+
+typedef enum {
+  TAC_OK = 0,
+  TAC_E_INVAL = 1,
+  TAC_E_UNSUPPORTED = 2,
+  TAC_E_CUDA = 3
+} tac_status;
+
+typedef enum { TAC_NORM_LINEAR = 0, TAC_NORM_LOG = 1 } tac_norm_mode;
+typedef enum { TAC_BF16 = 0, TAC_FP32 = 1 } tac_dtype;
+
+#define TAC_MAX_D 128
+#define TAC_MAX_JOBS 96
+
+/*
+ * One codebook: the quantizer of one (layer, K or V) cache (Sec. 3.2 assigns an
+ * independent (n_K, n_V) per layer; Sec. 3.3 picks the norm bits/mode per K/V).
+ * Plain host struct, passed by pointer and copied at each call.
+ */
+typedef struct {
+  int32_t d;          /* head dimension: 16, 32, 64 or 128 */
+  int32_t n_angle;    /* angle bins n: a power of two, 2..256 */
+  int32_t norm_bits;  /* b: 4 or 8 */
+  int32_t norm_mode;  /* tac_norm_mode */
+  uint32_t signs[TAC_MAX_D / 32]; /* D: bit j of the little-endian word array set <=> s_j = -1
+                                     (from tac_make_signs); bits >= d are ignored */
+} tac_layer_cfg;
+
+/* A block of rows: `rows` vectors of cfg.d elements, row i at data + i*row_stride elements. */
+typedef struct {
+  void* data;           /* device pointer */
+  int32_t dtype;        /* tac_dtype */
+  int64_t rows;         /* >= 0 */
+  int64_t row_stride;   /* elements, >= d */
+} tac_rows;
+
+/* One encode job of a batched launch: rows of x -> record slots (scatter-append). */
+typedef struct {
+  tac_layer_cfg cfg;
+  tac_rows x;            /* input rows (device) */
+  void* codes;           /* angle plane of the destination cache (device) */
+  void* norms;           /* norm + header planes of the destination cache (device) */
+  int64_t capacity;      /* record slots in the destination planes */
+  const int64_t* slot;   /* device, x.rows entries: destination slot of row i, each in
+                            [0, capacity); NULL means slot i (then x.rows <= capacity).
+                            Duplicate slots race (one of the writers wins). */
+} tac_encode_job;
+
+/* One decode job of a batched launch: record slots -> rows of y (gather). */
+typedef struct {
+  tac_layer_cfg cfg;
+  const void* codes;     /* angle plane of the source cache (device) */
+  const void* norms;     /* norm + header planes of the source cache (device) */
+  int64_t capacity;      /* record slots in the source planes */
+  const int64_t* slot;   /* device, y.rows entries: source slot of output row i, each in
+                            [0, capacity) (not checked on the device); NULL means slot i */
+  tac_rows y;            /* output rows (device), bf16 (round to nearest even) or fp32 */
+} tac_decode_job;
+
+/*
+ * D of Sec. 2 ("s_i ~ Uniform{+1,-1}", sampled once from a seeded PRNG, Sec. 3.1
+ * implementation note).  Counter-based SplitMix64 (Steele, Lea, Flood 2014):
+ *   key = output #q of the SplitMix64 stream seeded with `seed`, q = 2*layer + kv
+ *         (q = 0 when `shared` != 0: one D for every layer and K/V, as in the paper);
+ *   s_j = -1 iff bit 63 of output #j of the stream seeded with key is set.
+ * Output #i of the stream seeded with z is mix(z + (i+1)*0x9E3779B97F4A7C15).
+ * Writes ceil(d/32) words (host memory).  kv: 0 = K, 1 = V.  Host only.
+ */
+int tac_make_signs(uint64_t seed, int layer, int kv, int shared, int d, uint32_t* out_words);
+
+/* Bytes per row of each plane (Sec. 3.1 rate: log2(n) bits per pair; Eq. 3 norm bits
+ * per pair; 64 bits of header per vector).  Return -1 for an invalid cfg. */
+int64_t tac_angle_row_bytes(const tac_layer_cfg* cfg);   /* d/2 * log2(n) / 8 */
+int64_t tac_norm_row_bytes(const tac_layer_cfg* cfg);    /* d/2 * b / 8 */
+/* Byte offset of the header plane inside `norms` for a cache of `capacity` slots:
+ * capacity * tac_norm_row_bytes rounded up to a multiple of 16. */
+int64_t tac_header_offset(const tac_layer_cfg* cfg, int64_t capacity);
+int64_t tac_codes_bytes(const tac_layer_cfg* cfg, int64_t capacity); /* angle plane size */
+int64_t tac_norms_bytes(const tac_layer_cfg* cfg, int64_t capacity); /* norm + header planes */
+
+/* Eq. 1: (1/L) sum_l (log2 n_K^l + log2 n_V^l) / 4.  Returns NaN if an n is < 1. */
+double tac_avg_angle_bits(int num_layers, const int* n_k, const int* n_v);
+/* Eq. 3: b_angle + b_norm / 2 + 64 / d. */
+double tac_total_bits(double b_angle, double b_norm, int d);
+
+/*
+ * Encode x.rows rows (Alg. 1 + Eq. 2) into record slots 0..x.rows-1 of
+ * (out_codes, out_norms), a cache of capacity x.rows
+ * (sizes: tac_codes_bytes(cfg, x.rows), tac_norms_bytes(cfg, x.rows)).
+ */
+int tac_encode(const tac_rows* x, const tac_layer_cfg* cfg, void* out_codes, void* out_norms,
+               tac_stream_t stream);
+
+/*
+ * Decode y->rows records (slots 0..y->rows-1 of a cache of capacity y->rows) into y
+ * (Sec. 3.1 reconstruction with the Eq. 2 dequantization).
+ */
+int tac_decode(const void* codes, const void* norms, const tac_layer_cfg* cfg, tac_rows* y,
+               tac_stream_t stream);
+
+/*
+ * Batched encode: every job in one launch (one per TAC_MAX_JOBS jobs).  Jobs may
+ * mix codebooks, d and input dtypes of the same d; with `slot` the rows of a decode
+ * step land at per-sequence record slots (streaming append).  Jobs must not write
+ * overlapping slots.
+ */
+int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream);
+
+/* Batched decode: every job in one launch (one per TAC_MAX_JOBS jobs). */
+int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream);
+
+/*
+ * Transform only, for checking the butterfly: y = H D x (Sec. 2), normalized,
+ * written as fp32 rows of d elements (row stride d).  signs: host words as in
+ * tac_layer_cfg.signs.  d: any power of two 2..128.
+ */
+int tac_fwht_debug(const tac_rows* x, int d, const uint32_t* signs, float* y,
+                   tac_stream_t stream);
+
+/* Message of the last failed call on this host thread ("" if none). */
+const char* tac_last_error(void);
+
+/* Library version string. */
+const char* tac_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TAC_H_ */

@@ -1,0 +1,403 @@
+// libtac C ABI: argument checking, plane geometry, rate accounting, the sign
+// generator and the batched launch planner.  Kernels live in tac_encode.cu,
+// tac_decode.cu and tac_fwht_debug.cu.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "tac_common.cuh"
+
+namespace tac {
+cudaError_t launch_encode_16_bf16(const EncParams& p, int sms, cudaStream_t st);
+cudaError_t launch_encode_32_bf16(const EncParams& p, int sms, cudaStream_t st);
+cudaError_t launch_encode_64_bf16(const EncParams& p, int sms, cudaStream_t st);
+cudaError_t launch_encode_128_bf16(const EncParams& p, int sms, cudaStream_t st);
+cudaError_t launch_encode_16_f32(const EncParams& p, int sms, cudaStream_t st);
+cudaError_t launch_encode_32_f32(const EncParams& p, int sms, cudaStream_t st);
+cudaError_t launch_encode_64_f32(const EncParams& p, int sms, cudaStream_t st);
+cudaError_t launch_encode_128_f32(const EncParams& p, int sms, cudaStream_t st);
+cudaError_t launch_decode_16_bf16(const DecParams& p, int sms, cudaStream_t st);
+cudaError_t launch_decode_32_bf16(const DecParams& p, int sms, cudaStream_t st);
+cudaError_t launch_decode_64_bf16(const DecParams& p, int sms, cudaStream_t st);
+cudaError_t launch_decode_128_bf16(const DecParams& p, int sms, cudaStream_t st);
+cudaError_t launch_decode_16_f32(const DecParams& p, int sms, cudaStream_t st);
+cudaError_t launch_decode_32_f32(const DecParams& p, int sms, cudaStream_t st);
+cudaError_t launch_decode_64_f32(const DecParams& p, int sms, cudaStream_t st);
+cudaError_t launch_decode_128_f32(const DecParams& p, int sms, cudaStream_t st);
+
+static cudaError_t launch_encode(int d, int dtype, const EncParams& p, int sms, cudaStream_t st) {
+  const bool bf = dtype == TAC_BF16;
+  switch (d) {
+    case 16: return bf ? launch_encode_16_bf16(p, sms, st) : launch_encode_16_f32(p, sms, st);
+    case 32: return bf ? launch_encode_32_bf16(p, sms, st) : launch_encode_32_f32(p, sms, st);
+    case 64: return bf ? launch_encode_64_bf16(p, sms, st) : launch_encode_64_f32(p, sms, st);
+    case 128: return bf ? launch_encode_128_bf16(p, sms, st) : launch_encode_128_f32(p, sms, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+static cudaError_t launch_decode(int d, int dtype, const DecParams& p, int sms, cudaStream_t st) {
+  const bool bf = dtype == TAC_BF16;
+  switch (d) {
+    case 16: return bf ? launch_decode_16_bf16(p, sms, st) : launch_decode_16_f32(p, sms, st);
+    case 32: return bf ? launch_decode_32_bf16(p, sms, st) : launch_decode_32_f32(p, sms, st);
+    case 64: return bf ? launch_decode_64_bf16(p, sms, st) : launch_decode_64_f32(p, sms, st);
+    case 128: return bf ? launch_decode_128_bf16(p, sms, st) : launch_decode_128_f32(p, sms, st);
+  }
+  return cudaErrorInvalidValue;
+}
+cudaError_t launch_fwht_debug(int d, const void* x, int dtype, int64_t rows, int64_t stride,
+                              const uint32_t* signs, float* y, cudaStream_t st);
+}  // namespace tac
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+int ok() {
+  g_err.clear();
+  return TAC_OK;
+}
+
+int log2_exact(int v) {
+  if (v <= 0 || (v & (v - 1))) return -1;
+  int w = 0;
+  while ((1 << w) < v) ++w;
+  return w;
+}
+
+// SplitMix64 (Steele, Lea, Flood 2014): output #i of the stream seeded with z.
+uint64_t splitmix64(uint64_t z, uint64_t i) {
+  z += (i + 1u) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+int check_cfg(const tac_layer_cfg* c, const char* who) {
+  if (!c) return fail(TAC_E_INVAL, "%s: cfg is NULL", who);
+  if (c->d != 16 && c->d != 32 && c->d != 64 && c->d != 128) {
+    if (c->d > 0 && log2_exact(c->d) >= 1)
+      return fail(TAC_E_UNSUPPORTED, "%s: d = %d not implemented (16, 32, 64, 128)", who, c->d);
+    return fail(TAC_E_INVAL, "%s: d = %d is not a power of two", who, c->d);
+  }
+  const int w = log2_exact(c->n_angle);
+  if (w < 0) {
+    if (c->n_angle > 1) return fail(TAC_E_UNSUPPORTED, "%s: n = %d is not a power of two", who, c->n_angle);
+    return fail(TAC_E_INVAL, "%s: n = %d", who, c->n_angle);
+  }
+  if (w < 1 || w > 8) return fail(TAC_E_UNSUPPORTED, "%s: n = %d outside 2..256", who, c->n_angle);
+  if (c->norm_bits != 4 && c->norm_bits != 8) {
+    if (c->norm_bits >= 1 && c->norm_bits <= 16)
+      return fail(TAC_E_UNSUPPORTED, "%s: norm_bits = %d not implemented (4, 8)", who, c->norm_bits);
+    return fail(TAC_E_INVAL, "%s: norm_bits = %d", who, c->norm_bits);
+  }
+  if (c->norm_mode != TAC_NORM_LINEAR && c->norm_mode != TAC_NORM_LOG)
+    return fail(TAC_E_INVAL, "%s: norm_mode = %d", who, c->norm_mode);
+  return TAC_OK;
+}
+
+int64_t angle_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * log2_exact(c->n_angle) / 8; }
+int64_t norm_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * c->norm_bits / 8; }
+int64_t header_offset(const tac_layer_cfg* c, int64_t cap) { return (cap * norm_row_bytes(c) + 15) & ~(int64_t)15; }
+
+int esize(int dtype) { return dtype == TAC_BF16 ? 2 : dtype == TAC_FP32 ? 4 : 0; }
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+int check_rows(const tac_rows* r, int d, const char* who, const char* name) {
+  if (!r) return fail(TAC_E_INVAL, "%s: %s is NULL", who, name);
+  if (!esize(r->dtype)) return fail(TAC_E_INVAL, "%s: %s.dtype = %d", who, name, r->dtype);
+  if (r->rows < 0) return fail(TAC_E_INVAL, "%s: %s.rows = %lld", who, name, (long long)r->rows);
+  if (r->rows == 0) return TAC_OK;
+  if (!r->data) return fail(TAC_E_INVAL, "%s: %s.data is NULL", who, name);
+  if (!aligned16(r->data)) return fail(TAC_E_INVAL, "%s: %s.data is not 16-byte aligned", who, name);
+  if (r->row_stride < d) return fail(TAC_E_INVAL, "%s: %s.row_stride %lld < d %d", who, name, (long long)r->row_stride, d);
+  if ((r->row_stride * esize(r->dtype)) % 16)
+    return fail(TAC_E_INVAL, "%s: %s.row_stride * sizeof(element) is not a multiple of 16", who, name);
+  if (r->rows > ((int64_t)1 << 38)) return fail(TAC_E_UNSUPPORTED, "%s: %s.rows too large", who, name);
+  return TAC_OK;
+}
+
+int num_sms() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (dev < 0 || dev >= 64) return 0;
+  if (!cache[dev]) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    cache[dev] = v;
+  }
+  return cache[dev];
+}
+
+void copy_signs(uint32_t* dst, const tac_layer_cfg* c) {
+  for (int q = 0; q < 4; ++q) dst[q] = c->signs[q];
+  // bits beyond d are never read by the kernels; clear them for determinism
+  if (c->d < 128) {
+    for (int q = 0; q < 4; ++q) {
+      const int lo = 32 * q;
+      if (lo >= c->d) dst[q] = 0u;
+      else if (c->d - lo < 32) dst[q] &= (1u << (c->d - lo)) - 1u;
+    }
+  }
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* tac_last_error(void) { return g_err.c_str(); }
+
+const char* tac_version(void) { return "libtac 0.1.0 (TurboAngle encode/decode, sm_103a)"; }
+
+int tac_make_signs(uint64_t seed, int layer, int kv, int shared, int d, uint32_t* out_words) {
+  if (!out_words) return fail(TAC_E_INVAL, "tac_make_signs: out_words is NULL");
+  if (d < 1 || d > (1 << 20)) return fail(TAC_E_INVAL, "tac_make_signs: d = %d", d);
+  if (layer < 0) return fail(TAC_E_INVAL, "tac_make_signs: layer = %d", layer);
+  if (kv != 0 && kv != 1) return fail(TAC_E_INVAL, "tac_make_signs: kv = %d (0 = K, 1 = V)", kv);
+  const uint64_t q = shared ? 0u : (uint64_t)(2 * (int64_t)layer + kv);
+  const uint64_t key = splitmix64(seed, q);
+  const int nw = (d + 31) / 32;
+  for (int i = 0; i < nw; ++i) out_words[i] = 0u;
+  for (int j = 0; j < d; ++j)
+    if (splitmix64(key, (uint64_t)j) >> 63) out_words[j >> 5] |= 1u << (j & 31);
+  return ok();
+}
+
+int64_t tac_angle_row_bytes(const tac_layer_cfg* cfg) {
+  if (check_cfg(cfg, "tac_angle_row_bytes")) return -1;
+  return angle_row_bytes(cfg);
+}
+
+int64_t tac_norm_row_bytes(const tac_layer_cfg* cfg) {
+  if (check_cfg(cfg, "tac_norm_row_bytes")) return -1;
+  return norm_row_bytes(cfg);
+}
+
+int64_t tac_header_offset(const tac_layer_cfg* cfg, int64_t capacity) {
+  if (check_cfg(cfg, "tac_header_offset") || capacity < 0) return -1;
+  return header_offset(cfg, capacity);
+}
+
+int64_t tac_codes_bytes(const tac_layer_cfg* cfg, int64_t capacity) {
+  if (check_cfg(cfg, "tac_codes_bytes") || capacity < 0) return -1;
+  return capacity * angle_row_bytes(cfg);
+}
+
+int64_t tac_norms_bytes(const tac_layer_cfg* cfg, int64_t capacity) {
+  if (check_cfg(cfg, "tac_norms_bytes") || capacity < 0) return -1;
+  return header_offset(cfg, capacity) + 8 * capacity;
+}
+
+double tac_avg_angle_bits(int num_layers, const int* n_k, const int* n_v) {
+  if (num_layers <= 0 || !n_k || !n_v) return NAN;
+  double acc = 0.0;
+  for (int l = 0; l < num_layers; ++l) {
+    if (n_k[l] < 1 || n_v[l] < 1) return NAN;
+    acc += (std::log2((double)n_k[l]) + std::log2((double)n_v[l])) / 4.0;
+  }
+  return acc / (double)num_layers;
+}
+
+double tac_total_bits(double b_angle, double b_norm, int d) {
+  if (d <= 0) return NAN;
+  return b_angle + b_norm / 2.0 + 64.0 / (double)d;
+}
+
+int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream) {
+  static const char* who = "tac_encode_multi";
+  if (njobs < 0) return fail(TAC_E_INVAL, "%s: njobs = %d", who, njobs);
+  if (njobs > 0 && !jobs) return fail(TAC_E_INVAL, "%s: jobs is NULL", who);
+  // Validate everything before launching anything.
+  std::vector<int> live;
+  for (int j = 0; j < njobs; ++j) {
+    const tac_encode_job& J = jobs[j];
+    int rc = check_cfg(&J.cfg, who);
+    if (rc) return rc;
+    rc = check_rows(&J.x, J.cfg.d, who, "x");
+    if (rc) return rc;
+    if (J.capacity < 0) return fail(TAC_E_INVAL, "%s: job %d capacity < 0", who, j);
+    if (J.x.rows == 0) continue;
+    if (!J.codes || !J.norms) return fail(TAC_E_INVAL, "%s: job %d codes/norms is NULL", who, j);
+    if (!aligned16(J.codes) || !aligned16(J.norms))
+      return fail(TAC_E_INVAL, "%s: job %d codes/norms not 16-byte aligned", who, j);
+    if (!J.slot && J.x.rows > J.capacity)
+      return fail(TAC_E_INVAL, "%s: job %d rows %lld > capacity %lld", who, j, (long long)J.x.rows,
+                  (long long)J.capacity);
+    if (J.slot && ((uintptr_t)J.slot & 7u)) return fail(TAC_E_INVAL, "%s: job %d slot misaligned", who, j);
+    live.push_back(j);
+  }
+  const int sms = num_sms();
+  if (live.empty()) return ok();
+  if (sms <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
+  // Group by (d, dtype): one kernel instance per group, up to TAC_MAX_JOBS jobs per launch.
+  std::stable_sort(live.begin(), live.end(), [&](int a, int b) {
+    const int ka = jobs[a].cfg.d * 4 + jobs[a].x.dtype, kb = jobs[b].cfg.d * 4 + jobs[b].x.dtype;
+    return ka < kb;
+  });
+  static thread_local tac::EncParams P;
+  size_t i = 0;
+  while (i < live.size()) {
+    const int d = jobs[live[i]].cfg.d, dt = jobs[live[i]].x.dtype;
+    std::memset(&P, 0, sizeof(P));
+    int64_t tiles = 0;
+    while (i < live.size() && P.njobs < TAC_MAX_JOBS && jobs[live[i]].cfg.d == d && jobs[live[i]].x.dtype == dt) {
+      const tac_encode_job& J = jobs[live[i]];
+      const int64_t jt = (J.x.rows + tac::kTileRows - 1) / tac::kTileRows;
+      if (tiles + jt > 0x7fffffff) break;
+      tac::EncJob& E = P.job[P.njobs];
+      E.x = J.x.data;
+      E.codes = static_cast<uint8_t*>(J.codes);
+      E.norms = static_cast<uint8_t*>(J.norms);
+      E.hdr = static_cast<uint8_t*>(J.norms) + header_offset(&J.cfg, J.capacity);
+      E.slot = J.slot;
+      E.capacity = J.capacity;
+      E.rows = J.x.rows;
+      E.stride = J.x.row_stride;
+      copy_signs(E.signs, &J.cfg);
+      E.w = log2_exact(J.cfg.n_angle);
+      E.b = J.cfg.norm_bits;
+      E.mode = J.cfg.norm_mode;
+      E.tile0 = (int32_t)tiles;
+      tiles += jt;
+      ++P.njobs;
+      ++i;
+    }
+    if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many rows", who);
+    P.ntiles = (int32_t)tiles;
+    cudaError_t e = tac::launch_encode(d, dt, P, sms, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+  }
+  return ok();
+}
+
+int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream) {
+  static const char* who = "tac_decode_multi";
+  if (njobs < 0) return fail(TAC_E_INVAL, "%s: njobs = %d", who, njobs);
+  if (njobs > 0 && !jobs) return fail(TAC_E_INVAL, "%s: jobs is NULL", who);
+  std::vector<int> live;
+  for (int j = 0; j < njobs; ++j) {
+    const tac_decode_job& J = jobs[j];
+    int rc = check_cfg(&J.cfg, who);
+    if (rc) return rc;
+    rc = check_rows(&J.y, J.cfg.d, who, "y");
+    if (rc) return rc;
+    if (J.capacity < 0) return fail(TAC_E_INVAL, "%s: job %d capacity < 0", who, j);
+    if (J.y.rows == 0) continue;
+    if (!J.codes || !J.norms) return fail(TAC_E_INVAL, "%s: job %d codes/norms is NULL", who, j);
+    if (!aligned16(J.codes) || !aligned16(J.norms))
+      return fail(TAC_E_INVAL, "%s: job %d codes/norms not 16-byte aligned", who, j);
+    if (!J.slot && J.y.rows > J.capacity)
+      return fail(TAC_E_INVAL, "%s: job %d rows %lld > capacity %lld", who, j, (long long)J.y.rows,
+                  (long long)J.capacity);
+    if (J.slot && ((uintptr_t)J.slot & 7u)) return fail(TAC_E_INVAL, "%s: job %d slot misaligned", who, j);
+    live.push_back(j);
+  }
+  const int sms = num_sms();
+  if (live.empty()) return ok();
+  if (sms <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
+  std::stable_sort(live.begin(), live.end(), [&](int a, int b) {
+    const int ka = jobs[a].cfg.d * 4 + jobs[a].y.dtype, kb = jobs[b].cfg.d * 4 + jobs[b].y.dtype;
+    return ka < kb;
+  });
+  static thread_local tac::DecParams P;
+  size_t i = 0;
+  while (i < live.size()) {
+    const int d = jobs[live[i]].cfg.d, dt = jobs[live[i]].y.dtype;
+    std::memset(&P, 0, sizeof(P));
+    int64_t tiles = 0;
+    while (i < live.size() && P.njobs < TAC_MAX_JOBS && jobs[live[i]].cfg.d == d && jobs[live[i]].y.dtype == dt) {
+      const tac_decode_job& J = jobs[live[i]];
+      const int64_t jt = (J.y.rows + tac::kTileRows - 1) / tac::kTileRows;
+      if (tiles + jt > 0x7fffffff) break;
+      tac::DecJob& E = P.job[P.njobs];
+      E.codes = static_cast<const uint8_t*>(J.codes);
+      E.norms = static_cast<const uint8_t*>(J.norms);
+      E.hdr = static_cast<const uint8_t*>(J.norms) + header_offset(&J.cfg, J.capacity);
+      E.slot = J.slot;
+      E.capacity = J.capacity;
+      E.y = J.y.data;
+      E.rows = J.y.rows;
+      E.stride = J.y.row_stride;
+      copy_signs(E.signs, &J.cfg);
+      E.w = log2_exact(J.cfg.n_angle);
+      E.b = J.cfg.norm_bits;
+      E.mode = J.cfg.norm_mode;
+      E.tile0 = (int32_t)tiles;
+      tiles += jt;
+      ++P.njobs;
+      ++i;
+    }
+    if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many rows", who);
+    P.ntiles = (int32_t)tiles;
+    cudaError_t e = tac::launch_decode(d, dt, P, sms, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+  }
+  return ok();
+}
+
+int tac_encode(const tac_rows* x, const tac_layer_cfg* cfg, void* out_codes, void* out_norms,
+               tac_stream_t stream) {
+  if (!x) return fail(TAC_E_INVAL, "tac_encode: x is NULL");
+  if (!cfg) return fail(TAC_E_INVAL, "tac_encode: cfg is NULL");
+  tac_encode_job j;
+  std::memset(&j, 0, sizeof(j));
+  j.cfg = *cfg;
+  j.x = *x;
+  j.codes = out_codes;
+  j.norms = out_norms;
+  j.capacity = x->rows;
+  j.slot = nullptr;
+  return tac_encode_multi(&j, 1, stream);
+}
+
+int tac_decode(const void* codes, const void* norms, const tac_layer_cfg* cfg, tac_rows* y,
+               tac_stream_t stream) {
+  if (!y) return fail(TAC_E_INVAL, "tac_decode: y is NULL");
+  if (!cfg) return fail(TAC_E_INVAL, "tac_decode: cfg is NULL");
+  tac_decode_job j;
+  std::memset(&j, 0, sizeof(j));
+  j.cfg = *cfg;
+  j.codes = codes;
+  j.norms = norms;
+  j.capacity = y->rows;
+  j.slot = nullptr;
+  j.y = *y;
+  return tac_decode_multi(&j, 1, stream);
+}
+
+int tac_fwht_debug(const tac_rows* x, int d, const uint32_t* signs, float* y, tac_stream_t stream) {
+  static const char* who = "tac_fwht_debug";
+  if (d < 2 || d > 128 || (d & (d - 1))) return fail(TAC_E_INVAL, "%s: d = %d (powers of two 2..128)", who, d);
+  if (!signs) return fail(TAC_E_INVAL, "%s: signs is NULL", who);
+  int rc = check_rows(x, d, who, "x");
+  if (rc) return rc;
+  if (x->rows == 0) return ok();
+  if (!y || !aligned16(y)) return fail(TAC_E_INVAL, "%s: y is NULL or misaligned", who);
+  if (num_sms() <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
+  uint32_t s[4] = {0, 0, 0, 0};
+  for (int q = 0; q < (d + 31) / 32; ++q) s[q] = signs[q];
+  if (d < 32) s[0] &= (1u << d) - 1u;
+  cudaError_t e = tac::launch_fwht_debug(d, x->data, x->dtype, x->rows, x->row_stride, s, y,
+                                         reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+  return ok();
+}
+
+}  // extern "C"

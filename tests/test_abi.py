@@ -1,0 +1,155 @@
+"""Host-side checks of libtac's C ABI (no GPU needed): the library loads, exports
+every entry point include/tac.h declares, validates arguments before touching
+the device, and its host functions (signs, plane geometry, rates) agree with the
+oracle's independent implementations and the paper's printed rates."""
+import ctypes
+import math
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared_symbols():
+    src = open(os.path.join(ROOT, "include", "tac.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(tac_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_path(tac_host):
+    syms = _declared_symbols()
+    for name in ("tac_make_signs", "tac_encode", "tac_decode", "tac_encode_multi", "tac_decode_multi",
+                 "tac_fwht_debug", "tac_last_error"):
+        assert name in syms
+
+
+def test_library_exports_every_declared_symbol(tac_host):
+    lib = ctypes.CDLL(tac_host.library_path())
+    missing = [s for s in _declared_symbols() if not hasattr(lib, s)]
+    assert not missing, missing
+
+
+def test_version(tac_host):
+    assert "libtac" in tac_host.version()
+
+
+@pytest.mark.parametrize("seed,layer,kv,d,shared", [(0, 0, 0, 128, False), (0, 31, 1, 128, False),
+                                                    (12345, 7, 0, 64, False), (2**63 + 5, 3, 1, 16, False),
+                                                    (9, 4, 1, 128, True)])
+def test_signs_match_oracle(tac_host, orc, seed, layer, kv, d, shared):
+    words = tac_host.make_signs(seed, layer, kv, d, shared)
+    bits = np.array([(int(words[j // 32]) >> (j % 32)) & 1 for j in range(d)])
+    want = orc.signs(seed, layer, kv, d, shared=shared)
+    assert np.array_equal(np.where(bits == 1, -1, 1).astype(np.int8), want)
+
+
+def test_plane_geometry(tac_host):
+    for d in (16, 32, 64, 128):
+        for n in (2, 4, 16, 64, 128, 256):
+            for b, mode in ((8, 0), (4, 1)):
+                cfg = tac_host.LayerCfg(d, n, b, mode)
+                w = int(math.log2(n))
+                assert tac_host.angle_row_bytes(cfg) == d // 2 * w // 8
+                assert tac_host.norm_row_bytes(cfg) == d // 2 * b // 8
+                for cap in (0, 1, 7, 128, 1000):
+                    off = tac_host.header_offset(cfg, cap)
+                    assert off % 16 == 0 and off >= cap * (d // 2 * b // 8) and off - cap * d // 2 * b // 8 < 16
+                    assert tac_host.norms_bytes(cfg, cap) == off + 8 * cap
+                    assert tac_host.codes_bytes(cfg, cap) == cap * (d // 2 * w // 8)
+
+
+def test_record_bytes_match_rate_accounting(tac_host, orc):
+    # Eq. 3 total bits per element x d / 8 = record bytes per row (angle + norm + 8-byte header)
+    for n in (16, 64, 256):
+        for b in (4, 8):
+            cfg = tac_host.LayerCfg(128, n, b, 0)
+            rec = tac_host.angle_row_bytes(cfg) + tac_host.norm_row_bytes(cfg) + 8
+            assert rec * 8 / 128 == orc.total_bits(math.log2(n) / 2, b, 128)
+
+
+def test_rates_agree_with_oracle(tac_host, orc):
+    rng = np.random.default_rng(0)
+    for _ in range(20):
+        L = int(rng.integers(1, 48))
+        nk = [int(2 ** rng.integers(1, 9)) for _ in range(L)]
+        nv = [int(2 ** rng.integers(1, 9)) for _ in range(L)]
+        assert abs(tac_host.avg_angle_bits(nk, nv) - orc.avg_angle_bits(nk, nv)) < 1e-12
+    assert tac_host.total_bits(3.25, 6, 128) == 6.75
+
+
+def test_early_boost_schedule(tac_host):
+    nk, nv = tac_host.early_boost(32, 4, (256, 128), (128, 64))
+    assert abs(tac_host.avg_angle_bits(nk, nv) - 3.3125) < 1e-12
+    r = tac_host.rates(128, *tac_host.early_boost(32, 4, (256, 256), (64, 64)))
+    # Mistral-7B-shaped config: (4 * 4 + 28 * 3) / 32 = 3.125 angle bits; + 3 norm + 0.5 header
+    assert abs(r["angle_bits"] - 3.125) < 1e-12 and abs(r["total_bits"] - 6.625) < 1e-12
+
+
+def _cfg(tac, d=128, n=64, b=8, mode=0):
+    return tac.LayerCfg(d, n, b, mode).to_c()
+
+
+def test_invalid_arguments_rejected_before_launch(tac_host):
+    lib = tac_host.load()
+    rows = tac_host._Rows()
+    rows.data, rows.dtype, rows.rows, rows.row_stride = 16, 0, 4, 128
+    buf = 4096
+    cases = [
+        (dict(d=100), tac_host.TAC_E_INVAL),
+        (dict(d=256), tac_host.TAC_E_UNSUPPORTED),
+        (dict(n=3), tac_host.TAC_E_UNSUPPORTED),
+        (dict(n=0), tac_host.TAC_E_INVAL),
+        (dict(n=512), tac_host.TAC_E_UNSUPPORTED),
+        (dict(b=5), tac_host.TAC_E_UNSUPPORTED),
+        (dict(b=0), tac_host.TAC_E_INVAL),
+        (dict(mode=7), tac_host.TAC_E_INVAL),
+    ]
+    for kw, want in cases:
+        c = _cfg(tac_host, **kw)
+        assert lib.tac_encode(ctypes.byref(rows), ctypes.byref(c), buf, buf, None) == want, kw
+        assert tac_host.last_error()
+    c = _cfg(tac_host)
+    bad = tac_host._Rows()
+    for field, val in (("dtype", 9), ("rows", -1), ("row_stride", 64), ("data", 8), ("data", 0)):
+        bad.data, bad.dtype, bad.rows, bad.row_stride = 16, 0, 4, 128
+        setattr(bad, field, val)
+        assert lib.tac_encode(ctypes.byref(bad), ctypes.byref(c), buf, buf, None) == tac_host.TAC_E_INVAL, field
+    # stride * sizeof(bf16) not a multiple of 16
+    bad.data, bad.dtype, bad.rows, bad.row_stride = 16, 0, 4, 132
+    assert lib.tac_encode(ctypes.byref(bad), ctypes.byref(c), buf, buf, None) == tac_host.TAC_E_INVAL
+    # misaligned planes
+    assert lib.tac_encode(ctypes.byref(rows), ctypes.byref(c), buf + 8, buf, None) == tac_host.TAC_E_INVAL
+    assert lib.tac_encode(ctypes.byref(rows), ctypes.byref(c), None, buf, None) == tac_host.TAC_E_INVAL
+    # decode side
+    assert lib.tac_decode(buf, buf, ctypes.byref(_cfg(tac_host, n=3)), ctypes.byref(rows), None) == tac_host.TAC_E_UNSUPPORTED
+    # batched: negative count, NULL jobs, capacity too small without slots
+    assert lib.tac_encode_multi(None, -1, None) == tac_host.TAC_E_INVAL
+    assert lib.tac_encode_multi(None, 2, None) == tac_host.TAC_E_INVAL
+    jobs = (tac_host._EncJob * 1)()
+    jobs[0].cfg = c
+    jobs[0].x = rows
+    jobs[0].codes, jobs[0].norms, jobs[0].capacity, jobs[0].slot = buf, buf, 3, None
+    assert lib.tac_encode_multi(jobs, 1, None) == tac_host.TAC_E_INVAL
+    jobs[0].capacity, jobs[0].slot = 10, buf + 4  # misaligned slot array
+    assert lib.tac_encode_multi(jobs, 1, None) == tac_host.TAC_E_INVAL
+    # debug transform
+    s = (ctypes.c_uint32 * 4)()
+    assert lib.tac_fwht_debug(ctypes.byref(rows), 3, s, buf, None) == tac_host.TAC_E_INVAL
+    assert lib.tac_fwht_debug(ctypes.byref(rows), 256, s, buf, None) == tac_host.TAC_E_INVAL
+    # signs
+    assert lib.tac_make_signs(0, 0, 2, 0, 64, s) == tac_host.TAC_E_INVAL
+    assert lib.tac_make_signs(0, -1, 0, 0, 64, s) == tac_host.TAC_E_INVAL
+
+
+def test_empty_calls_succeed_without_device(tac_host):
+    lib = tac_host.load()
+    rows = tac_host._Rows()
+    rows.data, rows.dtype, rows.rows, rows.row_stride = 0, 0, 0, 128
+    c = _cfg(tac_host)
+    assert lib.tac_encode(ctypes.byref(rows), ctypes.byref(c), None, None, None) == tac_host.TAC_OK
+    assert lib.tac_decode(None, None, ctypes.byref(c), ctypes.byref(rows), None) == tac_host.TAC_OK
+    assert lib.tac_encode_multi(None, 0, None) == tac_host.TAC_OK
+    assert lib.tac_decode_multi(None, 0, None) == tac_host.TAC_OK

@@ -1,0 +1,175 @@
+"""CUDA encode/decode vs the CPU oracle, element by element (GB300)."""
+import math
+
+import numpy as np
+import pytest
+
+import parity
+import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def _oracle_cache(tac, orc, cfg, ref):
+    """A device cache holding the oracle's own records (for decode on identical codes)."""
+    torch = _torch()
+    rows = ref["k"].shape[0]
+    w = int(math.log2(cfg.n_angle))
+    cache = tac.Cache.empty(cfg, rows)
+    ang = orc.pack(ref["k"], w).reshape(-1)
+    nrm = orc.pack(ref["c"], cfg.norm_bits).reshape(-1)
+    off = tac.header_offset(cfg, rows)
+    nb = np.zeros(tac.norms_bytes(cfg, rows), dtype=np.uint8)
+    nb[: nrm.size] = nrm
+    nb[off: off + 8 * rows] = ref["hdr"].astype(np.float32).view(np.uint8).reshape(-1)
+    if ang.size:
+        cache.codes[: ang.size].copy_(torch.from_numpy(ang))
+    if nb.size:
+        cache.norms[: nb.size].copy_(torch.from_numpy(nb))
+    return cache
+
+
+def check_roundtrip(tac, orc, x, d, n, b, mode, seed=0, layer=0, kv=0, label="", decode_dtypes=("bf16", "fp32")):
+    torch = _torch()
+    rows = x.shape[0]
+    cfg = tac.layer_cfg(d, n, b, mode, seed, layer, kv)
+    cache = tac.encode(x, cfg)
+    torch.cuda.synchronize()
+    x64 = parity.to_f64(x)
+    s = orc.signs(seed, layer, kv, d)
+    assert np.array_equal(s, parity.signs_pm1(cfg.signs, d))
+    ref = orc.encode(x64, s, n, b, mode)
+    k, c, hdr = parity.gpu_codes(orc, cache, rows)
+    st = parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=label)
+    # decode on identical codes (the oracle's records) into bf16 and fp32
+    oc = _oracle_cache(tac, orc, cfg, ref)
+    v = orc.decode(ref["k"], ref["c"], ref["hdr"], s, n, b, mode)
+    for dt in decode_dtypes:
+        y = tac.decode(oc, cfg, dtype=torch.bfloat16 if dt == "bf16" else torch.float32)
+        torch.cuda.synchronize()
+        parity.compare_decode(parity.to_f64(y), v, dt, label=f"{label} decode {dt}")
+    # end to end: GPU encode -> GPU decode equals the oracle decode of the GPU's codes
+    y2 = tac.decode(cache, cfg, dtype=torch.float32)
+    torch.cuda.synchronize()
+    v2 = orc.decode(k, c, hdr, s, n, b, mode)
+    parity.compare_decode(parity.to_f64(y2), v2, "fp32", label=f"{label} e2e")
+    return st
+
+
+def _rows(w, rows, seed, dtype=None, layer=0, kv=0):
+    torch = _torch()
+    T = -(-rows // w.heads)
+    x = workloads.block(w, layer, kv, tokens=T, seed=seed, device="cuda", dtype=dtype)
+    return x[:rows].contiguous()
+
+
+def test_tiny_config_full(tac_gpu, orc):
+    """Config 1: K, V fp32 [8, 1024, 64], n = 64, K 8-bit linear, V 4-bit log, every row."""
+    w = workloads.CONFIGS["tiny"]
+    for kv in (workloads.K, workloads.V):
+        x = workloads.block(w, 0, kv, device="cuda")
+        d, n, b, mode = w.codebook(0, kv)
+        check_roundtrip(tac_gpu, orc, x, d, n, b, mode, layer=0, kv=kv, label=f"tiny kv={kv}")
+
+
+@pytest.mark.parametrize("n", [2, 4, 8, 16, 32, 64, 128, 256])
+@pytest.mark.parametrize("b,mode", [(8, 0), (4, 1)])
+def test_d128_bf16_every_codebook(tac_gpu, orc, n, b, mode):
+    w = workloads.CONFIGS["mistral7b"]
+    x = _rows(w, 1000, seed=n * 7 + b, layer=n % 32, kv=mode)  # 1000 rows: 7 full tiles + a ragged one
+    check_roundtrip(tac_gpu, orc, x, 128, n, b, mode, layer=n % 32, kv=mode, label=f"d128 n={n} b={b}")
+
+
+@pytest.mark.parametrize("d", [16, 32, 64])
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+@pytest.mark.parametrize("b,mode", [(8, 0), (4, 1), (8, 1), (4, 0)])
+def test_small_d_and_dtypes(tac_gpu, orc, d, dt, b, mode):
+    torch = _torch()
+    w = workloads.CONFIGS["llama1b"]
+    x = workloads.block(w, 1, 0, tokens=40, seed=d + b, device="cuda")[:, :d] if d <= 64 else None
+    x = x.to(torch.bfloat16 if dt == "bf16" else torch.float32).contiguous()
+    for n in (16, 256):
+        check_roundtrip(tac_gpu, orc, x, d, n, b, mode, seed=3, layer=2, kv=1, label=f"d{d} {dt} n{n}")
+
+
+def test_d128_fp32_input(tac_gpu, orc):
+    torch = _torch()
+    w = workloads.CONFIGS["mistral7b"]
+    x = _rows(w, 300, seed=5, dtype=torch.float32)
+    check_roundtrip(tac_gpu, orc, x, 128, 64, 8, 0, label="d128 fp32")
+
+
+@pytest.mark.parametrize("rows", [0, 1, 31, 127, 128, 129, 255, 257])
+def test_ragged_row_counts(tac_gpu, orc, rows):
+    w = workloads.CONFIGS["mistral7b"]
+    torch = _torch()
+    if rows == 0:
+        cfg = tac_gpu.layer_cfg(128, 64, 8, 0)
+        x = torch.empty((0, 128), dtype=torch.bfloat16, device="cuda")
+        cache = tac_gpu.encode(x, cfg)
+        y = tac_gpu.decode(cache, cfg, rows=0)
+        assert y.shape == (0, 128)
+        return
+    x = _rows(w, rows, seed=rows)
+    check_roundtrip(tac_gpu, orc, x, 128, 256, 8, 0, label=f"rows={rows}")
+    check_roundtrip(tac_gpu, orc, x, 128, 64, 4, 1, kv=1, label=f"rows={rows} V")
+
+
+def test_strided_rows(tac_gpu, orc):
+    """Rows that are not contiguous (row_stride > d), e.g. one head of a [T, H, d] cache."""
+    torch = _torch()
+    w = workloads.CONFIGS["mistral7b"]
+    big = _rows(w, 600, seed=9).reshape(200, 3, 128)
+    x = big[:, 1, :]
+    assert x.stride(0) == 384
+    check_roundtrip(tac_gpu, orc, x, 128, 64, 8, 0, label="strided")
+
+
+def test_degenerate_rows(tac_gpu, orc):
+    """Zero rows, constant rows, one-hot rows, huge and tiny magnitudes."""
+    torch = _torch()
+    d = 128
+    rng = np.random.default_rng(0)
+    rows = [np.zeros(d), np.ones(d), np.full(d, -3.0)]
+    for j in (0, 1, 64, 127):
+        e = np.zeros(d); e[j] = 2.5
+        rows.append(e)
+    rows.append(rng.standard_normal(d) * 2.0**50)
+    rows.append(rng.standard_normal(d) * 2.0**-60)
+    a = np.zeros(d); a[::2] = 1.0          # only even elements
+    rows.append(a)
+    a = np.zeros(d); a[1::2] = -1.0        # only odd elements
+    rows.append(a)
+    x = torch.tensor(np.array(rows), dtype=torch.float32).to(torch.bfloat16).cuda()
+    for n, b, mode in ((64, 8, 0), (64, 4, 1), (4, 8, 0), (2, 4, 1), (256, 8, 1)):
+        check_roundtrip(tac_gpu, orc, x, d, n, b, mode, label=f"degenerate n={n} b={b} m={mode}")
+
+
+def test_exact_bin_centres_and_ties(tac_gpu, orc):
+    """Pairs built on bin centres (robust codes) and on the n = 4 edges at pi/4
+    multiples where the oracle's rounding is exact (ties round up)."""
+    torch = _torch()
+    d = 64
+    s = orc.signs(0, 0, 0, d)
+    y = np.zeros((4, d))
+    y[0, 0::2], y[0, 1::2] = 1.0, 1.0        # theta = pi/4: n = 4 edge, tie -> k = 1
+    y[1, 0::2], y[1, 1::2] = 2.0, 0.0        # theta = 0
+    y[2, 0::2], y[2, 1::2] = 0.0, 3.0        # theta = pi/2
+    y[3, 0::2], y[3, 1::2] = -1.0, 0.0       # theta = pi
+    x = orc.transform(y, np.ones(d, dtype=np.int8)) * s   # x = D H y, exact (1/sqrt(64) = 1/8)
+    xt = torch.tensor(x, dtype=torch.float32).to(torch.bfloat16).cuda()
+    assert np.array_equal(parity.to_f64(xt), x)
+    for n in (4, 8, 64, 256):
+        cfg = tac_gpu.layer_cfg(d, n, 8, 0, 0, 0, 0)
+        cache = tac_gpu.encode(xt, cfg)
+        torch.cuda.synchronize()
+        k, c, hdr = parity.gpu_codes(orc, cache, 4)
+        want = orc.encode(x, s, n, 8, 0)["k"]
+        assert np.array_equal(k, want), (n, k[:, :3], want[:, :3])
+        if n == 4:
+            assert np.all(k[0] == 1) and np.all(k[1] == 0) and np.all(k[2] == 1) and np.all(k[3] == 2)
