@@ -269,6 +269,30 @@ def run_reference(args):
 
 
 # ---------------------------------------------------------------------------
+# multi-rank host logic (weak scaling: every rank runs an independent replica)
+# ---------------------------------------------------------------------------
+def rank_seed(rank: int) -> int:
+    """Each rank encodes/decodes its own cache (independent replica, its own inputs)."""
+    return rank
+
+
+def max_over_ranks(ms: float, world: int, device=None) -> float:
+    """Slowest rank's time: the job finishes when every replica has."""
+    if world <= 1:
+        return float(ms)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, bytes_per_rank_step: int, steps: int, total_ms: float) -> float:
+    """Whole-job GB/s: bytes every rank moved over the slowest rank's time."""
+    return world * bytes_per_rank_step * steps / (total_ms / 1e3) / 1e9
+
+
+# ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
 def main():
@@ -298,7 +322,7 @@ def main():
             dist.barrier()
         torch.cuda.synchronize()
 
-    ws = Workset(tac, args.config, seed=rank, device=dev)
+    ws = Workset(tac, args.config, seed=rank_seed(rank), device=dev)
     stream = torch.cuda.Stream(device=dev)
     enc_only = args.config == "append"
 
@@ -339,14 +363,11 @@ def main():
     total_ms = t_start.elapsed_time(t_end)
     enc_ms = [e[0].elapsed_time(e[1]) for e in ev]
     dec_ms = [e[1].elapsed_time(e[2]) for e in ev] if not enc_only else [0.0]
-    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, world, dev)
     launches_per_step = (1 if enc_only else 2) * (1 + (len(ws.enc_jobs) - 1) // 96)
 
     step_bytes = ws.enc_bytes + (0 if enc_only else ws.dec_bytes)
-    value = world * step_bytes * K / (total_ms / 1e3) / 1e9
+    value = job_throughput(world, step_bytes, K, total_ms)
     hbm, peak_kind = peaks()
     enc_avg = statistics.mean(enc_ms)
     dec_avg = statistics.mean(dec_ms)
@@ -377,11 +398,8 @@ def main():
                 hy.copy_(ws.y_all, non_blocking=True)
         e1.record(stream)
         barrier()
-        et = torch.tensor([e0.elapsed_time(e1)], dtype=torch.float64, device=dev)
-        if world > 1:
-            dist.all_reduce(et, op=dist.ReduceOp.MAX)
-        e2e_ms = float(et.item())
-        e2e = {"value": world * step_bytes * args.e2e_steps / (e2e_ms / 1e3) / 1e9, "unit": UNIT,
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+        e2e = {"value": job_throughput(world, step_bytes, args.e2e_steps, e2e_ms), "unit": UNIT,
                "h2d_bytes_per_step": hx.numel() * hx.element_size(),
                "d2h_bytes_per_step": hy.numel() * hy.element_size(),
                "ms_per_step": e2e_ms / args.e2e_steps}

@@ -85,12 +85,19 @@ void orc_hadamard(int d, double* H) {
       H[(size_t)a * d + j] = (popcount_u32((uint32_t)(a & j)) & 1) ? -scale : scale;
 }
 
-/* y = H D x for one vector (Alg. 1, first step), dense matrix-vector product. */
+/* y = H D x for one vector (Alg. 1, first step), dense matrix-vector product.
+ * H = (1/sqrt d) * (+-1 matrix) (Sec. 2): the +-1 sum is formed first and scaled
+ * once, so a coordinate that is exactly zero stays exactly zero (reading R3 then
+ * applies to exactly the pairs that are (0, 0)). */
 static void transform_one(const double* H, int d, const int8_t* s, const double* x, double* y) {
+  const double scale = 1.0 / sqrt((double)d);
   for (int a = 0; a < d; ++a) {
     double acc = 0.0;
-    for (int j = 0; j < d; ++j) acc += H[(size_t)a * d + j] * ((double)s[j] * x[j]);
-    y[a] = acc;
+    for (int j = 0; j < d; ++j) {
+      const double t = (double)s[j] * x[j];
+      acc += (H[(size_t)a * d + j] < 0.0) ? -t : t;
+    }
+    y[a] = acc * scale;
   }
 }
 
@@ -231,12 +238,14 @@ int orc_decode(const int32_t* k, const int32_t* c, const float* hdr, int64_t row
       yh[2 * i] = rh * cos(phi);
       yh[2 * i + 1] = rh * sin(phi);
     }
-    /* x^ = D H y^ : H is symmetric (Sec. 2), so row a of H is column a. */
+    /* x^ = D H y^ : H is symmetric (Sec. 2), so row a of H is column a; the
+     * +-1 sum is formed first and scaled by 1/sqrt(d) once. */
     double* out = y_out + row * d;
+    const double scale = 1.0 / sqrt((double)d);
     for (int j = 0; j < d; ++j) {
       double acc = 0.0;
-      for (int a = 0; a < d; ++a) acc += H[(size_t)j * d + a] * yh[a];
-      out[j] = (double)s[j] * acc;
+      for (int a = 0; a < d; ++a) acc += (H[(size_t)j * d + a] < 0.0) ? -yh[a] : yh[a];
+      out[j] = (double)s[j] * (acc * scale);
     }
   }
   free(H); free(yh);

@@ -119,7 +119,7 @@ int esize(int dtype) { return dtype == TAC_BF16 ? 2 : dtype == TAC_FP32 ? 4 : 0;
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
-int check_rows(const tac_rows* r, int d, const char* who, const char* name) {
+int check_rows(const tac_rows* r, int d, const char* who, const char* name, bool rows16 = true) {
   if (!r) return fail(TAC_E_INVAL, "%s: %s is NULL", who, name);
   if (!esize(r->dtype)) return fail(TAC_E_INVAL, "%s: %s.dtype = %d", who, name, r->dtype);
   if (r->rows < 0) return fail(TAC_E_INVAL, "%s: %s.rows = %lld", who, name, (long long)r->rows);
@@ -127,7 +127,7 @@ int check_rows(const tac_rows* r, int d, const char* who, const char* name) {
   if (!r->data) return fail(TAC_E_INVAL, "%s: %s.data is NULL", who, name);
   if (!aligned16(r->data)) return fail(TAC_E_INVAL, "%s: %s.data is not 16-byte aligned", who, name);
   if (r->row_stride < d) return fail(TAC_E_INVAL, "%s: %s.row_stride %lld < d %d", who, name, (long long)r->row_stride, d);
-  if ((r->row_stride * esize(r->dtype)) % 16)
+  if (rows16 && (r->row_stride * esize(r->dtype)) % 16)
     return fail(TAC_E_INVAL, "%s: %s.row_stride * sizeof(element) is not a multiple of 16", who, name);
   if (r->rows > ((int64_t)1 << 38)) return fail(TAC_E_UNSUPPORTED, "%s: %s.rows too large", who, name);
   return TAC_OK;
@@ -386,7 +386,7 @@ int tac_fwht_debug(const tac_rows* x, int d, const uint32_t* signs, float* y, ta
   static const char* who = "tac_fwht_debug";
   if (d < 2 || d > 128 || (d & (d - 1))) return fail(TAC_E_INVAL, "%s: d = %d (powers of two 2..128)", who, d);
   if (!signs) return fail(TAC_E_INVAL, "%s: signs is NULL", who);
-  int rc = check_rows(x, d, who, "x");
+  int rc = check_rows(x, d, who, "x", /*rows16=*/false);
   if (rc) return rc;
   if (x->rows == 0) return ok();
   if (!y || !aligned16(y)) return fail(TAC_E_INVAL, "%s: y is NULL or misaligned", who);

@@ -14,6 +14,12 @@ def _torch():
     return torch
 
 
+def _same_planes(a, b):
+    """Records equal plane by plane (bytes between the norm and header planes are padding)."""
+    for pa, pb in zip(a.planes(), b.planes()):
+        assert np.array_equal(pa.view(np.uint8), pb.view(np.uint8))
+
+
 def _jobs_spec():
     # (d, n, b, mode, dtype, rows, layer, kv)
     return [(128, 256, 8, 0, "bf16", 700, 0, 0), (128, 64, 4, 1, "bf16", 300, 0, 1),
@@ -43,8 +49,7 @@ def test_encode_multi_equals_single_calls(tac_gpu, orc):
     tac.encode_multi(jobs)
     torch.cuda.synchronize()
     for j, s in zip(jobs, singles):
-        assert torch.equal(j.cache.codes, s.codes)
-        assert torch.equal(j.cache.norms, s.norms)
+        _same_planes(j.cache, s)
     # and the batched output is oracle-exact too (codes and headers)
     j = jobs[0]
     x64 = parity.to_f64(j.x)
@@ -135,4 +140,4 @@ def test_many_jobs_split_across_launches(tac_gpu):
     tac.encode_multi(jobs)
     torch.cuda.synchronize()
     for j, r in zip(jobs, refs):
-        assert torch.equal(j.cache.codes, r.codes) and torch.equal(j.cache.norms, r.norms)
+        _same_planes(j.cache, r)
