@@ -44,6 +44,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="override tokens per (layer, K/V) block (smaller cases for profiling)")
     ap.add_argument("--cpu-rows", type=int, default=400_000,
                     help="rows in the bounded oracle sample (CPU baseline / reference arm)")
     return ap.parse_args()
@@ -142,7 +144,7 @@ def config_desc(name):
 class Workset:
     """Device-resident cache, records and decode output of one rank, plus byte accounting."""
 
-    def __init__(self, tac, name, seed, device):
+    def __init__(self, tac, name, seed, device, tokens=0):
         import torch
         self.name = name
         self.enc_jobs, self.dec_jobs = [], []
@@ -169,6 +171,9 @@ class Workset:
             self.y_all = None
             return
         w = workloads.CONFIGS[name]
+        if tokens:
+            import dataclasses
+            w = dataclasses.replace(w, tokens=tokens)
         blocks = w.blocks()
         R = w.rows_per_block
         self.x_all = torch.empty((len(blocks), R, w.d), dtype=torch.bfloat16, device=device)
@@ -322,7 +327,7 @@ def main():
             dist.barrier()
         torch.cuda.synchronize()
 
-    ws = Workset(tac, args.config, seed=rank_seed(rank), device=dev)
+    ws = Workset(tac, args.config, seed=rank_seed(rank), device=dev, tokens=args.tokens)
     stream = torch.cuda.Stream(device=dev)
     enc_only = args.config == "append"
 
@@ -415,7 +420,8 @@ def main():
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
             "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": config_desc(args.config), "io_dtype": "bf16",
+            "config": {"workload": config_desc(args.config) + (f" (tokens overridden: {args.tokens})" if args.tokens else ""),
+                       "io_dtype": "bf16",
                        "bytes_per_step_per_gpu": step_bytes,
                        "l2": "inputs larger than L2 (no flush needed): "
                              f"{ws.x_all.numel() * 2 / 1e9:.2f} GB of bf16 rows per step",

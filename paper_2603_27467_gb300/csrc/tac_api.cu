@@ -115,6 +115,9 @@ int64_t angle_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * l
 int64_t norm_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * c->norm_bits / 8; }
 int64_t header_offset(const tac_layer_cfg* c, int64_t cap) { return (cap * norm_row_bytes(c) + 15) & ~(int64_t)15; }
 
+// Rows per kernel tile: 256 threads, d/16 lanes per row (8 angle pairs per lane).
+int64_t tile_rows(int d) { return (int64_t)tac::kThreads / (d / 16); }
+
 int esize(int dtype) { return dtype == TAC_BF16 ? 2 : dtype == TAC_FP32 ? 4 : 0; }
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -259,7 +262,8 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
     int64_t tiles = 0;
     while (i < live.size() && P.njobs < TAC_MAX_JOBS && jobs[live[i]].cfg.d == d && jobs[live[i]].x.dtype == dt) {
       const tac_encode_job& J = jobs[live[i]];
-      const int64_t jt = (J.x.rows + tac::kTileRows - 1) / tac::kTileRows;
+      const int64_t tr = tile_rows(d);
+      const int64_t jt = (J.x.rows + tr - 1) / tr;
       if (tiles + jt > 0x7fffffff) break;
       tac::EncJob& E = P.job[P.njobs];
       E.x = J.x.data;
@@ -324,7 +328,8 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
     int64_t tiles = 0;
     while (i < live.size() && P.njobs < TAC_MAX_JOBS && jobs[live[i]].cfg.d == d && jobs[live[i]].y.dtype == dt) {
       const tac_decode_job& J = jobs[live[i]];
-      const int64_t jt = (J.y.rows + tac::kTileRows - 1) / tac::kTileRows;
+      const int64_t tr = tile_rows(d);
+      const int64_t jt = (J.y.rows + tr - 1) / tr;
       if (tiles + jt > 0x7fffffff) break;
       tac::DecJob& E = P.job[P.njobs];
       E.codes = static_cast<const uint8_t*>(J.codes);

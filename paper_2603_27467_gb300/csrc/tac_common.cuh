@@ -9,14 +9,47 @@
 
 namespace tac {
 
-constexpr int kTileRows = 128;     // rows per tile: one thread per row
-constexpr int kThreads = 128;      // threads per CTA
+constexpr int kThreads = 256;      // threads per CTA
+constexpr int kPairsPerThread = 8; // each thread owns 8 consecutive angle pairs (16 elements)
 constexpr int kMaxW = 8;           // log2 n <= 8 (n <= 256)
 constexpr int kTabEntries = 512;   // sum_{w=1..8} 2^w = 510, padded
 constexpr float kU = 5.9604644775390625e-08f;  // fp32 unit roundoff 2^-24
 
 // Offset of the table for n = 2^w inside a table holding every w = 1..8 back to back.
 __host__ __device__ constexpr int tab_offset(int w) { return (1 << w) - 2; }
+
+// ---------------------------------------------------------------------------
+// Tile geometry for head dimension D: P = D/2 pairs per row, L = P/8 lanes per
+// row (each lane owns 8 pairs), TR = 256/L rows per tile.
+// ---------------------------------------------------------------------------
+template <int D>
+struct Geo {
+  static constexpr int P = D / 2;
+  static constexpr int L = P / kPairsPerThread;
+  static constexpr int TR = kThreads / L;
+  static constexpr int LOGD = (D == 16) ? 4 : (D == 32) ? 5 : (D == 64) ? 6 : 7;
+  // Transpose buffer: one row of P float2 pairs, padded so that the phase-A
+  // pattern (lane l writes pairs l + L*m) and the phase-B pattern (lane l reads
+  // pairs 8l..8l+7 as four 16-byte granules) are both bank-conflict free.
+  static constexpr int ST = 8 * P + 32;
+  static constexpr int TP_B = TR * ST;
+  __device__ static __forceinline__ int tp(int r, int i) {
+    const int g = i >> 1;
+    return r * ST + ((g ^ ((g >> 2) & 7)) << 4) + ((i & 1) << 3);
+  }
+};
+
+// Row-major element tile with a per-row pad chosen so that lane l of a row
+// accessing pair l + L*m (element bytes [2i*ESZ, 2i*ESZ + 2*ESZ)) hits distinct
+// banks across the rows of a warp; rows start on 16-byte boundaries.
+template <int D, int ESZ>
+struct RowTile {
+  static constexpr int ROWB = D * ESZ;
+  static constexpr int CPR = ROWB / 16;
+  static constexpr int SPAN = 2 * ESZ * Geo<D>::L;
+  static constexpr int STRIDE = ROWB + (SPAN > 16 ? SPAN : 16);
+  static constexpr int BYTES = Geo<D>::TR * STRIDE;
+};
 
 // ---------------------------------------------------------------------------
 // Device job descriptors (kernel parameters, copied by value at launch).
@@ -76,6 +109,16 @@ __device__ __forceinline__ int find_job(const Params& p, int t) {
   return lo;
 }
 
+// XOR masks flipping the IEEE sign bits of elements 2i and 2i+1 where s_j = -1
+// (D of Sec. 2).  bf16 pairs share one 32-bit word (bits 15 and 31); fp32 pairs
+// use one word each.
+template <int ESZ>
+__device__ __forceinline__ uint2 pair_sign_mask(const uint32_t* signs, int i) {
+  const uint32_t two = (signs[(2 * i) >> 5] >> ((2 * i) & 31)) & 3u;
+  if constexpr (ESZ == 2) return make_uint2(((two & 1u) << 15) | ((two >> 1) << 31), 0u);
+  else return make_uint2((two & 1u) << 31, (two >> 1) << 31);
+}
+
 // ---------------------------------------------------------------------------
 // Exact-symmetry trig tables.  Every table entry is (cos, sin) of 2 pi Q / (8 n)
 // for an integer Q: the angle is reduced to an octant with integer arithmetic
@@ -102,8 +145,7 @@ __device__ __forceinline__ float2 cos_sin_q8(int Q, int n) {
     else sincospif((float)rr / (float)(4 * n), &s, &c);
     s = -s;                  // (cos(-b'), sin(-b'))
   }
-  // rotate (c, s) by quarter * pi/2
-  switch (quarter & 3) {
+  switch (quarter & 3) {     // rotate (c, s) by quarter * pi/2
     case 0: return make_float2(c, s);
     case 1: return make_float2(-s, c);
     case 2: return make_float2(-c, -s);
@@ -111,33 +153,60 @@ __device__ __forceinline__ float2 cos_sin_q8(int Q, int n) {
   }
 }
 
-// Same construction in fp64 for the exact-decision path.
-__device__ __forceinline__ double2 cos_sin_q8_d(int Q, int n) {
+// ---------------------------------------------------------------------------
+// fp64 edge directions for the exact-decision path, built by the host compiler:
+// cos/sin from their Taylor series on [0, pi/4] (|x| <= 0.79: 24 terms reach
+// full double precision) with the same integer octant reduction as above.
+// ---------------------------------------------------------------------------
+namespace cx {
+struct CS { double c, s; };
+constexpr double kPi = 3.141592653589793238462643383279502884;
+constexpr double sin_series(double x) {
+  double term = x, sum = x;
+  for (int k = 1; k < 24; ++k) { term *= -x * x / ((2.0 * k) * (2.0 * k + 1.0)); sum += term; }
+  return sum;
+}
+constexpr double cos_series(double x) {
+  double term = 1.0, sum = 1.0;
+  for (int k = 1; k < 24; ++k) { term *= -x * x / ((2.0 * k - 1.0) * (2.0 * k)); sum += term; }
+  return sum;
+}
+constexpr CS cos_sin_q8(int Q, int n) {
   const int N8 = 8 * n;
   Q %= N8;
   if (Q < 0) Q += N8;
-  const int o = Q / n;
-  const int rem = Q - o * n;
-  double c, s;
-  int quarter;
+  const int o = Q / n, rem = Q - o * n;
+  double c = 1.0, s = 0.0;
+  int quarter = 0;
   if ((o & 1) == 0) {
     quarter = o >> 1;
-    if (rem == 0) { s = 0.0; c = 1.0; }
-    else sincospi((double)rem / (double)(4 * n), &s, &c);
+    if (rem != 0) { const double a = kPi * rem / (4.0 * n); c = cos_series(a); s = sin_series(a); }
   } else {
     quarter = (o + 1) >> 1;
     const int rr = n - rem;
-    if (rr == n) { s = 0.70710678118654752440; c = 0.70710678118654752440; }
-    else sincospi((double)rr / (double)(4 * n), &s, &c);
+    if (rr == n) { c = 0.70710678118654752440; s = 0.70710678118654752440; }
+    else { const double a = kPi * rr / (4.0 * n); c = cos_series(a); s = sin_series(a); }
     s = -s;
   }
   switch (quarter & 3) {
-    case 0: return make_double2(c, s);
-    case 1: return make_double2(-s, c);
-    case 2: return make_double2(-c, -s);
-    default: return make_double2(s, -c);
+    case 0: return CS{c, s};
+    case 1: return CS{-s, c};
+    case 2: return CS{-c, -s};
+    default: return CS{s, -c};
   }
 }
+struct EdgeTable { CS v[kTabEntries]; };
+constexpr EdgeTable make_edge_table() {
+  EdgeTable t{};
+  for (int idx = 0; idx < kTabEntries - 2; ++idx) {
+    int w = 1;
+    while ((1 << (w + 1)) - 2 <= idx) ++w;
+    const int n = 1 << w, e = idx - ((1 << w) - 2);
+    t.v[idx] = cos_sin_q8(8 * e + 4 + n, n);
+  }
+  return t;
+}
+}  // namespace cx
 
 // Encode edge table for n = 2^w, entry e: direction psi_e = phi_e + pi/4 of the
 // edge phi_e = (e + 1/2) 2 pi / n between bins e and e+1, as (cos psi, sin psi).
@@ -148,20 +217,6 @@ __device__ __forceinline__ int edge_q8(int e, int n) { return 8 * e + 4 + n; }
 // Decode table for n = 2^w, entry k: (cos phi_k + sin phi_k, cos phi_k - sin phi_k)
 // = sqrt2 (sin(phi_k + pi/4), cos(phi_k + pi/4)), phi_k = 2 pi k / n (Sec. 3.1).
 __device__ __forceinline__ int centre_q8(int k, int n) { return 8 * k + n; }
-
-// ---------------------------------------------------------------------------
-// Shared-memory tile swizzle: the 16-byte chunk c of tile row r is stored at
-// chunk c ^ sw(r) of that row, so that one thread per row reading chunk c hits
-// eight distinct 16-byte bank groups per eight consecutive rows.
-// ---------------------------------------------------------------------------
-template <int ROWB>
-__device__ __forceinline__ int row_swz(int r) {
-  constexpr int CPR = ROWB / 16;
-  if constexpr (ROWB >= 128) return r & 7;
-  else if constexpr (ROWB == 64) return (r >> 1) & (CPR - 1);
-  else if constexpr (ROWB == 32) return (r >> 2) & (CPR - 1);
-  else return 0;
-}
 
 // ---------------------------------------------------------------------------
 // cp.async (sm_80+ async global -> shared copies, 16 bytes, zero-fill tail).
@@ -185,8 +240,45 @@ __device__ __forceinline__ float2 sub2(float2 a, float2 b) {
 }
 __device__ __forceinline__ float2 mul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
 
+// In-register butterfly over the 8 values of v: the stages on index bits with
+// HLO <= 2^bit < HHI (<1, 8>: all three).
+template <int HHI = 8, int HLO = 1>
+__device__ __forceinline__ void butterfly8(float2 (&v)[8]) {
+#pragma unroll
+  for (int h = HLO; h < HHI; h <<= 1) {
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+      if ((m & h) == 0) {
+        const float2 a = v[m], b = v[m + h];
+        v[m] = add2(a, b);
+        v[m + h] = sub2(a, b);
+      }
+    }
+  }
+}
+
 // bf16 <-> fp32 (exact widening; bf16 is the high half of an fp32).
 __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// Hardware approximations (MUFU): relative error of a few fp32 ulp.
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float r; asm("sqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x)); return r;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r; asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x)); return r;
+}
+__device__ __forceinline__ float lg2_approx(float x) {
+  float r; asm("lg2.approx.f32 %0, %1;" : "=f"(r) : "f"(x)); return r;
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float r; asm("ex2.approx.f32 %0, %1;" : "=f"(r) : "f"(x)); return r;
+}
+__device__ __forceinline__ float min3(float a, float b, float c) {
+  float r; asm("min.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c)); return r;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float r; asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c)); return r;
+}
 
 }  // namespace tac

@@ -1,40 +1,49 @@
 // TurboAngle decode kernel for sm_103a (Sec. 3.1 reconstruction with the Eq. 2
 // dequantization of arXiv 2603.27467).
 //
-// One thread owns one row of a 128-row tile:
+// A 256-thread CTA decodes a tile of TR = 256/L rows, L = d/16 lanes per row,
+// 8 angle pairs per lane:
 //   1. the tile's records (angle / norm / header planes) are staged global ->
 //      shared with cp.async: coalesced 16-byte chunks for contiguous slots,
 //      per-row copies for gathered slots; double buffered;
-//   2. each pair is rebuilt from its bin-centre angle by table lookup: the table
-//      holds (cos phi_k + sin phi_k, cos phi_k - sin phi_k) / sqrt(d), i.e. the
+//   2. lane l unpacks its 8 consecutive codes (pairs 8l..8l+7) and rebuilds each
+//      pair from its bin-centre angle by table lookup: the table holds
+//      (cos phi_k + sin phi_k, cos phi_k - sin phi_k) / sqrt(d), i.e. the
 //      element-pair butterfly stage and the 1/sqrt(d) normalization are folded
-//      into the lookup, so the remaining log2(d) - 1 butterfly stages run on
-//      packed fp32 pairs (FADD2/FFMA2) straight from (E_i, O_i) = r^_i * T[k_i];
-//   3. D is applied as a sign XOR on the output bits (after bf16 RNE rounding,
-//      or on fp32), rows are staged swizzled and written with coalesced stores.
+//      into the lookup, so the remaining butterfly stages run straight from
+//      (E_i, O_i) = r^_i * T[k_i] on packed fp32 pairs (FADD2/FFMA2): the low
+//      pair-index bits in registers, an intra-warp shared-memory transpose, the
+//      high bits;
+//   3. D is a sign XOR on the output bits (after bf16 round-to-nearest-even, or
+//      on fp32); rows are staged in shared memory and written with coalesced
+//      16-byte stores.
 #include "tac_common.cuh"
 
 namespace tac {
 
+constexpr int kStages = 4;  // record tiles per CTA: 3 in flight while one is decoded
+
 template <int D, typename TOut>
 struct Dec {
-  static constexpr int P = D / 2;
+  using G = Geo<D>;
+  using OT = RowTile<D, (int)sizeof(TOut)>;
+  static constexpr int P = G::P, L = G::L, TR = G::TR;
   static constexpr int ESZ = (int)sizeof(TOut);
-  static constexpr int ROWB = D * ESZ;                 // output row bytes
-  static constexpr int CPR = ROWB / 16;
-  static constexpr int ABMAX = P;                      // angle record bytes at w = 8
-  static constexpr int NBMAX = P;                      // norm record bytes at b = 8
-  static constexpr int REC_B = kTileRows * (ABMAX + NBMAX + 8);  // one record buffer
+  static constexpr int ABMAX = P;                        // angle record bytes at w = 8
+  static constexpr int NBMAX = P;                        // norm record bytes at b = 8
+  static constexpr int R_ANG = 0;                        // inside a record buffer
+  static constexpr int R_NRM = TR * ABMAX;
+  static constexpr int R_HDR = R_NRM + TR * NBMAX;
+  static constexpr int REC_B = R_HDR + TR * 8 + 16;      // + slack for 3-word angle reads
   // shared memory layout (bytes)
-  static constexpr int OFF_REC = 0;                    // 2 record buffers
-  static constexpr int OFF_OUT = OFF_REC + 2 * REC_B;  // output tile
-  static constexpr int OFF_TAB = OFF_OUT + kTileRows * ROWB;
-  static constexpr int OFF_MSK = OFF_TAB + kTabEntries * 8;
-  static constexpr int SMEM = OFF_MSK + P * 8;
-  // inside a record buffer
-  static constexpr int R_ANG = 0;
-  static constexpr int R_NRM = kTileRows * ABMAX;
-  static constexpr int R_HDR = R_NRM + kTileRows * NBMAX;
+  static constexpr int OFF_REC = 0;                      // kStages record buffers
+  static constexpr int OFF_TP = OFF_REC + kStages * REC_B; // transpose buffer
+  static constexpr int OFF_OUT = OFF_TP + G::TP_B;       // output tile
+  static constexpr int OFF_TAB = OFF_OUT + OT::BYTES;    // centre tables, every n
+  static constexpr int SMEM = OFF_TAB + kTabEntries * 8;
+  static constexpr int CHUNKS = TR * OT::CPR / kThreads;
+  static_assert(TR * OT::CPR % kThreads == 0, "tile chunks");
+  static_assert(REC_B % 16 == 0, "record buffer alignment");
 };
 
 // Cooperative cp.async of `bytes` contiguous bytes (16-byte aligned global base),
@@ -50,162 +59,127 @@ __device__ __forceinline__ void cta_copy_in(uint8_t* s, const uint8_t* g, int by
 template <int D, typename TOut>
 __device__ __forceinline__ void issue_rec_load(const DecJob& J, int row0, int nrows, uint8_t* buf, int tid) {
   using C = Dec<D, TOut>;
-  const int P = C::P;
-  const int AB = P * J.w / 8, NB = P * J.b / 8;
+  const int AB = C::P * J.w / 8, NB = C::P * J.b / 8;
   if (J.slot == nullptr) {
     cta_copy_in(buf + C::R_ANG, J.codes + (int64_t)row0 * AB, nrows * AB, tid);
     cta_copy_in(buf + C::R_NRM, J.norms + (int64_t)row0 * NB, nrows * NB, tid);
     cta_copy_in(buf + C::R_HDR, J.hdr + (int64_t)row0 * 8, nrows * 8, tid);
-  } else if (tid < nrows) {
-    // Gather: this thread's record, byte-exact, with plain loads (records of odd
-    // size are not 16-byte aligned in the source planes).
-    int64_t s = J.slot[row0 + tid];
-    uint8_t* da = buf + C::R_ANG + tid * AB;
-    uint8_t* dn = buf + C::R_NRM + tid * NB;
-    float2* dh = reinterpret_cast<float2*>(buf + C::R_HDR) + tid;
-    if (s < 0 || s >= J.capacity) {  // out-of-range slot: decodes as an all-zero record
-      for (int q = 0; q < AB; ++q) da[q] = 0;
-      for (int q = 0; q < NB; ++q) dn[q] = 0;
-      *dh = make_float2(0.f, 0.f);
-      return;
-    }
-    const uint8_t* sa = J.codes + s * AB;
-    const uint8_t* sn = J.norms + s * NB;
-    if ((AB & 3) == 0) {
-      for (int q = 0; q < AB / 4; ++q) reinterpret_cast<uint32_t*>(da)[q] = __ldg(reinterpret_cast<const uint32_t*>(sa) + q);
-    } else {
-      for (int q = 0; q < AB; ++q) da[q] = __ldg(sa + q);
-    }
-    if ((NB & 3) == 0) {
-      for (int q = 0; q < NB / 4; ++q) reinterpret_cast<uint32_t*>(dn)[q] = __ldg(reinterpret_cast<const uint32_t*>(sn) + q);
-    } else {
-      for (int q = 0; q < NB; ++q) dn[q] = __ldg(sn + q);
-    }
-    *dh = __ldg(reinterpret_cast<const float2*>(J.hdr) + s);
-  }
-}
-
-template <int D, typename TOut>
-__device__ __forceinline__ void build_dec_masks(const DecJob& J, uint2* msk, int tid) {
-  using C = Dec<D, TOut>;
-  for (int i = tid; i < C::P; i += kThreads) {
-    const uint32_t b0 = (J.signs[(2 * i) >> 5] >> ((2 * i) & 31)) & 1u;
-    const uint32_t b1 = (J.signs[(2 * i + 1) >> 5] >> ((2 * i + 1) & 31)) & 1u;
-    if constexpr (C::ESZ == 2) msk[i] = make_uint2((b0 << 15) | (b1 << 31), 0u);
-    else msk[i] = make_uint2(b0 << 31, b1 << 31);
-  }
-}
-
-// Read W bits at bit offset `bit` of a little-endian word array (compile-time offsets).
-template <int W>
-__device__ __forceinline__ uint32_t get_bits(const uint32_t* a, int bit) {
-  const int wi = bit >> 5, sh = bit & 31;
-  uint32_t v = a[wi] >> sh;
-  if (sh + W > 32) v |= a[wi + 1] << (32 - sh);
-  return v & ((1u << W) - 1u);
-}
-
-template <int BYTES, int NWORDS>
-__device__ __forceinline__ void load_record(uint32_t (&w)[NWORDS], const uint8_t* src) {
-  if constexpr (BYTES % 16 == 0) {
-#pragma unroll
-    for (int q = 0; q < BYTES / 16; ++q) {
-      const uint4 t = reinterpret_cast<const uint4*>(src)[q];
-      w[4 * q] = t.x; w[4 * q + 1] = t.y; w[4 * q + 2] = t.z; w[4 * q + 3] = t.w;
-    }
-  } else if constexpr (BYTES % 8 == 0) {
-#pragma unroll
-    for (int q = 0; q < BYTES / 8; ++q) {
-      const uint2 t = reinterpret_cast<const uint2*>(src)[q];
-      w[2 * q] = t.x; w[2 * q + 1] = t.y;
-    }
-  } else if constexpr (BYTES % 4 == 0) {
-#pragma unroll
-    for (int q = 0; q < BYTES / 4; ++q) w[q] = reinterpret_cast<const uint32_t*>(src)[q];
   } else {
-#pragma unroll
-    for (int q = 0; q < NWORDS; ++q) w[q] = 0u;
-#pragma unroll
-    for (int q = 0; q < BYTES; ++q) w[q >> 2] |= (uint32_t)src[q] << (8 * (q & 3));
+    // Gather: one thread per row copies its record byte-exactly with plain loads
+    // (records of odd size are not 16-byte aligned in the source planes).
+    for (int rr = tid; rr < nrows; rr += kThreads) {
+      const int64_t s = J.slot[row0 + rr];
+      uint8_t* da = buf + C::R_ANG + rr * AB;
+      uint8_t* dn = buf + C::R_NRM + rr * NB;
+      float2* dh = reinterpret_cast<float2*>(buf + C::R_HDR) + rr;
+      if (s < 0 || s >= J.capacity) {  // out-of-range slot: decodes as an all-zero record
+        for (int q = 0; q < AB; ++q) da[q] = 0;
+        for (int q = 0; q < NB; ++q) dn[q] = 0;
+        *dh = make_float2(0.f, 0.f);
+        continue;
+      }
+      const uint8_t* sa = J.codes + s * AB;
+      const uint8_t* sn = J.norms + s * NB;
+      if ((AB & 3) == 0) {
+        for (int q = 0; q < AB / 4; ++q) reinterpret_cast<uint32_t*>(da)[q] = __ldg(reinterpret_cast<const uint32_t*>(sa) + q);
+      } else {
+        for (int q = 0; q < AB; ++q) da[q] = __ldg(sa + q);
+      }
+      if ((NB & 3) == 0) {
+        for (int q = 0; q < NB / 4; ++q) reinterpret_cast<uint32_t*>(dn)[q] = __ldg(reinterpret_cast<const uint32_t*>(sn) + q);
+      } else {
+        for (int q = 0; q < NB; ++q) dn[q] = __ldg(sn + q);
+      }
+      *dh = __ldg(reinterpret_cast<const float2*>(J.hdr) + s);
+    }
+  }
+}
+
+// Read NBYTES (<= 8) bytes starting at shared byte address p (any alignment).
+template <int NBYTES>
+__device__ __forceinline__ uint64_t load_bytes(const uint8_t* p) {
+  if constexpr (NBYTES == 8) {
+    const uint2 t = *reinterpret_cast<const uint2*>(p);
+    return (uint64_t)t.x | ((uint64_t)t.y << 32);
+  } else if constexpr (NBYTES == 4) {
+    return *reinterpret_cast<const uint32_t*>(p);
+  } else {
+    const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+    const uint32_t* w = reinterpret_cast<const uint32_t*>(a & ~(uintptr_t)3);
+    const int sh = (int)(a & 3) * 8;
+    const uint64_t lo = (uint64_t)w[0] | ((uint64_t)w[1] << 32);
+    uint64_t v = lo >> sh;
+    if (sh) v |= (uint64_t)w[2] << (64 - sh);
+    return v;
   }
 }
 
 template <int D, typename TOut, int W, int B>
-__device__ __forceinline__ void decode_row(const DecJob& J, const uint8_t* rec, uint8_t* smem, int tid) {
+__device__ __forceinline__ void decode_row(const DecJob& J, const uint8_t* rec, uint8_t* smem, int tid,
+                                           const uint2 (&msk)[8]) {
   using C = Dec<D, TOut>;
-  constexpr int P = C::P;
+  using G = Geo<D>;
+  using OT = typename C::OT;
+  constexpr int P = C::P, L = C::L;
+  constexpr int n = 1 << W;
   constexpr int AB = P * W / 8;
   constexpr int NB = P * B / 8;
-  constexpr int AW = (P * W + 31) / 32;
-  constexpr int NW = (P * B + 31) / 32;
-  constexpr int L = (1 << B) - 1;
+  constexpr int Lq = (1 << B) - 1;
+  const int r = tid / L, l = tid % L;
   const float2* ttab = reinterpret_cast<const float2*>(smem + C::OFF_TAB) + tab_offset(W);
-  const uint2* msk = reinterpret_cast<const uint2*>(smem + C::OFF_MSK);
 
-  uint32_t aw[AW], nw[NW];
-  load_record<AB>(aw, rec + C::R_ANG + tid * AB);
-  load_record<NB>(nw, rec + C::R_NRM + tid * NB);
-  const float2 h = reinterpret_cast<const float2*>(rec + C::R_HDR)[tid];
+  const uint64_t acc_a = load_bytes<W>(rec + C::R_ANG + r * AB + l * W);
+  const uint64_t acc_n = load_bytes<B>(rec + C::R_NRM + r * NB + l * B);
+  const float2 h = reinterpret_cast<const float2*>(rec + C::R_HDR)[r];
   const float hmin = h.x, hmax = h.y;
 
-  // Dequantization (reading of Eq. 2's inverse): linear r^ = r_min + c (r_max - r_min)/L,
+  // Dequantization (the inverse of Eq. 2): linear r^ = r_min + c (r_max - r_min)/L,
   // log r^ = 2^(l_min + c (l_max - l_min)/L); r_max == r_min gives r^ = r_min.
-  const bool flat = !(hmax != hmin);
+  const bool spread = hmax > hmin;
   float base, step;
   if (J.mode == TAC_NORM_LINEAR) {
     base = hmin;
-    step = __fdiv_rn(__fsub_rn(hmax, hmin), (float)L);
+    step = spread ? (hmax - hmin) * (1.0f / (float)Lq) : 0.f;
   } else {
-    base = flat ? 0.f : log2f(hmin);
-    step = flat ? 0.f : __fdiv_rn(__fsub_rn(log2f(hmax), base), (float)L);
+    base = lg2_approx(hmin);
+    step = spread ? (lg2_approx(hmax) - base) * (1.0f / (float)Lq) : 0.f;
   }
 
-  float2 v[P];
+  float2 v[8];
 #pragma unroll
-  for (int i = 0; i < P; ++i) {
-    const uint32_t k = get_bits<W>(aw, i * W);
-    const uint32_t c = get_bits<B>(nw, i * B);
-    float r;
-    if (J.mode == TAC_NORM_LINEAR) r = __fmaf_rn((float)c, step, base);
-    else r = exp2f(__fmaf_rn((float)c, step, base));
-    if (flat) r = hmin;
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t k = (uint32_t)(acc_a >> (j * W)) & (uint32_t)(n - 1);
+    const uint32_t c = (uint32_t)(acc_n >> (j * B)) & (uint32_t)Lq;
+    float rh = __fmaf_rn(__uint2float_rn(c), step, base);
+    if (J.mode != TAC_NORM_LINEAR) rh = ex2_approx(rh);
     const float2 t = ttab[k];
-    v[i] = mul2(make_float2(r, r), t);
+    v[j] = make_float2(rh * t.x, rh * t.y);
   }
-  // Remaining butterfly stages (input bits 1..log2 d - 1); H is its own inverse (Sec. 2).
+  // Butterfly stages on pair-index bits 0..2 (this lane holds pairs 8l..8l+7).
+  butterfly8<8>(v);
+  if constexpr (L > 1) {
+    uint8_t* tpb = smem + C::OFF_TP;
 #pragma unroll
-  for (int hh = 1; hh < P; hh <<= 1) {
+    for (int q = 0; q < 4; ++q)
+      *reinterpret_cast<float4*>(tpb + G::tp(r, 8 * l + 2 * q)) =
+          make_float4(v[2 * q].x, v[2 * q].y, v[2 * q + 1].x, v[2 * q + 1].y);
+    __syncwarp();
 #pragma unroll
-    for (int i = 0; i < P; ++i) {
-      if ((i & hh) == 0) {
-        const float2 a = v[i], b = v[i + hh];
-        v[i] = add2(a, b);
-        v[i + hh] = sub2(a, b);
-      }
-    }
+    for (int m = 0; m < 8; ++m) v[m] = *reinterpret_cast<const float2*>(tpb + G::tp(r, l + L * m));
+    // Stages on pair-index bits 3..log2(P)-1 (this lane now holds pairs l + L*m).
+    butterfly8<8, 8 / L>(v);
   }
-  // D, convert, stage the row (swizzled).
-  uint8_t* orow = smem + C::OFF_OUT + tid * C::ROWB;
-  const int sw = row_swz<C::ROWB>(tid);
-  if constexpr (C::ESZ == 2) {
+  // D, convert, stage the row: pair i = l + L*m is element pair (2i, 2i+1).
+  uint8_t* orow = smem + C::OFF_OUT + r * OT::STRIDE;
 #pragma unroll
-    for (int c = 0; c < C::CPR; ++c) {
-      uint32_t q[4];
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        const int i = 4 * c + t;
-        const __nv_bfloat162 b = __floats2bfloat162_rn(v[i].x, v[i].y);
-        q[t] = (*reinterpret_cast<const uint32_t*>(&b)) ^ msk[i].x;
-      }
-      *reinterpret_cast<uint4*>(orow + ((c ^ sw) << 4)) = make_uint4(q[0], q[1], q[2], q[3]);
-    }
-  } else {
-#pragma unroll
-    for (int c = 0; c < C::CPR; ++c) {
-      const int i0 = 2 * c, i1 = 2 * c + 1;
-      *reinterpret_cast<uint4*>(orow + ((c ^ sw) << 4)) =
-          make_uint4(__float_as_uint(v[i0].x) ^ msk[i0].x, __float_as_uint(v[i0].y) ^ msk[i0].y,
-                     __float_as_uint(v[i1].x) ^ msk[i1].x, __float_as_uint(v[i1].y) ^ msk[i1].y);
+  for (int m = 0; m < 8; ++m) {
+    const int i = l + L * m;
+    if constexpr (C::ESZ == 2) {
+      const __nv_bfloat162 bb = __floats2bfloat162_rn(v[m].x, v[m].y);
+      *reinterpret_cast<uint32_t*>(orow + 4 * i) = (*reinterpret_cast<const uint32_t*>(&bb)) ^ msk[m].x;
+    } else {
+      *reinterpret_cast<uint2*>(orow + 8 * i) =
+          make_uint2(__float_as_uint(v[m].x) ^ msk[m].x, __float_as_uint(v[m].y) ^ msk[m].y);
     }
   }
 }
@@ -213,18 +187,22 @@ __device__ __forceinline__ void decode_row(const DecJob& J, const uint8_t* rec, 
 template <int D, typename TOut>
 __device__ __forceinline__ void store_out_tile(const DecJob& J, const uint8_t* smem, int row0, int nrows, int tid) {
   using C = Dec<D, TOut>;
+  using OT = typename C::OT;
   uint8_t* y = reinterpret_cast<uint8_t*>(J.y);
-  const int total = nrows * C::CPR;
-  for (int id = tid; id < total; id += kThreads) {
-    const int r = id / C::CPR;
-    const int c = id - r * C::CPR;
-    const uint4 q = *reinterpret_cast<const uint4*>(smem + C::OFF_OUT + r * C::ROWB + ((c ^ row_swz<C::ROWB>(r)) << 4));
-    *reinterpret_cast<uint4*>(y + ((int64_t)(row0 + r) * J.stride) * C::ESZ + c * 16) = q;
+#pragma unroll
+  for (int q = 0; q < C::CHUNKS; ++q) {
+    const int id = q * kThreads + tid;
+    const int r = id / OT::CPR;
+    const int c = id - r * OT::CPR;
+    if (r < nrows) {
+      const uint4 v = *reinterpret_cast<const uint4*>(smem + C::OFF_OUT + r * OT::STRIDE + c * 16);
+      *reinterpret_cast<uint4*>(y + ((int64_t)(row0 + r) * J.stride) * C::ESZ + c * 16) = v;
+    }
   }
 }
 
 template <int D, typename TOut>
-__global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_constant__ DecParams p) {
+__global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_constant__ DecParams p) {
   using C = Dec<D, TOut>;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
@@ -243,34 +221,50 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
   }
 
   int jid = find_job(p, t);
-  build_dec_masks<D, TOut>(p.job[jid], reinterpret_cast<uint2*>(smem + C::OFF_MSK), tid);
-  {
-    const DecJob& J = p.job[jid];
-    const int row0 = (t - J.tile0) * kTileRows;
-    issue_rec_load<D, TOut>(J, row0, (int)min((int64_t)kTileRows, J.rows - row0), smem + C::OFF_REC, tid);
-    cp_async_commit();
-    const int t1 = t + G;
-    if (t1 < p.ntiles) {
-      const DecJob& J1 = p.job[find_job(p, t1)];
-      const int r1 = (t1 - J1.tile0) * kTileRows;
-      issue_rec_load<D, TOut>(J1, r1, (int)min((int64_t)kTileRows, J1.rows - r1), smem + C::OFF_REC + C::REC_B, tid);
+  int mask_jid = -1;
+  uint2 msk[8];
+#pragma unroll
+  for (int s = 0; s < kStages - 1; ++s) {
+    const int ts = t + s * G;
+    if (ts < p.ntiles) {
+      const DecJob& Js = p.job[find_job(p, ts)];
+      const int rs = (ts - Js.tile0) * C::TR;
+      issue_rec_load<D, TOut>(Js, rs, (int)min((int64_t)C::TR, Js.rows - rs), smem + C::OFF_REC + s * C::REC_B, tid);
     }
     cp_async_commit();
   }
 
   int cur = 0;
   for (; t < p.ntiles; t += G) {
-    cp_async_wait<1>();
-    __syncthreads();
+    cp_async_wait<kStages - 2>();   // this tile's group has landed
+    __syncthreads();                // ... and every thread is done with the previous tile
+    {
+      // Refill the buffer of the previous tile with the tile kStages - 1 ahead.
+      const int tn = t + (kStages - 1) * G;
+      int nb = cur + kStages - 1;
+      if (nb >= kStages) nb -= kStages;
+      if (tn < p.ntiles) {
+        const DecJob& Jn = p.job[find_job(p, tn)];
+        const int rn = (tn - Jn.tile0) * C::TR;
+        issue_rec_load<D, TOut>(Jn, rn, (int)min((int64_t)C::TR, Jn.rows - rn), smem + C::OFF_REC + nb * C::REC_B, tid);
+      }
+      cp_async_commit();
+    }
     const DecJob& J = p.job[jid];
-    const int row0 = (t - J.tile0) * kTileRows;
-    const int nrows = (int)min((int64_t)kTileRows, J.rows - row0);
+    if (jid != mask_jid) {
+      const int l = tid % C::L;
+#pragma unroll
+      for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
+      mask_jid = jid;
+    }
+    const int row0 = (t - J.tile0) * C::TR;
+    const int nrows = (int)min((int64_t)C::TR, J.rows - row0);
     const uint8_t* rec = smem + C::OFF_REC + cur * C::REC_B;
 
 #define TAC_DEC_CASE(WW)                                                      \
   case WW:                                                                    \
-    if (J.b == 8) decode_row<D, TOut, WW, 8>(J, rec, smem, tid);              \
-    else decode_row<D, TOut, WW, 4>(J, rec, smem, tid);                       \
+    if (J.b == 8) decode_row<D, TOut, WW, 8>(J, rec, smem, tid, msk);         \
+    else decode_row<D, TOut, WW, 4>(J, rec, smem, tid, msk);                  \
     break;
     switch (J.w) {
       TAC_DEC_CASE(1) TAC_DEC_CASE(2) TAC_DEC_CASE(3) TAC_DEC_CASE(4)
@@ -281,18 +275,8 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
     __syncthreads();
     store_out_tile<D, TOut>(J, smem, row0, nrows, tid);
 
-    const int t2 = t + 2 * G;
-    if (t2 < p.ntiles) {
-      const DecJob& J2 = p.job[find_job(p, t2)];
-      const int r2 = (t2 - J2.tile0) * kTileRows;
-      issue_rec_load<D, TOut>(J2, r2, (int)min((int64_t)kTileRows, J2.rows - r2), smem + C::OFF_REC + cur * C::REC_B, tid);
-    }
-    cp_async_commit();
-    if (t + G < p.ntiles) {
-      jid = find_job(p, t + G);
-      build_dec_masks<D, TOut>(p.job[jid], reinterpret_cast<uint2*>(smem + C::OFF_MSK), tid);
-    }
-    cur ^= 1;
+    if (t + G < p.ntiles) jid = find_job(p, t + G);
+    cur = (cur + 1 == kStages) ? 0 : cur + 1;
   }
   cp_async_wait<0>();
 }

@@ -5,9 +5,10 @@ Rules (derived in the design notes from the fp32 arithmetic of the kernels):
 angle codes   bit-exact wherever the oracle's angle lies 1e-5 rad or more from a
               bin edge; inside that band a differing code is counted, and the
               count must not exceed 1e-6 of all codes (below 10^6 codes: zero).
-header        |r_gpu - r_oracle| <= eps_h, eps_h = (2/sqrt d) gamma + 3 u r_max,
+header        |r_gpu - r_oracle| <= eps_h, eps_h = (2/sqrt d) gamma + 4 u r_max,
               gamma = (log2 d - 1) u ||x||_1: the first-order bound of the fp32
-              butterfly's rounding on a pair (u = 2^-24).
+              butterfly's rounding on a pair (u = 2^-24), plus the energy's
+              rounding and the hardware square root (<= 2 ulp).
 norm codes    bit-exact wherever the oracle's Eq. 2 pre-round value lies more than
               beta_i from a rounding midpoint, beta_i the propagated bound of the
               fp32 norm, header and Eq. 2 arithmetic; inside, a code may differ by
@@ -56,8 +57,11 @@ def _gamma(x64: np.ndarray) -> np.ndarray:
 
 
 def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, mode: int,
-                   label: str = "") -> dict:
-    """Check GPU codes (k, c, hdr) against oracle output `ref` for input rows x64."""
+                   label: str = "", structured: bool = False) -> dict:
+    """Check GPU codes (k, c, hdr) against oracle output `ref` for input rows x64.
+
+    `structured`: hand-built rows (constants, one-hots) put Eq. 2 values exactly on
+    rounding midpoints, so only the band rule (not the statistical rate) applies."""
     rows, d = x64.shape
     P = d // 2
     L = (1 << b) - 1
@@ -75,7 +79,7 @@ def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, m
     # ---- header ----
     gam = _gamma(x64)
     hmax_o = ref["hdr"][:, 1].astype(np.float64)
-    eps_h = (2.0 / math.sqrt(d)) * gam + 3 * U * hmax_o + 1e-45
+    eps_h = (2.0 / math.sqrt(d)) * gam + 4 * U * hmax_o + 1e-45
     dh = np.abs(hdr.astype(np.float64) - ref["hdr"].astype(np.float64))
     st["header_max_err_over_bound"] = float((dh / eps_h[:, None]).max()) if rows else 0.0
     assert np.all(dh <= eps_h[:, None]), (label, st)
@@ -83,7 +87,7 @@ def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, m
     # ---- norm codes ----
     hmin_o = ref["hdr"][:, 0].astype(np.float64)
     r = ref["r"]
-    eps_r = (2.0 / math.sqrt(d)) * gam[:, None] + 2 * U * r
+    eps_r = (2.0 / math.sqrt(d)) * gam[:, None] + 4 * U * r
     dh_range = np.maximum(hmax_o - hmin_o, 1e-300)
     if mode == 0:
         beta = L * (eps_r + 3 * eps_h[:, None]) / dh_range[:, None] + 4 * U * L
@@ -92,9 +96,10 @@ def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, m
         lmin = np.log2(np.maximum(hmin_o, 1e-300))
         lmax = np.log2(np.maximum(hmax_o, 1e-300))
         lrange = np.maximum(lmax - lmin, 1e-300)
-        dl = (eps_r / floor_r + 2 * U) / math.log(2) + 4 * U * np.abs(np.log2(floor_r))
-        dlmin = (eps_h / np.maximum(hmin_o, 1e-300) + 2 * U) / math.log(2) + 4 * U * np.abs(lmin)
-        dlmax = (eps_h / np.maximum(hmax_o, 1e-300) + 2 * U) / math.log(2) + 4 * U * np.abs(lmax)
+        # hardware log2: absolute error <= 2^-21 (plus relative rounding of the result)
+        dl = (eps_r / floor_r + 2 * U) / math.log(2) + 4 * U * np.abs(np.log2(floor_r)) + 2.0**-21
+        dlmin = (eps_h / np.maximum(hmin_o, 1e-300) + 2 * U) / math.log(2) + 4 * U * np.abs(lmin) + 2.0**-21
+        dlmax = (eps_h / np.maximum(hmax_o, 1e-300) + 2 * U) / math.log(2) + 4 * U * np.abs(lmax) + 2.0**-21
         beta = L * (dl + 3 * np.maximum(dlmin, dlmax)[:, None]) / lrange[:, None] + 4 * U * L
     flat = (ref["hdr"][:, 0] == ref["hdr"][:, 1])
     beta[flat] = 0.0
@@ -106,7 +111,8 @@ def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, m
     st["norm_mismatch_outside_band"] = int(bad.sum())
     st["norm_band_population"] = int((dist_mid <= beta).sum())
     assert st["norm_mismatch_outside_band"] == 0, (label, st, np.argwhere(bad)[:5])
-    assert st["norm_mismatch"] <= max(2, 1e-4 * st["codes"]), (label, st)
+    if not structured:
+        assert st["norm_mismatch"] <= max(2, 1e-4 * st["codes"]), (label, st)
     return st
 
 

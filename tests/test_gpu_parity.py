@@ -34,7 +34,8 @@ def _oracle_cache(tac, orc, cfg, ref):
     return cache
 
 
-def check_roundtrip(tac, orc, x, d, n, b, mode, seed=0, layer=0, kv=0, label="", decode_dtypes=("bf16", "fp32")):
+def check_roundtrip(tac, orc, x, d, n, b, mode, seed=0, layer=0, kv=0, label="", decode_dtypes=("bf16", "fp32"),
+                    structured=False):
     torch = _torch()
     rows = x.shape[0]
     cfg = tac.layer_cfg(d, n, b, mode, seed, layer, kv)
@@ -45,7 +46,7 @@ def check_roundtrip(tac, orc, x, d, n, b, mode, seed=0, layer=0, kv=0, label="",
     assert np.array_equal(s, parity.signs_pm1(cfg.signs, d))
     ref = orc.encode(x64, s, n, b, mode)
     k, c, hdr = parity.gpu_codes(orc, cache, rows)
-    st = parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=label)
+    st = parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=label, structured=structured)
     # decode on identical codes (the oracle's records) into bf16 and fp32
     oc = _oracle_cache(tac, orc, cfg, ref)
     v = orc.decode(ref["k"], ref["c"], ref["hdr"], s, n, b, mode)
@@ -147,7 +148,8 @@ def test_degenerate_rows(tac_gpu, orc):
     rows.append(a)
     x = torch.tensor(np.array(rows), dtype=torch.float32).to(torch.bfloat16).cuda()
     for n, b, mode in ((64, 8, 0), (64, 4, 1), (4, 8, 0), (2, 4, 1), (256, 8, 1)):
-        check_roundtrip(tac_gpu, orc, x, d, n, b, mode, label=f"degenerate n={n} b={b} m={mode}")
+        check_roundtrip(tac_gpu, orc, x, d, n, b, mode, label=f"degenerate n={n} b={b} m={mode}",
+                        structured=True)
 
 
 def test_exact_bin_centres_and_ties(tac_gpu, orc):
@@ -173,3 +175,43 @@ def test_exact_bin_centres_and_ties(tac_gpu, orc):
         assert np.array_equal(k, want), (n, k[:, :3], want[:, :3])
         if n == 4:
             assert np.all(k[0] == 1) and np.all(k[1] == 0) and np.all(k[2] == 1) and np.all(k[3] == 2)
+
+
+@pytest.mark.parametrize("d,n,b,mode", [(128, 64, 8, 0), (128, 256, 4, 1), (64, 128, 8, 0)])
+def test_many_tiles_per_cta_every_row(tac_gpu, orc, d, n, b, mode):
+    """Enough rows that every CTA of the persistent grid loops over many tiles
+    (exercising the multi-stage cp.async pipeline); every row is compared."""
+    import os
+    torch = _torch()
+    w = workloads.CONFIGS["mistral7b" if d == 128 else "llama1b"]
+    rows = 160_000 if d == 128 else 120_000
+    x = _rows(w, rows, seed=d + n, layer=3, kv=mode)
+    cfg = tac_gpu.layer_cfg(d, n, b, mode, 0, 3, mode)
+    cache = tac_gpu.encode(x, cfg)
+    y = tac_gpu.decode(cache, cfg)
+    torch.cuda.synchronize()
+    x64 = parity.to_f64(x)
+    s = orc.signs(0, 3, mode, d)
+    threads = os.cpu_count() or 1
+    ref = _encode_diag_threads(orc, x64, s, n, b, mode, threads)
+    k, c, hdr = parity.gpu_codes(orc, cache, rows)
+    parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=f"many tiles d{d} n{n}")
+    v = orc.decode_threads(k, c, hdr, s, n, b, mode, threads)
+    parity.compare_decode(parity.to_f64(y), v, "bf16", label=f"many tiles decode d{d} n{n}")
+
+
+def _encode_diag_threads(orc, x64, s, n, b, mode, threads):
+    """The oracle's encode with diagnostics, split over host threads by rows."""
+    import threading
+    parts = np.array_split(np.arange(x64.shape[0]), threads)
+    out = [None] * len(parts)
+
+    def work(i, idx):
+        out[i] = orc.encode(x64[idx[0]: idx[-1] + 1], s, n, b, mode)
+
+    ts = [threading.Thread(target=work, args=(i, p)) for i, p in enumerate(parts) if len(p)]
+    for t in ts:
+        t.start()
+    for t in ts:
+        t.join()
+    return {key: np.concatenate([o[key] for o in out if o is not None]) for key in out[0]}
