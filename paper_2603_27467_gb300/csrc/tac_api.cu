@@ -115,8 +115,8 @@ int64_t angle_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * l
 int64_t norm_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * c->norm_bits / 8; }
 int64_t header_offset(const tac_layer_cfg* c, int64_t cap) { return (cap * norm_row_bytes(c) + 15) & ~(int64_t)15; }
 
-// Rows per kernel tile: 256 threads, d/16 lanes per row (8 angle pairs per lane).
-int64_t tile_rows(int d) { return (int64_t)tac::kThreads / (d / 16); }
+// Rows per warp tile: 32 lanes, d/16 lanes per row (8 angle pairs per lane).
+int64_t tile_rows(int d) { return (int64_t)32 / (d / 16); }
 
 int esize(int dtype) { return dtype == TAC_BF16 ? 2 : dtype == TAC_FP32 ? 4 : 0; }
 

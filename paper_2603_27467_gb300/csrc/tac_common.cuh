@@ -19,36 +19,40 @@ constexpr float kU = 5.9604644775390625e-08f;  // fp32 unit roundoff 2^-24
 __host__ __device__ constexpr int tab_offset(int w) { return (1 << w) - 2; }
 
 // ---------------------------------------------------------------------------
-// Tile geometry for head dimension D: P = D/2 pairs per row, L = P/8 lanes per
-// row (each lane owns 8 pairs), TR = 256/L rows per tile.
+// Geometry for head dimension D.  P = D/2 angle pairs per row; each lane owns 8
+// pairs, so L = P/8 lanes share a row and a warp covers RW = 32/L rows (its
+// "warp tile").  Every warp runs its own pipeline over warp tiles.
 // ---------------------------------------------------------------------------
+constexpr int kWarps = kThreads / 32;
+
 template <int D>
 struct Geo {
   static constexpr int P = D / 2;
   static constexpr int L = P / kPairsPerThread;
-  static constexpr int TR = kThreads / L;
+  static constexpr int RW = 32 / L;
   static constexpr int LOGD = (D == 16) ? 4 : (D == 32) ? 5 : (D == 64) ? 6 : 7;
-  // Transpose buffer: one row of P float2 pairs, padded so that the phase-A
-  // pattern (lane l writes pairs l + L*m) and the phase-B pattern (lane l reads
-  // pairs 8l..8l+7 as four 16-byte granules) are both bank-conflict free.
-  static constexpr int ST = 8 * P + 32;
-  static constexpr int TP_B = TR * ST;
-  __device__ static __forceinline__ int tp(int r, int i) {
-    const int g = i >> 1;
-    return r * ST + ((g ^ ((g >> 2) & 7)) << 4) + ((i & 1) << 3);
-  }
+  // Transpose buffer (L > 1): pair i of warp-tile row r at
+  //   r*ST + (i / L)*SM + (i % L)*8.
+  // Lane l writes pairs l + L*m (m = 0..7: offsets m*SM, a linear stride) and
+  // reads pairs 8l..8l+7 as four 16-byte granules at (8/L)*l*SM + fixed offsets.
+  // SM and ST are padded so both patterns are bank-conflict free (d = 32..128).
+  static constexpr int SM = 8 * L + 16;
+  static constexpr int ST = 8 * SM + (L == 8 ? 64 : 16);
+  static constexpr int TP_W = (L > 1) ? RW * ST : 0;
+  __host__ __device__ static constexpr int tp_pair(int i) { return (i / L) * SM + (i % L) * 8; }
 };
 
-// Row-major element tile with a per-row pad chosen so that lane l of a row
-// accessing pair l + L*m (element bytes [2i*ESZ, 2i*ESZ + 2*ESZ)) hits distinct
-// banks across the rows of a warp; rows start on 16-byte boundaries.
+// Row-major element rows of a warp tile with a per-row pad such that lane l of a
+// row reading pair l + L*m (bytes [2i*ESZ, 2i*ESZ + 2*ESZ)) hits distinct banks
+// across the rows of the warp; rows start on 16-byte boundaries.
 template <int D, int ESZ>
 struct RowTile {
   static constexpr int ROWB = D * ESZ;
   static constexpr int CPR = ROWB / 16;
   static constexpr int SPAN = 2 * ESZ * Geo<D>::L;
   static constexpr int STRIDE = ROWB + (SPAN > 16 ? SPAN : 16);
-  static constexpr int BYTES = Geo<D>::TR * STRIDE;
+  static constexpr int BYTES = Geo<D>::RW * STRIDE;            // one warp tile
+  static constexpr int CHUNKS = Geo<D>::RW * CPR / 32;         // 16-byte chunks per lane
 };
 
 // ---------------------------------------------------------------------------

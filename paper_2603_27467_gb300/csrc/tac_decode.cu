@@ -21,77 +21,85 @@
 
 namespace tac {
 
-constexpr int kStages = 4;  // record tiles per CTA: 3 in flight while one is decoded
+constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles of records in flight
 
 template <int D, typename TOut>
 struct Dec {
   using G = Geo<D>;
   using OT = RowTile<D, (int)sizeof(TOut)>;
-  static constexpr int P = G::P, L = G::L, TR = G::TR;
+  static constexpr int P = G::P, L = G::L, RW = G::RW;
   static constexpr int ESZ = (int)sizeof(TOut);
-  static constexpr int ABMAX = P;                        // angle record bytes at w = 8
-  static constexpr int NBMAX = P;                        // norm record bytes at b = 8
-  static constexpr int R_ANG = 0;                        // inside a record buffer
-  static constexpr int R_NRM = TR * ABMAX;
-  static constexpr int R_HDR = R_NRM + TR * NBMAX;
-  static constexpr int REC_B = R_HDR + TR * 8 + 16;      // + slack for 3-word angle reads
-  // shared memory layout (bytes)
-  static constexpr int OFF_REC = 0;                      // kStages record buffers
-  static constexpr int OFF_TP = OFF_REC + kStages * REC_B; // transpose buffer
-  static constexpr int OFF_OUT = OFF_TP + G::TP_B;       // output tile
-  static constexpr int OFF_TAB = OFF_OUT + OT::BYTES;    // centre tables, every n
+  // one record stage of a warp tile: angle, norm and header segments
+  static constexpr int R_ANG = 0;
+  static constexpr int R_NRM = RW * P;                      // angle records <= P bytes per row
+  static constexpr int R_HDR = R_NRM + RW * P;              // norm records <= P bytes per row
+  static constexpr int REC_W = R_HDR + RW * 8 + 16;         // + slack for 3-word angle reads
+  // per-warp shared memory region
+  static constexpr int W_REC = 0;                           // kNS record stages
+  static constexpr int W_TP = W_REC + kNS * REC_W;          // transpose rows
+  static constexpr int W_OUT = W_TP + G::TP_W;              // output rows
+  static constexpr int W_JOB = W_OUT + OT::BYTES;           // current job (DecWarpJob)
+  static constexpr int WARP_B = W_JOB + 128;
+  static constexpr int OFF_TAB = kWarps * WARP_B;           // centre tables, every n
   static constexpr int SMEM = OFF_TAB + kTabEntries * 8;
-  static constexpr int CHUNKS = TR * OT::CPR / kThreads;
-  static_assert(TR * OT::CPR % kThreads == 0, "tile chunks");
-  static_assert(REC_B % 16 == 0, "record buffer alignment");
+  static_assert(REC_W % 16 == 0 && W_OUT % 16 == 0 && W_JOB % 16 == 0, "alignment");
 };
 
-// Cooperative cp.async of `bytes` contiguous bytes (16-byte aligned global base),
-// zero-filling the tail of the last chunk.
-__device__ __forceinline__ void cta_copy_in(uint8_t* s, const uint8_t* g, int bytes, int tid) {
-  const int nch = (bytes + 15) >> 4;
-  for (int q = tid; q < nch; q += kThreads) {
-    const int rem = bytes - (q << 4);
-    cp_async16(s + (q << 4), g + (q << 4), rem >= 16 ? 16 : rem);
-  }
-}
+struct DecWarpJob {
+  void* y;
+  int64_t rows;
+  int64_t stride;  // elements
+  int32_t t0, end, variant, pad_;
+};
+static_assert(sizeof(DecWarpJob) <= 128, "DecWarpJob");
 
+// Stage the records of warp tile (row0, nrows) of a job into `stage`.
+// Contiguous slots: 16-byte cp.async chunks of the three plane segments (a
+// segment of a full tile is a multiple of 16 bytes; a tail tile's last chunk is
+// zero-filled).  Gathered slots: lane r < nrows copies row r's record with plain loads.
 template <int D, typename TOut>
-__device__ __forceinline__ void issue_rec_load(const DecJob& J, int row0, int nrows, uint8_t* buf, int tid) {
+__device__ __forceinline__ void stage_records(const uint8_t* codes, const uint8_t* norms, const uint8_t* hdr,
+                                              const int64_t* slot, int64_t capacity, int64_t row0, int nrows,
+                                              int AB, int NB, uint8_t* stage, int lane) {
   using C = Dec<D, TOut>;
-  const int AB = C::P * J.w / 8, NB = C::P * J.b / 8;
-  if (J.slot == nullptr) {
-    cta_copy_in(buf + C::R_ANG, J.codes + (int64_t)row0 * AB, nrows * AB, tid);
-    cta_copy_in(buf + C::R_NRM, J.norms + (int64_t)row0 * NB, nrows * NB, tid);
-    cta_copy_in(buf + C::R_HDR, J.hdr + (int64_t)row0 * 8, nrows * 8, tid);
-  } else {
-    // Gather: one thread per row copies its record byte-exactly with plain loads
-    // (records of odd size are not 16-byte aligned in the source planes).
-    for (int rr = tid; rr < nrows; rr += kThreads) {
-      const int64_t s = J.slot[row0 + rr];
-      uint8_t* da = buf + C::R_ANG + rr * AB;
-      uint8_t* dn = buf + C::R_NRM + rr * NB;
-      float2* dh = reinterpret_cast<float2*>(buf + C::R_HDR) + rr;
-      if (s < 0 || s >= J.capacity) {  // out-of-range slot: decodes as an all-zero record
-        for (int q = 0; q < AB; ++q) da[q] = 0;
-        for (int q = 0; q < NB; ++q) dn[q] = 0;
-        *dh = make_float2(0.f, 0.f);
-        continue;
-      }
-      const uint8_t* sa = J.codes + s * AB;
-      const uint8_t* sn = J.norms + s * NB;
-      if ((AB & 3) == 0) {
-        for (int q = 0; q < AB / 4; ++q) reinterpret_cast<uint32_t*>(da)[q] = __ldg(reinterpret_cast<const uint32_t*>(sa) + q);
+  if (slot == nullptr) {
+    const int ba = nrows * AB, bn = nrows * NB, bh = nrows * 8;
+    const int ca = (ba + 15) >> 4, cn = (bn + 15) >> 4, ch = (bh + 15) >> 4;
+    const uint8_t* ga = codes + row0 * AB;
+    const uint8_t* gn = norms + row0 * NB;
+    const uint8_t* gh = hdr + row0 * 8;
+    for (int q = lane; q < ca + cn + ch; q += 32) {
+      if (q < ca) {
+        const int rem = ba - 16 * q;
+        cp_async16(stage + C::R_ANG + 16 * q, ga + 16 * q, rem >= 16 ? 16 : rem);
+      } else if (q < ca + cn) {
+        const int qq = q - ca, rem = bn - 16 * qq;
+        cp_async16(stage + C::R_NRM + 16 * qq, gn + 16 * qq, rem >= 16 ? 16 : rem);
       } else {
-        for (int q = 0; q < AB; ++q) da[q] = __ldg(sa + q);
+        const int qq = q - ca - cn, rem = bh - 16 * qq;
+        cp_async16(stage + C::R_HDR + 16 * qq, gh + 16 * qq, rem >= 16 ? 16 : rem);
       }
-      if ((NB & 3) == 0) {
-        for (int q = 0; q < NB / 4; ++q) reinterpret_cast<uint32_t*>(dn)[q] = __ldg(reinterpret_cast<const uint32_t*>(sn) + q);
-      } else {
-        for (int q = 0; q < NB; ++q) dn[q] = __ldg(sn + q);
-      }
-      *dh = __ldg(reinterpret_cast<const float2*>(J.hdr) + s);
     }
+  } else if (lane < nrows) {
+    const int64_t s = slot[row0 + lane];
+    uint8_t* da = stage + C::R_ANG + lane * AB;
+    uint8_t* dn = stage + C::R_NRM + lane * NB;
+    float2* dh = reinterpret_cast<float2*>(stage + C::R_HDR) + lane;
+    if (s < 0 || s >= capacity) {  // out-of-range slot: decodes as an all-zero record
+      for (int q = 0; q < AB; ++q) da[q] = 0;
+      for (int q = 0; q < NB; ++q) dn[q] = 0;
+      *dh = make_float2(0.f, 0.f);
+      return;
+    }
+    const uint8_t* sa = codes + s * AB;
+    const uint8_t* sn = norms + s * NB;
+    if ((AB & 3) == 0) {
+      for (int q = 0; q < AB / 4; ++q) reinterpret_cast<uint32_t*>(da)[q] = __ldg(reinterpret_cast<const uint32_t*>(sa) + q);
+    } else {
+      for (int q = 0; q < AB; ++q) da[q] = __ldg(sa + q);
+    }
+    for (int q = 0; q < NB / 4; ++q) reinterpret_cast<uint32_t*>(dn)[q] = __ldg(reinterpret_cast<const uint32_t*>(sn) + q);
+    *dh = __ldg(reinterpret_cast<const float2*>(hdr) + s);
   }
 }
 
@@ -114,9 +122,10 @@ __device__ __forceinline__ uint64_t load_bytes(const uint8_t* p) {
   }
 }
 
-template <int D, typename TOut, int W, int B>
-__device__ __forceinline__ void decode_row(const DecJob& J, const uint8_t* rec, uint8_t* smem, int tid,
-                                           const uint2 (&msk)[8]) {
+// Decode this lane's 8 pairs of warp-tile row r and stage the output row segment.
+template <int D, typename TOut, int W, int B, int MODE>
+__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab_all, int lane,
+                                            const uint2 (&msk)[8]) {
   using C = Dec<D, TOut>;
   using G = Geo<D>;
   using OT = typename C::OT;
@@ -125,8 +134,8 @@ __device__ __forceinline__ void decode_row(const DecJob& J, const uint8_t* rec, 
   constexpr int AB = P * W / 8;
   constexpr int NB = P * B / 8;
   constexpr int Lq = (1 << B) - 1;
-  const int r = tid / L, l = tid % L;
-  const float2* ttab = reinterpret_cast<const float2*>(smem + C::OFF_TAB) + tab_offset(W);
+  const int r = lane / L, l = lane % L;
+  const float2* ttab = ttab_all + tab_offset(W);
 
   const uint64_t acc_a = load_bytes<W>(rec + C::R_ANG + r * AB + l * W);
   const uint64_t acc_n = load_bytes<B>(rec + C::R_NRM + r * NB + l * B);
@@ -137,7 +146,7 @@ __device__ __forceinline__ void decode_row(const DecJob& J, const uint8_t* rec, 
   // log r^ = 2^(l_min + c (l_max - l_min)/L); r_max == r_min gives r^ = r_min.
   const bool spread = hmax > hmin;
   float base, step;
-  if (J.mode == TAC_NORM_LINEAR) {
+  if constexpr (MODE == TAC_NORM_LINEAR) {
     base = hmin;
     step = spread ? (hmax - hmin) * (1.0f / (float)Lq) : 0.f;
   } else {
@@ -151,52 +160,35 @@ __device__ __forceinline__ void decode_row(const DecJob& J, const uint8_t* rec, 
     const uint32_t k = (uint32_t)(acc_a >> (j * W)) & (uint32_t)(n - 1);
     const uint32_t c = (uint32_t)(acc_n >> (j * B)) & (uint32_t)Lq;
     float rh = __fmaf_rn(__uint2float_rn(c), step, base);
-    if (J.mode != TAC_NORM_LINEAR) rh = ex2_approx(rh);
+    if constexpr (MODE != TAC_NORM_LINEAR) rh = ex2_approx(rh);
     const float2 t = ttab[k];
     v[j] = make_float2(rh * t.x, rh * t.y);
   }
   // Butterfly stages on pair-index bits 0..2 (this lane holds pairs 8l..8l+7).
   butterfly8<8>(v);
   if constexpr (L > 1) {
-    uint8_t* tpb = smem + C::OFF_TP;
+    uint8_t* tpr = wsm + C::W_TP + r * G::ST;
+    uint8_t* tpl = tpr + (8 / L) * l * G::SM;
 #pragma unroll
     for (int q = 0; q < 4; ++q)
-      *reinterpret_cast<float4*>(tpb + G::tp(r, 8 * l + 2 * q)) =
+      *reinterpret_cast<float4*>(tpl + G::tp_pair(2 * q)) =
           make_float4(v[2 * q].x, v[2 * q].y, v[2 * q + 1].x, v[2 * q + 1].y);
     __syncwarp();
 #pragma unroll
-    for (int m = 0; m < 8; ++m) v[m] = *reinterpret_cast<const float2*>(tpb + G::tp(r, l + L * m));
+    for (int m = 0; m < 8; ++m) v[m] = *reinterpret_cast<const float2*>(tpr + m * G::SM + 8 * l);
     // Stages on pair-index bits 3..log2(P)-1 (this lane now holds pairs l + L*m).
     butterfly8<8, 8 / L>(v);
   }
   // D, convert, stage the row: pair i = l + L*m is element pair (2i, 2i+1).
-  uint8_t* orow = smem + C::OFF_OUT + r * OT::STRIDE;
+  uint8_t* orow = wsm + C::W_OUT + r * OT::STRIDE + 2 * C::ESZ * l;
 #pragma unroll
   for (int m = 0; m < 8; ++m) {
-    const int i = l + L * m;
     if constexpr (C::ESZ == 2) {
       const __nv_bfloat162 bb = __floats2bfloat162_rn(v[m].x, v[m].y);
-      *reinterpret_cast<uint32_t*>(orow + 4 * i) = (*reinterpret_cast<const uint32_t*>(&bb)) ^ msk[m].x;
+      *reinterpret_cast<uint32_t*>(orow + 4 * L * m) = (*reinterpret_cast<const uint32_t*>(&bb)) ^ msk[m].x;
     } else {
-      *reinterpret_cast<uint2*>(orow + 8 * i) =
+      *reinterpret_cast<uint2*>(orow + 8 * L * m) =
           make_uint2(__float_as_uint(v[m].x) ^ msk[m].x, __float_as_uint(v[m].y) ^ msk[m].y);
-    }
-  }
-}
-
-template <int D, typename TOut>
-__device__ __forceinline__ void store_out_tile(const DecJob& J, const uint8_t* smem, int row0, int nrows, int tid) {
-  using C = Dec<D, TOut>;
-  using OT = typename C::OT;
-  uint8_t* y = reinterpret_cast<uint8_t*>(J.y);
-#pragma unroll
-  for (int q = 0; q < C::CHUNKS; ++q) {
-    const int id = q * kThreads + tid;
-    const int r = id / OT::CPR;
-    const int c = id - r * OT::CPR;
-    if (r < nrows) {
-      const uint4 v = *reinterpret_cast<const uint4*>(smem + C::OFF_OUT + r * OT::STRIDE + c * 16);
-      *reinterpret_cast<uint4*>(y + ((int64_t)(row0 + r) * J.stride) * C::ESZ + c * 16) = v;
     }
   }
 }
@@ -204,11 +196,10 @@ __device__ __forceinline__ void store_out_tile(const DecJob& J, const uint8_t* s
 template <int D, typename TOut>
 __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_constant__ DecParams p) {
   using C = Dec<D, TOut>;
+  using OT = typename C::OT;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
-  const int G = gridDim.x;
-  int t = blockIdx.x;
-  if (t >= p.ntiles) return;
+  const int warp = tid >> 5, lane = tid & 31;
 
   // Centre tables for every n = 2..256: (cos + sin, cos - sin)(2 pi k / n) / sqrt(d).
   float2* ttab = reinterpret_cast<float2*>(smem + C::OFF_TAB);
@@ -219,64 +210,92 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
     const float2 cs = cos_sin_q8(centre_q8(k, 1 << w), 1 << w);  // (cos psi, sin psi), psi = phi + pi/4
     ttab[idx] = make_float2(sc * cs.y, sc * cs.x);
   }
+  __syncthreads();
 
-  int jid = find_job(p, t);
-  int mask_jid = -1;
-  uint2 msk[8];
-#pragma unroll
-  for (int s = 0; s < kStages - 1; ++s) {
-    const int ts = t + s * G;
-    if (ts < p.ntiles) {
-      const DecJob& Js = p.job[find_job(p, ts)];
-      const int rs = (ts - Js.tile0) * C::TR;
-      issue_rec_load<D, TOut>(Js, rs, (int)min((int64_t)C::TR, Js.rows - rs), smem + C::OFF_REC + s * C::REC_B, tid);
+  const int Gw = gridDim.x * kWarps;
+  int t = blockIdx.x * kWarps + warp;
+  if (t >= p.ntiles) return;
+  uint8_t* wsm = smem + warp * C::WARP_B;
+
+  // Prefetch cursor: the job of the next warp tile whose records are staged.
+  int pj = find_job(p, t);
+  int p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
+  auto issue = [&](int tt, int stg) {
+    if (tt < p.ntiles) {
+      while (tt >= p_end) {
+        ++pj;
+        p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
+      }
+      const DecJob& J = p.job[pj];
+      const int64_t row0 = (int64_t)(tt - J.tile0) * C::RW;
+      const int nrows = (int)min((int64_t)C::RW, J.rows - row0);
+      stage_records<D, TOut>(J.codes, J.norms, J.hdr, J.slot, J.capacity, row0, nrows, C::P * J.w / 8,
+                             C::P * J.b / 8, wsm + C::W_REC + stg * C::REC_W, lane);
     }
     cp_async_commit();
-  }
+  };
+#pragma unroll
+  for (int s = 0; s < kNS - 1; ++s) issue(t + s * Gw, s);
 
-  int cur = 0;
-  for (; t < p.ntiles; t += G) {
-    cp_async_wait<kStages - 2>();   // this tile's group has landed
-    __syncthreads();                // ... and every thread is done with the previous tile
+  DecWarpJob* wj = reinterpret_cast<DecWarpJob*>(wsm + C::W_JOB);
+  int cj = -1, c_end = 0;
+  uint2 msk[8];
+#pragma unroll
+  for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
+
+  int stage = 0;
+  for (; t < p.ntiles; t += Gw) {
+    cp_async_wait<kNS - 2>();   // this warp tile's records have landed
+    __syncwarp();               // ... and every lane is done with the previous tile
     {
-      // Refill the buffer of the previous tile with the tile kStages - 1 ahead.
-      const int tn = t + (kStages - 1) * G;
-      int nb = cur + kStages - 1;
-      if (nb >= kStages) nb -= kStages;
-      if (tn < p.ntiles) {
-        const DecJob& Jn = p.job[find_job(p, tn)];
-        const int rn = (tn - Jn.tile0) * C::TR;
-        issue_rec_load<D, TOut>(Jn, rn, (int)min((int64_t)C::TR, Jn.rows - rn), smem + C::OFF_REC + nb * C::REC_B, tid);
-      }
-      cp_async_commit();
+      int ns = stage + kNS - 1;
+      if (ns >= kNS) ns -= kNS;
+      issue(t + (kNS - 1) * Gw, ns);
     }
-    const DecJob& J = p.job[jid];
-    if (jid != mask_jid) {
-      const int l = tid % C::L;
+    if (t >= c_end) {  // next job: copy its descriptor to shared memory
+      cj = (cj < 0) ? find_job(p, t) : cj + 1;
+      while (cj + 1 < p.njobs && p.job[cj + 1].tile0 <= t) ++cj;
+      const DecJob& J = p.job[cj];
+      c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
+      if (lane == 0) {
+        wj->y = J.y; wj->rows = J.rows; wj->stride = J.stride; wj->t0 = J.tile0; wj->end = c_end;
+        wj->variant = (J.w - 1) * 4 + (J.b == 8 ? 2 : 0) + (J.mode == TAC_NORM_LOG ? 1 : 0);
+      }
+      const int l = lane % C::L;
 #pragma unroll
       for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
-      mask_jid = jid;
+      __syncwarp();
     }
-    const int row0 = (t - J.tile0) * C::TR;
-    const int nrows = (int)min((int64_t)C::TR, J.rows - row0);
-    const uint8_t* rec = smem + C::OFF_REC + cur * C::REC_B;
+    const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;
 
-#define TAC_DEC_CASE(WW)                                                      \
-  case WW:                                                                    \
-    if (J.b == 8) decode_row<D, TOut, WW, 8>(J, rec, smem, tid, msk);         \
-    else decode_row<D, TOut, WW, 4>(J, rec, smem, tid, msk);                  \
-    break;
-    switch (J.w) {
+#define TAC_DEC_CASE(WW)                                                                              \
+  case (WW - 1) * 4 + 0: decode_body<D, TOut, WW, 4, TAC_NORM_LINEAR>(rec, wsm, ttab, lane, msk); break;  \
+  case (WW - 1) * 4 + 1: decode_body<D, TOut, WW, 4, TAC_NORM_LOG>(rec, wsm, ttab, lane, msk); break;     \
+  case (WW - 1) * 4 + 2: decode_body<D, TOut, WW, 8, TAC_NORM_LINEAR>(rec, wsm, ttab, lane, msk); break;  \
+  case (WW - 1) * 4 + 3: decode_body<D, TOut, WW, 8, TAC_NORM_LOG>(rec, wsm, ttab, lane, msk); break;
+    switch (wj->variant) {
       TAC_DEC_CASE(1) TAC_DEC_CASE(2) TAC_DEC_CASE(3) TAC_DEC_CASE(4)
       TAC_DEC_CASE(5) TAC_DEC_CASE(6) TAC_DEC_CASE(7) TAC_DEC_CASE(8)
       default: break;
     }
 #undef TAC_DEC_CASE
-    __syncthreads();
-    store_out_tile<D, TOut>(J, smem, row0, nrows, tid);
-
-    if (t + G < p.ntiles) jid = find_job(p, t + G);
-    cur = (cur + 1 == kStages) ? 0 : cur + 1;
+    __syncwarp();
+    // Write the warp tile's rows: 16-byte chunks, coalesced.
+    {
+      const int64_t row0 = (int64_t)(t - wj->t0) * C::RW;
+      const int nrows = (int)min((int64_t)C::RW, wj->rows - row0);
+      uint8_t* y = reinterpret_cast<uint8_t*>(wj->y);
+      const int64_t sb = wj->stride * C::ESZ;
+#pragma unroll
+      for (int q = 0; q < OT::CHUNKS; ++q) {
+        const int id = q * 32 + lane;
+        const int rr = id / OT::CPR, col = (id % OT::CPR) * 16;
+        if (rr < nrows)
+          *reinterpret_cast<uint4*>(y + (row0 + rr) * sb + col) =
+              *reinterpret_cast<const uint4*>(wsm + C::W_OUT + rr * OT::STRIDE + col);
+      }
+    }
+    stage = (stage + 1 == kNS) ? 0 : stage + 1;
   }
   cp_async_wait<0>();
 }
@@ -298,7 +317,8 @@ static cudaError_t launch_decode_t(const DecParams& p, int grid_cap, cudaStream_
   if (e != cudaSuccess) return e;
   if (per_sm < 1) per_sm = 1;
   int grid = grid_cap * per_sm;
-  if (grid > p.ntiles) grid = p.ntiles;
+  const int need = (p.ntiles + kWarps - 1) / kWarps;
+  if (grid > need) grid = need;
   if (grid < 1) return cudaSuccess;
   kern<<<grid, kThreads, C::SMEM, st>>>(p);
   return cudaGetLastError();

@@ -1,9 +1,10 @@
 // TurboAngle encode kernel for sm_103a (Alg. 1 + Sec. 3.3 / Eq. 2 of arXiv 2603.27467).
 //
-// A 256-thread CTA encodes a tile of TR = 256/L rows; each row is shared by
-// L = d/16 consecutive lanes and each lane owns 8 angle pairs (16 elements).
-//   1. Tiles are staged global -> shared with cp.async (coalesced 16-byte
-//      chunks, double buffered, padded rows).
+// Work is split into warp tiles: L = d/16 lanes share a row, each lane owns 8
+// angle pairs (16 elements), so a warp encodes RW = 32/L rows at a time.  Every
+// warp runs its own pipeline (no block-wide barrier in the main loop):
+//   1. a kNS-stage cp.async ring stages its warp tiles global -> shared
+//      (coalesced 16-byte chunks, padded rows);
 //   2. D is a sign XOR on the raw input bits.  The unnormalized Walsh-Hadamard
 //      butterfly runs in two register phases on packed fp32 pairs (FADD2/FFMA2):
 //      phase A over the pair-index bits held in registers (lane l holds pairs
@@ -11,18 +12,18 @@
 //      bits (lane l then holds pairs 8l..8l+7).  The element-pair stage (input
 //      bit 0) is never executed: for output pair i the butterfly halves
 //      E_i = WHT_i(x_even), O_i = WHT_i(x_odd) give (y_2i, y_2i+1) = (E+O, E-O),
-//      so r_i^2 = 2 (E_i^2 + O_i^2) / d and the angle test works on (E_i, O_i).
+//      so r_i^2 = 2 (E_i^2 + O_i^2) / d and the angle test works on (E_i, O_i);
 //   3. Alg. 1's k_i = floor(n theta/2pi + 1/2) mod n is decided by an exact edge
 //      test: a candidate edge from an octant-reduced arctangent polynomial
 //      (max error 0.0038 rad: Rajan, Wang, Inkol, Joyal, "Efficient
 //      approximations for the arctangent function", IEEE SPM 2006), then the sign
 //      of the cross product of (E, O) with the edge direction.  The test is
 //      certified by a rigorous bound on the fp32 error; pairs inside it are
-//      re-decided by the warp in fp64 from the staged input (exact sums).
-//   4. Eq. 2 norm codes (linear, or on log2 r) against the stored fp32 (r_min, r_max).
-//   5. Each lane packs its 8 codes (8 log2(n) bits, 8 b bits) LSB-first; records
-//      are staged in shared memory and written with coalesced stores, or to per-row
-//      slots (scatter-append).
+//      re-decided by the warp in fp64 from the staged input (exact sums);
+//   4. Eq. 2 norm codes (linear, or on log2 r) against the stored fp32 (r_min, r_max);
+//   5. each lane packs its 8 codes LSB-first; the warp stages its records in
+//      shared memory and writes them with 16-byte stores (contiguous slots) or
+//      per row (scatter-append slots).
 #include "tac_common.cuh"
 
 namespace tac {
@@ -31,110 +32,82 @@ namespace tac {
 // warp-uniformly by the exact-decision path.
 __constant__ cx::EdgeTable g_edge_dir = cx::make_edge_table();
 
-constexpr int kStages = 4;  // input tiles per CTA: 3 in flight while one is encoded
+constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles in flight
 
 template <int D, typename TIn>
 struct Enc {
   using G = Geo<D>;
   using IT = RowTile<D, (int)sizeof(TIn)>;
-  static constexpr int P = G::P, L = G::L, TR = G::TR;
+  static constexpr int P = G::P, L = G::L, RW = G::RW;
   static constexpr int ESZ = (int)sizeof(TIn);
-  static constexpr int ABMAX = P;   // angle record bytes at w = 8
-  static constexpr int NBMAX = P;   // norm record bytes at b = 8
-  // shared memory layout (bytes)
-  static constexpr int OFF_IN = 0;                           // kStages input tiles
-  static constexpr int OFF_TP = OFF_IN + kStages * IT::BYTES; // transpose buffer
-  static constexpr int OFF_ANG = OFF_TP + G::TP_B;           // staged angle records
-  static constexpr int OFF_NRM = OFF_ANG + TR * ABMAX;       // staged norm records
-  static constexpr int OFF_HDR = OFF_NRM + TR * NBMAX;       // staged headers
-  static constexpr int OFF_TAB = OFF_HDR + TR * 8;           // edge tables, every n
+  // per-warp shared memory region
+  static constexpr int W_IN = 0;                            // kNS input stages
+  static constexpr int W_TP = W_IN + kNS * IT::BYTES;       // transpose rows
+  static constexpr int W_ANG = W_TP + G::TP_W;              // staged angle records (<= P bytes/row)
+  static constexpr int W_NRM = W_ANG + RW * P;              // staged norm records (<= P bytes/row)
+  static constexpr int W_HDR = W_NRM + RW * P;              // staged headers
+  static constexpr int W_JOB = (W_HDR + RW * 8 + 15) / 16 * 16;  // current job (WarpJob)
+  static constexpr int WARP_B = W_JOB + 128;
+  static constexpr int OFF_TAB = kWarps * WARP_B;           // fp32 edge tables, every n
   static constexpr int SMEM = OFF_TAB + kTabEntries * 8;
-  static constexpr int CHUNKS = TR * IT::CPR / kThreads;     // cp.async chunks per thread
-  static_assert(TR * IT::CPR % kThreads == 0, "tile chunks");
 };
 
-__device__ __forceinline__ void cta_copy_out(uint8_t* g, const uint8_t* s, int bytes, int tid) {
-  const int n16 = bytes >> 4;
-  for (int q = tid; q < n16; q += kThreads)
-    reinterpret_cast<uint4*>(g)[q] = reinterpret_cast<const uint4*>(s)[q];
-  for (int q = (n16 << 4) + tid; q < bytes; q += kThreads) g[q] = s[q];
-}
+// The job a warp is encoding, copied from the kernel parameters into the warp's
+// shared region when the warp reaches a new job (keeps it out of registers).
+struct WarpJob {
+  uint8_t* codes;
+  uint8_t* norms;
+  uint8_t* hdr;
+  const int64_t* slot;
+  int64_t capacity;
+  int64_t rows;
+  int32_t t0, end, variant, ab, nb, pad_;
+  uint32_t signs[4];
+};
+static_assert(sizeof(WarpJob) <= 128, "WarpJob");
 
-// Copy BYTES bytes (one record) shared -> global at a slot.
-template <int BYTES>
-__device__ __forceinline__ void copy_record(uint8_t* g, const uint8_t* s) {
-  if constexpr (BYTES % 16 == 0) {
-#pragma unroll
-    for (int q = 0; q < BYTES / 16; ++q) reinterpret_cast<uint4*>(g)[q] = reinterpret_cast<const uint4*>(s)[q];
-  } else if constexpr (BYTES % 8 == 0) {
-#pragma unroll
-    for (int q = 0; q < BYTES / 8; ++q) reinterpret_cast<uint2*>(g)[q] = reinterpret_cast<const uint2*>(s)[q];
-  } else if constexpr (BYTES % 4 == 0) {
-#pragma unroll
-    for (int q = 0; q < BYTES / 4; ++q) reinterpret_cast<uint32_t*>(g)[q] = reinterpret_cast<const uint32_t*>(s)[q];
-  } else {
-#pragma unroll
-    for (int q = 0; q < BYTES; ++q) g[q] = s[q];
-  }
-}
-
-// Store the low NBYTES bytes of v at a shared address aligned to gcd(NBYTES, 8).
+// Store the low NBYTES (<= 8) bytes of (hi:lo) at a shared address aligned to gcd(NBYTES, 8).
 template <int NBYTES>
-__device__ __forceinline__ void store_bytes(uint8_t* dst, uint64_t v) {
+__device__ __forceinline__ void store_bytes(uint8_t* dst, uint32_t lo, uint32_t hi) {
   if constexpr (NBYTES == 8) {
-    *reinterpret_cast<uint2*>(dst) = make_uint2((uint32_t)v, (uint32_t)(v >> 32));
+    *reinterpret_cast<uint2*>(dst) = make_uint2(lo, hi);
   } else if constexpr (NBYTES == 4) {
-    *reinterpret_cast<uint32_t*>(dst) = (uint32_t)v;
+    *reinterpret_cast<uint32_t*>(dst) = lo;
   } else if constexpr (NBYTES % 2 == 0) {
 #pragma unroll
-    for (int q = 0; q < NBYTES / 2; ++q) reinterpret_cast<uint16_t*>(dst)[q] = (uint16_t)(v >> (16 * q));
+    for (int q = 0; q < NBYTES / 2; ++q)
+      reinterpret_cast<uint16_t*>(dst)[q] = (uint16_t)((q < 2 ? lo : hi) >> (16 * (q & 1)));
   } else {
 #pragma unroll
-    for (int q = 0; q < NBYTES; ++q) dst[q] = (uint8_t)(v >> (8 * q));
+    for (int q = 0; q < NBYTES; ++q) dst[q] = (uint8_t)((q < 4 ? lo : hi) >> (8 * (q & 3)));
   }
 }
 
+// Exact re-decision of pair i of warp-tile row rr by the whole warp (all lanes
+// call it with the same arguments).  E_i, O_i are summed in fp64 from the staged
+// input (each term is an exactly representable signed input element), the
+// candidate edge comes from an fp32 atan2 of the exact values and the edge test
+// is evaluated in fp64 against an fp64 edge direction.  Returns k in every lane.
 template <int D, typename TIn>
-__device__ __forceinline__ void issue_tile_load(const EncJob& J, int row0, uint8_t* buf, int tid) {
+__device__ __forceinline__ int exact_angle_code(const uint32_t* signs, int w, const uint8_t* in, int rr, int i,
+                                             int lane) {
   using C = Enc<D, TIn>;
   using IT = typename C::IT;
-  const uint8_t* x = reinterpret_cast<const uint8_t*>(J.x);
-#pragma unroll
-  for (int q = 0; q < C::CHUNKS; ++q) {
-    const int id = q * kThreads + tid;
-    const int r = id / IT::CPR;
-    const int c = id - r * IT::CPR;
-    const int64_t grow = (int64_t)row0 + r;
-    const bool ok = grow < J.rows;
-    const uint8_t* src = ok ? x + (grow * J.stride) * C::ESZ + c * 16 : x;
-    cp_async16(buf + r * IT::STRIDE + c * 16, src, ok ? 16 : 0);
-  }
-}
-
-// Exact re-decision of pair i of tile row rr by one warp (all lanes call it with
-// the same arguments).  E_i, O_i are summed in fp64 from the staged input (each
-// term is an exactly representable signed input element), the candidate edge is
-// taken from an fp32 atan2 of the exact values and the edge test is evaluated in
-// fp64 against an fp64 edge direction.  Returns k (valid in every lane).
-template <int D, typename TIn>
-__device__ __noinline__ int exact_angle_code(const EncJob& J, const uint8_t* in, int rr, int i, int lane) {
-  using C = Enc<D, TIn>;
-  using IT = typename C::IT;
-  const int n = 1 << J.w;
+  const int n = 1 << w;
   double Ep = 0.0, Op = 0.0;
   const uint8_t* row = in + rr * IT::STRIDE;
   for (int jj = lane; jj < C::P; jj += 32) {
     const int j0 = 2 * jj, j1 = 2 * jj + 1;
     float x0, x1;
     if constexpr (C::ESZ == 2) {
-      const uint32_t w = *reinterpret_cast<const uint32_t*>(row + 4 * jj);
-      x0 = bf16lo(w); x1 = bf16hi(w);
+      const uint32_t u = *reinterpret_cast<const uint32_t*>(row + 4 * jj);
+      x0 = bf16lo(u); x1 = bf16hi(u);
     } else {
-      const float2 w = *reinterpret_cast<const float2*>(row + 8 * jj);
-      x0 = w.x; x1 = w.y;
+      const float2 u = *reinterpret_cast<const float2*>(row + 8 * jj);
+      x0 = u.x; x1 = u.y;
     }
-    if ((J.signs[j0 >> 5] >> (j0 & 31)) & 1u) x0 = -x0;
-    if ((J.signs[j1 >> 5] >> (j1 & 31)) & 1u) x1 = -x1;
+    if ((signs[j0 >> 5] >> (j0 & 31)) & 1u) x0 = -x0;
+    if ((signs[j1 >> 5] >> (j1 & 31)) & 1u) x1 = -x1;
     const bool neg = __popc((unsigned)(i & jj)) & 1;
     Ep += neg ? -(double)x0 : (double)x0;
     Op += neg ? -(double)x1 : (double)x1;
@@ -147,7 +120,7 @@ __device__ __noinline__ int exact_angle_code(const EncJob& J, const uint8_t* in,
   if (Ep == 0.0 && Op == 0.0) return 0;  // pair (0, 0) -> bin 0
   const float th = atan2f((float)(Ep - Op), (float)(Ep + Op));
   const int e = ((int)floorf(th * ((float)n * 0.15915494309189535f))) & (n - 1);
-  const cx::CS ab = g_edge_dir.v[tab_offset(J.w) + e];
+  const cx::CS ab = g_edge_dir.v[tab_offset(w) + e];
   const double m = fma(Ep, ab.c, -(Op * ab.s));
   return (e + (m >= 0.0 ? 1 : 0)) & (n - 1);
 }
@@ -161,11 +134,37 @@ __device__ __forceinline__ void patch_code(uint8_t* rec, int i, int W, int k) {
   }
 }
 
-// Encode one tile: this thread's 8 pairs of row r (lane l) of the staged tile.
-// W = log2 n, B = norm bits.
-template <int D, typename TIn, int W, int B>
-__device__ __forceinline__ void tile_body(const EncJob& J, uint8_t* smem, const uint8_t* in, int nrows,
-                                          int tid, const uint2 (&msk)[8]) {
+// Alg. 1 bin of the pair (E, O) (butterfly halves, y = (E + O, E - O)) for
+// n = 2^W by the edge test: candidate edge from the arctangent polynomial, then
+// the sign of the cross product with the edge direction.  Returns k; m is the
+// signed cross product (its magnitude is the certification margin).
+template <int W>
+__device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et, float& m) {
+  constexpr int n = 1 << W;
+  constexpr float nb = (float)n * 0.15915494309189535f;  // bins per radian
+  constexpr float c1 = (0.78539816f + 0.273f) * nb;       // atan(t) ~ t (pi/4 + 0.273 (1 - t))
+  constexpr float c2 = 0.273f * nb;
+  const float aE = fabsf(E), aO = fabsf(O);
+  const float mx = fmaxf(aE, aO), mn = fminf(aE, aO);
+  const float t = mn * rcp_approx(mx);
+  const float phi = t * __fmaf_rn(t, -c2, c1);                 // octant angle, bins
+  float fb = (aO > aE) ? (0.25f * n - phi) : phi;              // angle of (|E|, |O|)
+  fb = (E < 0.f) ? (0.5f * n - fb) : fb;                       // angle of (E, |O|)
+  const float ab = __uint_as_float(__float_as_uint(fb) ^ (__float_as_uint(O) & 0x80000000u));
+  // theta = pi/4 - angle(E, O): round(v - 1/2) is the candidate edge index
+  const float vm = (0.125f * n - 0.5f) - ab;
+  const int e = __float_as_int(vm + 12582912.0f) & (n - 1);
+  const float2 dir = et[e];
+  m = __fmaf_rn(E, dir.x, -__fmul_rn(O, dir.y));
+  return (uint32_t)(e + 1 + (__float_as_int(m) >> 31)) & (uint32_t)(n - 1);
+}
+
+// Encode this lane's 8 pairs of warp-tile row r (lane l of the row) and stage
+// the records; W = log2 n, B = norm bits, MODE = TAC_NORM_LINEAR / TAC_NORM_LOG.
+template <int D, typename TIn, int W, int B, int MODE>
+__device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const float2* etab, int nrows,
+                                          int lane, const uint2 (&msk)[8], const uint32_t* signs) {
+  // (for bf16 only msk[m].x is used; the .y words are constant zero)
   using C = Enc<D, TIn>;
   using G = Geo<D>;
   using IT = typename C::IT;
@@ -174,40 +173,40 @@ __device__ __forceinline__ void tile_body(const EncJob& J, uint8_t* smem, const 
   constexpr int AB = P * W / 8;           // angle record bytes
   constexpr int NB = P * B / 8;           // norm record bytes
   constexpr int Lq = (1 << B) - 1;
-  const int r = tid / L, l = tid % L;
+  const int r = lane / L, l = lane % L;
   const bool live = r < nrows;
 
   // ---- load 8 pairs (i = l + L*m), apply D, widen ----
   float2 v[8];
   {
-    const uint8_t* row = in + r * IT::STRIDE;
+    const uint8_t* row = in + r * IT::STRIDE + 2 * C::ESZ * l;
 #pragma unroll
     for (int m = 0; m < 8; ++m) {
-      const int i = l + L * m;
       if constexpr (C::ESZ == 2) {
-        const uint32_t w = *reinterpret_cast<const uint32_t*>(row + 4 * i) ^ msk[m].x;
-        v[m] = make_float2(bf16lo(w), bf16hi(w));
+        const uint32_t u = *reinterpret_cast<const uint32_t*>(row + 4 * L * m) ^ msk[m].x;
+        v[m] = make_float2(bf16lo(u), bf16hi(u));
       } else {
-        const uint2 w = *reinterpret_cast<const uint2*>(row + 8 * i);
-        v[m] = make_float2(__uint_as_float(w.x ^ msk[m].x), __uint_as_float(w.y ^ msk[m].y));
+        const uint2 u = *reinterpret_cast<const uint2*>(row + 8 * L * m);
+        v[m] = make_float2(__uint_as_float(u.x ^ msk[m].x), __uint_as_float(u.y ^ msk[m].y));
       }
     }
   }
   // ---- phase A: butterfly over pair-index bits log2(L)..log2(L)+2 ----
   butterfly8<8>(v);
-  // ---- transpose within the warp: lane l now owns pairs 8l..8l+7 ----
-  uint8_t* tpb = smem + C::OFF_TP;
   if constexpr (L > 1) {
+    // ---- transpose within the warp: lane l now owns pairs 8l..8l+7 ----
+    uint8_t* tpr = wsm + C::W_TP + r * G::ST;
 #pragma unroll
-    for (int m = 0; m < 8; ++m) *reinterpret_cast<float2*>(tpb + G::tp(r, l + L * m)) = v[m];
+    for (int m = 0; m < 8; ++m) *reinterpret_cast<float2*>(tpr + m * G::SM + 8 * l) = v[m];
     __syncwarp();
+    const uint8_t* tpl = tpr + (8 / L) * l * G::SM;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      const float4 t = *reinterpret_cast<const float4*>(tpb + G::tp(r, 8 * l + 2 * q));
+      const float4 t = *reinterpret_cast<const float4*>(tpl + G::tp_pair(2 * q));
       v[2 * q] = make_float2(t.x, t.y);
       v[2 * q + 1] = make_float2(t.z, t.w);
     }
-    // ---- phase B: butterfly over pair-index bits 0..log2(L)-1 (phase A did the rest) ----
+    // ---- phase B: butterfly over pair-index bits 0..log2(L)-1 ----
     butterfly8<L>(v);
   }
 
@@ -215,7 +214,8 @@ __device__ __forceinline__ void tile_body(const EncJob& J, uint8_t* smem, const 
   float s[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) s[j] = __fmaf_rn(v[j].x, v[j].x, __fmul_rn(v[j].y, v[j].y));
-  float smin = min3(min3(s[0], s[1], s[2]), min3(s[3], s[4], s[5]), fminf(s[6], s[7]));
+  const float lmin_s = min3(min3(s[0], s[1], s[2]), min3(s[3], s[4], s[5]), fminf(s[6], s[7]));
+  float smin = lmin_s;
   float smax = max3(max3(s[0], s[1], s[2]), max3(s[3], s[4], s[5]), fmaxf(s[6], s[7]));
 #pragma unroll
   for (int off = 1; off < L; off <<= 1) {
@@ -224,25 +224,29 @@ __device__ __forceinline__ void tile_body(const EncJob& J, uint8_t* smem, const 
   }
   const bool zero_row = !(smax > 0.f);
 
-  // ---- row constants: stored header (Sec. 3.3), Eq. 2 scale, certification bound ----
-  const float k2 = 2.0f / (float)D;
-  float hmin, hmax, qscale, qbase, sfloor = 0.f;
-  if (J.mode == TAC_NORM_LINEAR) {
+  // ---- row constants: stored header (Sec. 3.3), Eq. 2 as code = floor(f(s) qs + qo) ----
+  constexpr float k2 = 2.0f / (float)D;
+  float hmin, hmax, qs, qo, sfloor = 0.f;
+  if constexpr (MODE == TAC_NORM_LINEAR) {
     hmin = sqrt_approx(smin * k2);
     hmax = sqrt_approx(smax * k2);
-    qscale = (float)Lq * rcp_approx(hmax - hmin);
-    qbase = hmin;
-  } else {  // log-space: norms floored at 2^-24 r_max
-    sfloor = smax * 3.5527136788005009e-15f;  // 2^-48 on the energy
+    const float sc = (float)Lq * rcp_approx(hmax - hmin);
+    qs = sc * sqrt_approx(k2);                  // f(s) = sqrt(s)
+    qo = __fmaf_rn(-hmin, sc, 0.5f);
+    if (!(hmax > hmin) || !(sc <= 3.0e38f)) { qs = 0.f; qo = 0.5f; }
+  } else {  // log-space, norms floored at 2^-24 r_max
+    sfloor = smax * 3.5527136788005009e-15f;    // 2^-48 on the energy
     hmin = sqrt_approx(fmaxf(smin, sfloor) * k2);
     hmax = sqrt_approx(smax * k2);
     const float lmin = lg2_approx(hmin);
-    qscale = (float)Lq * rcp_approx(lg2_approx(hmax) - lmin);
-    qbase = lmin;
+    const float sc = (float)Lq * rcp_approx(lg2_approx(hmax) - lmin);
+    qs = 0.5f * sc;                             // f(s) = log2 s; log2 r = (log2 s + log2 k2)/2
+    qo = __fmaf_rn(0.5f * (float)(G::LOGD == 4 ? -3 : G::LOGD == 5 ? -4 : G::LOGD == 6 ? -5 : -6) - lmin,
+                   sc, 0.5f);
+    if (!(hmax > hmin) || !(sc <= 3.0e38f)) { qs = 0.f; qo = 0.5f; }
   }
-  if (!(hmax > hmin) || !(qscale <= 3.0e38f)) qscale = 0.f;
-  // |dE|, |dO| <= (log2 d - 1) u ||x||_1 with ||x||_1 <= sqrt(d) ||x||_2 <= sqrt(d smax);
-  // edge direction (1 ulp), product and fma add <= 4 u (|E| + |O|) <= 4 u sqrt(2 smax).
+  // Certification bound: |dE|, |dO| <= (log2 d - 1) u ||x||_1, ||x||_1 <= sqrt(d smax);
+  // edge direction (<= 1 ulp), product and fma add <= 4 u (|E| + |O|) <= 4 u sqrt(2 smax).
   const float rmx = sqrt_approx(smax);
   const float ty = (float)(G::LOGD - 1) * kU * 1.002f * sqrt_approx((float)D) * rmx;
   const float tau = ty + 5.f * kU * 1.4143f * rmx;
@@ -252,93 +256,103 @@ __device__ __forceinline__ void tile_body(const EncJob& J, uint8_t* smem, const 
   const float sthr = rthr * rthr;
 
   // ---- pass 2: angle codes (Alg. 1), norm codes (Eq. 2), packing ----
-  const float2* et = reinterpret_cast<const float2*>(smem + C::OFF_TAB) + tab_offset(W);
-  const float nb = (float)n * 0.15915494309189535f;  // bins per radian
-  const float c1 = (0.78539816f + 0.273f) * nb;       // atan(t) ~ t (pi/4 + 0.273 (1 - t))
-  const float c2 = 0.273f * nb;
-  uint64_t acc_a = 0, acc_n = 0;
-  uint32_t fm = 0;
+  const float2* et = etab + tab_offset(W);
+  uint32_t alo = 0, ahi = 0, nlo = 0, nhi = 0;
+  float mmin = __int_as_float(0x7f800000);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    const float E = v[j].x, O = v[j].y;
-    const float aE = fabsf(E), aO = fabsf(O);
-    const float mx = fmaxf(aE, aO), mn = fminf(aE, aO);
-    const float t = mn * rcp_approx(mx);
-    const float phi = t * __fmaf_rn(t, -c2, c1);                 // octant angle, bins
-    float fb = (aO > aE) ? (0.25f * n - phi) : phi;              // angle of (|E|, |O|)
-    fb = (E < 0.f) ? (0.5f * n - fb) : fb;                       // angle of (E, |O|)
-    const float ab = __uint_as_float(__float_as_uint(fb) ^ (__float_as_uint(O) & 0x80000000u));
-    // theta = pi/4 - angle(E, O): candidate v - 1/2 rounded to an integer edge index
-    const float vm = (0.125f * n - 0.5f) - ab;
-    const int e = (__float_as_int(vm + 12582912.0f) - 0x4B400000) & (n - 1);
-    const float2 dir = et[e];
-    const float m = __fmaf_rn(E, dir.x, -__fmul_rn(O, dir.y));
-    const int k = (e + 1 + (__float_as_int(m) >> 31)) & (n - 1);
-    if (fabsf(m) < tau) fm |= 1u << j;
-    float val;
-    if (J.mode == TAC_NORM_LINEAR) val = sqrt_approx(s[j] * k2);
-    else val = 0.5f * lg2_approx(fmaxf(s[j], sfloor) * k2);
-    int c = __float2int_rd(__fmaf_rn(val - qbase, qscale, 0.5f));
-    c = min(max(c, 0), Lq);
-    acc_a |= (uint64_t)(uint32_t)k << (j * W);
-    acc_n |= (uint64_t)(uint32_t)c << (j * B);
+    float m;
+    const uint32_t k = edge_test<W>(v[j].x, v[j].y, et, m);
+    mmin = fminf(mmin, fabsf(m));
+    float f;
+    if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_approx(s[j]);
+    else f = lg2_approx(fmaxf(s[j], sfloor));
+    const uint32_t c = min(__float2uint_rd(__fmaf_rn(f, qs, qo)), (uint32_t)Lq);
+    const int sa = j * W, sn = j * B;
+    if (sa + W <= 32) alo |= k << sa;
+    else if (sa >= 32) ahi |= k << (sa - 32);
+    else { alo |= k << sa; ahi |= k >> (32 - sa); }
+    if (sn < 32) nlo |= c << sn; else nhi |= c << (sn - 32);
   }
-  if (zero_row) { acc_a = 0; acc_n = 0; fm = 0; hmin = 0.f; hmax = 0.f; }
-  else if (smin < sthr) {
+  uint32_t fm = 0;
+  if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; }
+  else if (mmin < tau || lmin_s < sthr) {  // rare: name the uncertified pairs
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
-      if (s[j] < sthr) fm |= 1u << j;
+    for (int j = 0; j < 8; ++j) {
+      float m;
+      edge_test<W>(v[j].x, v[j].y, et, m);
+      if (fabsf(m) < tau || s[j] < sthr) fm |= 1u << j;
+    }
   }
   if (!live) fm = 0;
 
   // ---- stage the records ----
   if (live) {
-    store_bytes<W>(smem + C::OFF_ANG + r * AB + l * W, acc_a);
-    store_bytes<B>(smem + C::OFF_NRM + r * NB + l * B, acc_n);
-    if (l == 0) reinterpret_cast<float2*>(smem + C::OFF_HDR)[r] = make_float2(hmin, hmax);
+    store_bytes<W>(wsm + C::W_ANG + r * AB + l * W, alo, ahi);
+    store_bytes<B>(wsm + C::W_NRM + r * NB + l * B, nlo, nhi);
+    if (l == 0) reinterpret_cast<float2*>(wsm + C::W_HDR)[r] = make_float2(hmin, hmax);
   }
   __syncwarp();
 
   // ---- exact re-decision of the uncertified pairs, one warp per pair ----
-  const int lane = tid & 31;
-  const int wtid0 = tid & ~31;
   unsigned ball = __ballot_sync(0xffffffffu, fm != 0u);
   while (ball) {
     const int owner = __ffs(ball) - 1;
     ball &= ball - 1;
     uint32_t mm = __shfl_sync(0xffffffffu, fm, owner);
-    const int otid = wtid0 + owner;
-    const int rr = otid / L, ol = otid % L;
+    const int rr = owner / L, ol = owner % L;
     while (mm) {
       const int j = __ffs(mm) - 1;
       mm &= mm - 1;
       const int i = 8 * ol + j;
-      const int k = exact_angle_code<D, TIn>(J, in, rr, i, lane);
-      if (lane == 0) patch_code(smem + C::OFF_ANG + rr * AB, i, W, k);
+      const int kk = exact_angle_code<D, TIn>(signs, W, in, rr, i, lane);
+      if (lane == 0) patch_code(wsm + C::W_ANG + rr * AB, i, W, kk);
     }
     __syncwarp();
   }
 }
 
-template <int D, typename TIn, int W, int B>
-__device__ __forceinline__ void copy_tile_out(const EncJob& J, const uint8_t* smem, int row0, int nrows,
-                                              int tid) {
-  using C = Enc<D, TIn>;
-  constexpr int P = C::P;
-  constexpr int AB = P * W / 8;
-  constexpr int NB = P * B / 8;
-  if (J.slot == nullptr) {
-    cta_copy_out(J.codes + (int64_t)row0 * AB, smem + C::OFF_ANG, nrows * AB, tid);
-    cta_copy_out(J.norms + (int64_t)row0 * NB, smem + C::OFF_NRM, nrows * NB, tid);
-    cta_copy_out(J.hdr + (int64_t)row0 * 8, smem + C::OFF_HDR, nrows * 8, tid);
-  } else {
-    for (int rr = tid; rr < nrows; rr += kThreads) {
-      const int64_t s = J.slot[row0 + rr];
-      if (s < 0 || s >= J.capacity) continue;  // out-of-range slots are skipped
-      copy_record<AB>(J.codes + s * AB, smem + C::OFF_ANG + rr * AB);
-      copy_record<NB>(J.norms + s * NB, smem + C::OFF_NRM + rr * NB);
-      reinterpret_cast<float2*>(J.hdr)[s] = reinterpret_cast<const float2*>(smem + C::OFF_HDR)[rr];
+// Write the warp tile's staged records (nrows rows from row0) to the planes.
+__device__ __forceinline__ void warp_copy_out(uint8_t* codes, uint8_t* norms, uint8_t* hdr, const int64_t* slot,
+                                              int64_t capacity, const uint8_t* sang, const uint8_t* snrm,
+                                              const uint8_t* shdr, int64_t row0, int nrows, int RW, int AB, int NB,
+                                              int lane) {
+  if (slot == nullptr) {
+    uint8_t* ga = codes + row0 * AB;
+    uint8_t* gn = norms + row0 * NB;
+    uint8_t* gh = hdr + row0 * 8;
+    if (nrows == RW) {  // full tile: each plane segment is a 16-byte multiple (32 w, 32 b, 8 RW bytes)
+      const int na = RW * AB / 16, nn = RW * NB / 16, nh = RW / 2;
+      if (lane < na) reinterpret_cast<uint4*>(ga)[lane] = reinterpret_cast<const uint4*>(sang)[lane];
+      if (lane < nn) reinterpret_cast<uint4*>(gn)[lane] = reinterpret_cast<const uint4*>(snrm)[lane];
+      if (lane < nh) reinterpret_cast<uint4*>(gh)[lane] = reinterpret_cast<const uint4*>(shdr)[lane];
+    } else {
+      for (int q = lane; q < nrows * AB; q += 32) ga[q] = sang[q];
+      for (int q = lane; q < nrows * NB; q += 32) gn[q] = snrm[q];
+      for (int q = lane; q < nrows * 8; q += 32) gh[q] = shdr[q];
     }
+  } else if (lane < nrows) {
+    const int64_t s = slot[row0 + lane];
+    if (s < 0 || s >= capacity) return;  // out-of-range slots are skipped
+    uint8_t* ga = codes + s * AB;
+    uint8_t* gn = norms + s * NB;
+    const uint8_t* a = sang + lane * AB;
+    const uint8_t* nn = snrm + lane * NB;
+    if ((AB & 15) == 0) {
+      for (int q = 0; q < AB / 16; ++q) reinterpret_cast<uint4*>(ga)[q] = reinterpret_cast<const uint4*>(a)[q];
+    } else if ((AB & 7) == 0) {
+      for (int q = 0; q < AB / 8; ++q) reinterpret_cast<uint2*>(ga)[q] = reinterpret_cast<const uint2*>(a)[q];
+    } else if ((AB & 3) == 0) {
+      for (int q = 0; q < AB / 4; ++q) reinterpret_cast<uint32_t*>(ga)[q] = reinterpret_cast<const uint32_t*>(a)[q];
+    } else {
+      for (int q = 0; q < AB; ++q) ga[q] = a[q];
+    }
+    if ((NB & 7) == 0) {
+      for (int q = 0; q < NB / 8; ++q) reinterpret_cast<uint2*>(gn)[q] = reinterpret_cast<const uint2*>(nn)[q];
+    } else {
+      for (int q = 0; q < NB / 4; ++q) reinterpret_cast<uint32_t*>(gn)[q] = reinterpret_cast<const uint32_t*>(nn)[q];
+    }
+    reinterpret_cast<float2*>(hdr)[s] = reinterpret_cast<const float2*>(shdr)[lane];
   }
 }
 
@@ -348,85 +362,109 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
   using IT = typename C::IT;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
-  const int G = gridDim.x;
-  int t = blockIdx.x;
-  if (t >= p.ntiles) return;
+  const int warp = tid >> 5, lane = tid & 31;
 
-  // Edge tables for every n = 2..256.
+  // fp32 edge tables for every n = 2..256 (shared by the CTA).
   float2* etab = reinterpret_cast<float2*>(smem + C::OFF_TAB);
   for (int idx = tid; idx < kTabEntries - 2; idx += kThreads) {
     const int w = 31 - __clz(idx + 2);
     const int e = idx - tab_offset(w);
     etab[idx] = cos_sin_q8(edge_q8(e, 1 << w), 1 << w);
   }
+  __syncthreads();
 
-  int jid = find_job(p, t);
-  int mask_jid = -1;
-  uint2 msk[8];
-  // Prologue: kStages - 1 tiles in flight (one cp.async group per tile, possibly empty).
+  const int Gw = gridDim.x * kWarps;
+  int t = blockIdx.x * kWarps + warp;
+  if (t >= p.ntiles) return;
+  uint8_t* wsm = smem + warp * C::WARP_B;
+
+
+  // Prefetch cursor (job of the next warp tile to load) and its registers.
+  int pj = find_job(p, t);
+  int p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
+  int p_t0 = p.job[pj].tile0;
+  const uint8_t* p_x = reinterpret_cast<const uint8_t*>(p.job[pj].x);
+  int64_t p_rows = p.job[pj].rows, p_sb = p.job[pj].stride * C::ESZ;
+  auto issue = [&](int tt, int stg) {
+    if (tt < p.ntiles) {
+      while (tt >= p_end) {  // monotone: a warp's tiles only move forward
+        ++pj;
+        p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
+        p_t0 = p.job[pj].tile0;
+        p_x = reinterpret_cast<const uint8_t*>(p.job[pj].x);
+        p_rows = p.job[pj].rows;
+        p_sb = p.job[pj].stride * C::ESZ;
+      }
+      const int64_t row0 = (int64_t)(tt - p_t0) * C::RW;
+      uint8_t* dst = wsm + C::W_IN + stg * IT::BYTES;
 #pragma unroll
-  for (int s = 0; s < kStages - 1; ++s) {
-    const int ts = t + s * G;
-    if (ts < p.ntiles) {
-      const EncJob& Js = p.job[find_job(p, ts)];
-      issue_tile_load<D, TIn>(Js, (ts - Js.tile0) * C::TR, smem + C::OFF_IN + s * IT::BYTES, tid);
+      for (int q = 0; q < IT::CHUNKS; ++q) {
+        const int id = q * 32 + lane;            // chunk id -> (row, column) of the warp tile
+        const int cr = id / IT::CPR, ccol = (id % IT::CPR) * 16;
+        const int64_t row = row0 + cr;
+        const bool ok = row < p_rows;
+        cp_async16(dst + cr * IT::STRIDE + ccol, ok ? p_x + row * p_sb + ccol : p_x, ok ? 16 : 0);
+      }
     }
     cp_async_commit();
-  }
+  };
+#pragma unroll
+  for (int s = 0; s < kNS - 1; ++s) issue(t + s * Gw, s);
 
-  int cur = 0;
-  for (; t < p.ntiles; t += G) {
-    cp_async_wait<kStages - 2>();   // this tile's group has landed
-    __syncthreads();                // ... and every thread is done with the previous tile
+  // Compute cursor: the current job lives in the warp's shared region.
+  WarpJob* wj = reinterpret_cast<WarpJob*>(wsm + C::W_JOB);
+  int cj = -1, c_end = 0;
+  uint2 msk[8];
+#pragma unroll
+  for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
+
+  int stage = 0;
+  for (; t < p.ntiles; t += Gw) {
+    cp_async_wait<kNS - 2>();   // this warp tile has landed
+    __syncwarp();               // ... and every lane is done with the previous one
     {
-      // Refill the buffer of the previous tile with the tile kStages - 1 ahead.
-      const int tn = t + (kStages - 1) * G;
-      int nb = cur + kStages - 1;
-      if (nb >= kStages) nb -= kStages;
-      if (tn < p.ntiles) {
-        const EncJob& Jn = p.job[find_job(p, tn)];
-        issue_tile_load<D, TIn>(Jn, (tn - Jn.tile0) * C::TR, smem + C::OFF_IN + nb * IT::BYTES, tid);
-      }
-      cp_async_commit();
+      int ns = stage + kNS - 1;
+      if (ns >= kNS) ns -= kNS;
+      issue(t + (kNS - 1) * Gw, ns);
     }
-    const EncJob& J = p.job[jid];
-    if (jid != mask_jid) {
-      const int l = tid % C::L;
+    if (t >= c_end) {  // next job: copy its descriptor to shared memory
+      cj = (cj < 0) ? find_job(p, t) : cj + 1;
+      while (cj + 1 < p.njobs && p.job[cj + 1].tile0 <= t) ++cj;
+      const EncJob& J = p.job[cj];
+      c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
+      if (lane == 0) {
+        wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot;
+        wj->capacity = J.capacity; wj->rows = J.rows; wj->t0 = J.tile0; wj->end = c_end;
+        wj->variant = (J.w - 1) * 4 + (J.b == 8 ? 2 : 0) + (J.mode == TAC_NORM_LOG ? 1 : 0);
+        wj->ab = C::P * J.w / 8; wj->nb = C::P * J.b / 8;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) wj->signs[q] = J.signs[q];
+      }
+      const int l = lane % C::L;
 #pragma unroll
       for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
-      mask_jid = jid;
+      __syncwarp();
     }
-    const int row0 = (t - J.tile0) * C::TR;
-    const int nrows = (int)min((int64_t)C::TR, J.rows - row0);
-    const uint8_t* in = smem + C::OFF_IN + cur * IT::BYTES;
+    const int64_t row0 = (int64_t)(t - wj->t0) * C::RW;
+    const int nrows = (int)min((int64_t)C::RW, wj->rows - row0);
+    const int variant = wj->variant;
+    const uint8_t* in = wsm + C::W_IN + stage * IT::BYTES;
 
-#define TAC_ENC_CASE(WW)                                                          \
-  case WW:                                                                        \
-    if (J.b == 8) tile_body<D, TIn, WW, 8>(J, smem, in, nrows, tid, msk);         \
-    else tile_body<D, TIn, WW, 4>(J, smem, in, nrows, tid, msk);                  \
-    break;
-    switch (J.w) {
+#define TAC_ENC_CASE(WW)                                                                                       \
+  case (WW - 1) * 4 + 0: tile_body<D, TIn, WW, 4, TAC_NORM_LINEAR>(in, wsm, etab, nrows, lane, msk, wj->signs); break; \
+  case (WW - 1) * 4 + 1: tile_body<D, TIn, WW, 4, TAC_NORM_LOG>(in, wsm, etab, nrows, lane, msk, wj->signs); break;    \
+  case (WW - 1) * 4 + 2: tile_body<D, TIn, WW, 8, TAC_NORM_LINEAR>(in, wsm, etab, nrows, lane, msk, wj->signs); break; \
+  case (WW - 1) * 4 + 3: tile_body<D, TIn, WW, 8, TAC_NORM_LOG>(in, wsm, etab, nrows, lane, msk, wj->signs); break;
+    switch (variant) {
       TAC_ENC_CASE(1) TAC_ENC_CASE(2) TAC_ENC_CASE(3) TAC_ENC_CASE(4)
       TAC_ENC_CASE(5) TAC_ENC_CASE(6) TAC_ENC_CASE(7) TAC_ENC_CASE(8)
       default: break;
     }
 #undef TAC_ENC_CASE
-    __syncthreads();
-
-#define TAC_OUT_CASE(WW)                                                          \
-  case WW:                                                                        \
-    if (J.b == 8) copy_tile_out<D, TIn, WW, 8>(J, smem, row0, nrows, tid);        \
-    else copy_tile_out<D, TIn, WW, 4>(J, smem, row0, nrows, tid);                 \
-    break;
-    switch (J.w) {
-      TAC_OUT_CASE(1) TAC_OUT_CASE(2) TAC_OUT_CASE(3) TAC_OUT_CASE(4)
-      TAC_OUT_CASE(5) TAC_OUT_CASE(6) TAC_OUT_CASE(7) TAC_OUT_CASE(8)
-      default: break;
-    }
-#undef TAC_OUT_CASE
-
-    if (t + G < p.ntiles) jid = find_job(p, t + G);
-    cur = (cur + 1 == kStages) ? 0 : cur + 1;
+    __syncwarp();
+    warp_copy_out(wj->codes, wj->norms, wj->hdr, wj->slot, wj->capacity, wsm + C::W_ANG, wsm + C::W_NRM,
+                  wsm + C::W_HDR, row0, nrows, C::RW, wj->ab, wj->nb, lane);
+    stage = (stage + 1 == kNS) ? 0 : stage + 1;
   }
   cp_async_wait<0>();
 }
@@ -451,7 +489,8 @@ static cudaError_t launch_encode_t(const EncParams& p, int grid_cap, cudaStream_
   if (e != cudaSuccess) return e;
   if (per_sm < 1) per_sm = 1;
   int grid = grid_cap * per_sm;
-  if (grid > p.ntiles) grid = p.ntiles;
+  const int need = (p.ntiles + kWarps - 1) / kWarps;
+  if (grid > need) grid = need;
   if (grid < 1) return cudaSuccess;
   kern<<<grid, kThreads, C::SMEM, st>>>(p);
   return cudaGetLastError();
