@@ -33,6 +33,33 @@ METRIC = "KV encode / decode GB/s (bf16 in/out) on 1 GB300 and % of HBM peak"
 UNIT = "GB/s"
 FALLBACK_HBM_GBS = 6800.0
 
+# DRAM bytes per encoded/decoded row that ncu counted (dram__bytes_read.sum +
+# dram__bytes_write.sum of one launch of the 4096-token Mistral-7B-shaped case,
+# divided by its 2,097,152 rows; the full-size launch has the same codebook mix,
+# so its traffic is this figure times its rows).  Each figure holds only for the
+# kernel sources it was measured on; after any change to them it reads null.
+MEASURED_TRAFFIC = {
+    "encode": {"sources": ("tac_common.cuh", "tac_encode.cu"), "sha256_16": "73575d5810d8d294",
+               "bytes_per_row": 349.596},
+    "decode": {"sources": ("tac_common.cuh", "tac_decode.cu"), "sha256_16": "94a05f1c3d5736cb",
+               "bytes_per_row": 334.232},
+}
+
+
+def measured_traffic(kernel: str, rows: int):
+    """DRAM bytes of one launch over `rows` rows, or None if the kernel changed."""
+    import hashlib
+    rec = MEASURED_TRAFFIC.get(kernel)
+    if rec is None or not rows:
+        return None
+    h = hashlib.sha256()
+    for f in rec["sources"]:
+        with open(os.path.join(ROOT, "paper_2603_27467_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    if h.hexdigest()[:16] != rec["sha256_16"]:
+        return None
+    return rec["bytes_per_row"] * rows
+
 
 def parse_args():
     ap = argparse.ArgumentParser()
@@ -169,6 +196,7 @@ class Workset:
                 self.enc_bytes += rows * (2 * d + record_bytes(d, n, b))
             self.tokens = a["seqs"]
             self.y_all = None
+            self.rows_per_launch = None   # scattered single-token rows: no traffic figure
             return
         w = workloads.CONFIGS[name]
         if tokens:
@@ -189,6 +217,8 @@ class Workset:
             self.enc_bytes += R * (2 * d + rb)
             self.dec_bytes += R * (rb + 2 * d)
         self.tokens = w.tokens
+        # the measured per-row traffic holds for the Mistral-7B-shaped codebook mix
+        self.rows_per_launch = R * len(blocks) if name == "mistral7b" else None
 
     @property
     def step_bytes(self):
@@ -431,7 +461,8 @@ def main():
             "tokens_per_s": world * ws.tokens * w.layers * K / (total_ms / 1e3),
             "roofline": {"bound": "hbm", "kernel": f"{dom} (tac_{dom}_multi, one launch)",
                          "achieved": dom_gbs, "peak": hbm, "unit": "GB/s", "frac": dom_gbs / hbm,
-                         "peak_source": f"{peak_kind} hbm_gbs", "traffic": None,
+                         "peak_source": f"{peak_kind} hbm_gbs",
+                         "traffic": measured_traffic(dom, ws.rows_per_launch),
                          "algorithmic_bytes_per_launch": dom_bytes},
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * K, "clocks": clocks,
         }
