@@ -399,7 +399,7 @@ def main():
     enc_ms = [e[0].elapsed_time(e[1]) for e in ev]
     dec_ms = [e[1].elapsed_time(e[2]) for e in ev] if not enc_only else [0.0]
     total_ms = max_over_ranks(total_ms, world, dev)
-    launches_per_step = (1 if enc_only else 2) * (1 + (len(ws.enc_jobs) - 1) // 96)
+    launches_per_step = tac.launch_count(ws.enc_jobs) + (0 if enc_only else tac.launch_count(ws.dec_jobs))
 
     step_bytes = ws.enc_bytes + (0 if enc_only else ws.dec_bytes)
     value = job_throughput(world, step_bytes, K, total_ms)

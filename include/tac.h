@@ -146,14 +146,15 @@ int tac_decode(const void* codes, const void* norms, const tac_layer_cfg* cfg, t
                tac_stream_t stream);
 
 /*
- * Batched encode: every job in one launch (one per TAC_MAX_JOBS jobs).  Jobs may
- * mix codebooks, d and input dtypes of the same d; with `slot` the rows of a decode
- * step land at per-sequence record slots (streaming append).  Jobs must not write
- * overlapping slots.
+ * Batched encode.  Jobs may mix d, input dtypes and codebooks; jobs that share
+ * the kernel shape (d, dtype, n_angle, norm_bits, norm_mode) run in one launch
+ * (one per TAC_MAX_JOBS such jobs), the groups run back to back on `stream`.
+ * With `slot` the rows of a decode step land at per-sequence record slots
+ * (streaming append).  Jobs must not write overlapping slots.
  */
 int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream);
 
-/* Batched decode: every job in one launch (one per TAC_MAX_JOBS jobs). */
+/* Batched decode, grouped into launches like tac_encode_multi. */
 int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream);
 
 /*

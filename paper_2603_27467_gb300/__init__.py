@@ -30,6 +30,7 @@ TAC_OK, TAC_E_INVAL, TAC_E_UNSUPPORTED, TAC_E_CUDA = 0, 1, 2, 3
 NORM_LINEAR, NORM_LOG = 0, 1
 BF16, FP32 = 0, 1
 MAX_D = 128
+MAX_JOBS = 96  # TAC_MAX_JOBS: jobs per kernel launch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "_build", "libtac.so")
@@ -306,7 +307,7 @@ def decode(cache: Cache, cfg: LayerCfg, rows: int | None = None, dtype=None, y=N
 
 
 def encode_multi(jobs, stream=None) -> None:
-    """tac_encode_multi: every job in one launch per (d, dtype) group."""
+    """tac_encode_multi: one launch per kernel group (see launch_count)."""
     arr = (_EncJob * max(1, len(jobs)))()
     for i, j in enumerate(jobs):
         e = arr[i]
@@ -320,7 +321,7 @@ def encode_multi(jobs, stream=None) -> None:
 
 
 def decode_multi(jobs, stream=None) -> None:
-    """tac_decode_multi: every job in one launch per (d, dtype) group."""
+    """tac_decode_multi: one launch per kernel group (see launch_count)."""
     arr = (_DecJob * max(1, len(jobs)))()
     for i, j in enumerate(jobs):
         e = arr[i]
@@ -331,6 +332,20 @@ def decode_multi(jobs, stream=None) -> None:
         e.slot = j.slot.data_ptr() if j.slot is not None else None
         e.y = _rows(j.y, j.cfg.d)
     _check(load().tac_decode_multi(arr, len(jobs), _stream_ptr(stream)))
+
+
+def launch_count(jobs) -> int:
+    """Kernel launches one encode_multi / decode_multi call makes for `jobs`:
+    jobs with rows are grouped by kernel (d, dtype, n, norm bits, norm mode),
+    at most MAX_JOBS jobs per launch."""
+    groups: dict = {}
+    for j in jobs:
+        t = j.x if isinstance(j, EncodeJob) else j.y
+        if t.shape[0] == 0:
+            continue
+        key = (j.cfg.d, str(t.dtype), j.cfg.n_angle, j.cfg.norm_bits, j.cfg.norm_mode)
+        groups[key] = groups.get(key, 0) + 1
+    return sum(-(-c // MAX_JOBS) for c in groups.values())
 
 
 def fwht_debug(x, signs: np.ndarray, d: int, stream=None):

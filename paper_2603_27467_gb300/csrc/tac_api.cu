@@ -12,41 +12,59 @@
 #include "tac_common.cuh"
 
 namespace tac {
-cudaError_t launch_encode_16_bf16(const EncParams& p, int sms, cudaStream_t st);
-cudaError_t launch_encode_32_bf16(const EncParams& p, int sms, cudaStream_t st);
-cudaError_t launch_encode_64_bf16(const EncParams& p, int sms, cudaStream_t st);
-cudaError_t launch_encode_128_bf16(const EncParams& p, int sms, cudaStream_t st);
-cudaError_t launch_encode_16_f32(const EncParams& p, int sms, cudaStream_t st);
-cudaError_t launch_encode_32_f32(const EncParams& p, int sms, cudaStream_t st);
-cudaError_t launch_encode_64_f32(const EncParams& p, int sms, cudaStream_t st);
-cudaError_t launch_encode_128_f32(const EncParams& p, int sms, cudaStream_t st);
-cudaError_t launch_decode_16_bf16(const DecParams& p, int sms, cudaStream_t st);
-cudaError_t launch_decode_32_bf16(const DecParams& p, int sms, cudaStream_t st);
-cudaError_t launch_decode_64_bf16(const DecParams& p, int sms, cudaStream_t st);
-cudaError_t launch_decode_128_bf16(const DecParams& p, int sms, cudaStream_t st);
-cudaError_t launch_decode_16_f32(const DecParams& p, int sms, cudaStream_t st);
-cudaError_t launch_decode_32_f32(const DecParams& p, int sms, cudaStream_t st);
-cudaError_t launch_decode_64_f32(const DecParams& p, int sms, cudaStream_t st);
-cudaError_t launch_decode_128_f32(const DecParams& p, int sms, cudaStream_t st);
+cudaError_t launch_encode_16_bf16(const EncParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_encode_32_bf16(const EncParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_encode_64_bf16(const EncParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_encode_128_bf16(const EncParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_encode_16_f32(const EncParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_encode_32_f32(const EncParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_encode_64_f32(const EncParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_encode_128_f32(const EncParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_decode_16_bf16(const DecParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_decode_32_bf16(const DecParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_decode_64_bf16(const DecParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_decode_128_bf16(const DecParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_decode_16_f32(const DecParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_decode_32_f32(const DecParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_decode_64_f32(const DecParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
+cudaError_t launch_decode_128_f32(const DecParams& p, int w, int b, int mode, int sms,
+                                 cudaStream_t st);
 
-static cudaError_t launch_encode(int d, int dtype, const EncParams& p, int sms, cudaStream_t st) {
+static cudaError_t launch_encode(int d, int dtype, int w, int b, int mode, const EncParams& p, int sms,
+                                 cudaStream_t st) {
   const bool bf = dtype == TAC_BF16;
   switch (d) {
-    case 16: return bf ? launch_encode_16_bf16(p, sms, st) : launch_encode_16_f32(p, sms, st);
-    case 32: return bf ? launch_encode_32_bf16(p, sms, st) : launch_encode_32_f32(p, sms, st);
-    case 64: return bf ? launch_encode_64_bf16(p, sms, st) : launch_encode_64_f32(p, sms, st);
-    case 128: return bf ? launch_encode_128_bf16(p, sms, st) : launch_encode_128_f32(p, sms, st);
+    case 16: return bf ? launch_encode_16_bf16(p, w, b, mode, sms, st) : launch_encode_16_f32(p, w, b, mode, sms, st);
+    case 32: return bf ? launch_encode_32_bf16(p, w, b, mode, sms, st) : launch_encode_32_f32(p, w, b, mode, sms, st);
+    case 64: return bf ? launch_encode_64_bf16(p, w, b, mode, sms, st) : launch_encode_64_f32(p, w, b, mode, sms, st);
+    case 128: return bf ? launch_encode_128_bf16(p, w, b, mode, sms, st) : launch_encode_128_f32(p, w, b, mode, sms, st);
   }
   return cudaErrorInvalidValue;
 }
 
-static cudaError_t launch_decode(int d, int dtype, const DecParams& p, int sms, cudaStream_t st) {
+static cudaError_t launch_decode(int d, int dtype, int w, int b, int mode, const DecParams& p, int sms,
+                                 cudaStream_t st) {
   const bool bf = dtype == TAC_BF16;
   switch (d) {
-    case 16: return bf ? launch_decode_16_bf16(p, sms, st) : launch_decode_16_f32(p, sms, st);
-    case 32: return bf ? launch_decode_32_bf16(p, sms, st) : launch_decode_32_f32(p, sms, st);
-    case 64: return bf ? launch_decode_64_bf16(p, sms, st) : launch_decode_64_f32(p, sms, st);
-    case 128: return bf ? launch_decode_128_bf16(p, sms, st) : launch_decode_128_f32(p, sms, st);
+    case 16: return bf ? launch_decode_16_bf16(p, w, b, mode, sms, st) : launch_decode_16_f32(p, w, b, mode, sms, st);
+    case 32: return bf ? launch_decode_32_bf16(p, w, b, mode, sms, st) : launch_decode_32_f32(p, w, b, mode, sms, st);
+    case 64: return bf ? launch_decode_64_bf16(p, w, b, mode, sms, st) : launch_decode_64_f32(p, w, b, mode, sms, st);
+    case 128: return bf ? launch_decode_128_bf16(p, w, b, mode, sms, st) : launch_decode_128_f32(p, w, b, mode, sms, st);
   }
   return cudaErrorInvalidValue;
 }
@@ -249,18 +267,24 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
   const int sms = num_sms();
   if (live.empty()) return ok();
   if (sms <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
-  // Group by (d, dtype): one kernel instance per group, up to TAC_MAX_JOBS jobs per launch.
-  std::stable_sort(live.begin(), live.end(), [&](int a, int b) {
-    const int ka = jobs[a].cfg.d * 4 + jobs[a].x.dtype, kb = jobs[b].cfg.d * 4 + jobs[b].x.dtype;
-    return ka < kb;
-  });
+  // Group by kernel: (d, dtype, n, norm bits, norm mode); one launch per group
+  // and up to TAC_MAX_JOBS jobs per launch.
+  auto kernel_key = [&](int j) {
+    const tac_encode_job& J = jobs[j];
+    return (((J.cfg.d * 4 + J.x.dtype) * 16 + log2_exact(J.cfg.n_angle)) * 16 + J.cfg.norm_bits) * 4 +
+           J.cfg.norm_mode;
+  };
+  std::stable_sort(live.begin(), live.end(), [&](int a, int b) { return kernel_key(a) < kernel_key(b); });
   static thread_local tac::EncParams P;
   size_t i = 0;
   while (i < live.size()) {
-    const int d = jobs[live[i]].cfg.d, dt = jobs[live[i]].x.dtype;
+    const int key = kernel_key(live[i]);
+    const tac_layer_cfg& c0 = jobs[live[i]].cfg;
+    const int d = c0.d, dt = jobs[live[i]].x.dtype;
+    const int w = log2_exact(c0.n_angle), nb = c0.norm_bits, mode = c0.norm_mode;
     std::memset(&P, 0, sizeof(P));
     int64_t tiles = 0;
-    while (i < live.size() && P.njobs < TAC_MAX_JOBS && jobs[live[i]].cfg.d == d && jobs[live[i]].x.dtype == dt) {
+    while (i < live.size() && P.njobs < TAC_MAX_JOBS && kernel_key(live[i]) == key) {
       const tac_encode_job& J = jobs[live[i]];
       const int64_t tr = tile_rows(d);
       const int64_t jt = (J.x.rows + tr - 1) / tr;
@@ -285,7 +309,7 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
     }
     if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many rows", who);
     P.ntiles = (int32_t)tiles;
-    cudaError_t e = tac::launch_encode(d, dt, P, sms, reinterpret_cast<cudaStream_t>(stream));
+    cudaError_t e = tac::launch_encode(d, dt, w, nb, mode, P, sms, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
   }
   return ok();
@@ -316,17 +340,24 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
   const int sms = num_sms();
   if (live.empty()) return ok();
   if (sms <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
-  std::stable_sort(live.begin(), live.end(), [&](int a, int b) {
-    const int ka = jobs[a].cfg.d * 4 + jobs[a].y.dtype, kb = jobs[b].cfg.d * 4 + jobs[b].y.dtype;
-    return ka < kb;
-  });
+  // Group by kernel: (d, dtype, n, norm bits, norm mode); one launch per group
+  // and up to TAC_MAX_JOBS jobs per launch.
+  auto kernel_key = [&](int j) {
+    const tac_decode_job& J = jobs[j];
+    return (((J.cfg.d * 4 + J.y.dtype) * 16 + log2_exact(J.cfg.n_angle)) * 16 + J.cfg.norm_bits) * 4 +
+           J.cfg.norm_mode;
+  };
+  std::stable_sort(live.begin(), live.end(), [&](int a, int b) { return kernel_key(a) < kernel_key(b); });
   static thread_local tac::DecParams P;
   size_t i = 0;
   while (i < live.size()) {
-    const int d = jobs[live[i]].cfg.d, dt = jobs[live[i]].y.dtype;
+    const int key = kernel_key(live[i]);
+    const tac_layer_cfg& c0 = jobs[live[i]].cfg;
+    const int d = c0.d, dt = jobs[live[i]].y.dtype;
+    const int w = log2_exact(c0.n_angle), nb = c0.norm_bits, mode = c0.norm_mode;
     std::memset(&P, 0, sizeof(P));
     int64_t tiles = 0;
-    while (i < live.size() && P.njobs < TAC_MAX_JOBS && jobs[live[i]].cfg.d == d && jobs[live[i]].y.dtype == dt) {
+    while (i < live.size() && P.njobs < TAC_MAX_JOBS && kernel_key(live[i]) == key) {
       const tac_decode_job& J = jobs[live[i]];
       const int64_t tr = tile_rows(d);
       const int64_t jt = (J.y.rows + tr - 1) / tr;
@@ -351,7 +382,7 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
     }
     if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many rows", who);
     P.ntiles = (int32_t)tiles;
-    cudaError_t e = tac::launch_decode(d, dt, P, sms, reinterpret_cast<cudaStream_t>(stream));
+    cudaError_t e = tac::launch_decode(d, dt, w, nb, mode, P, sms, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
   }
   return ok();

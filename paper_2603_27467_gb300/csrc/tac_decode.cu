@@ -1,11 +1,12 @@
 // TurboAngle decode kernel for sm_103a (Sec. 3.1 reconstruction with the Eq. 2
 // dequantization of arXiv 2603.27467).
 //
-// A 256-thread CTA decodes a tile of TR = 256/L rows, L = d/16 lanes per row,
-// 8 angle pairs per lane:
-//   1. the tile's records (angle / norm / header planes) are staged global ->
-//      shared with cp.async: coalesced 16-byte chunks for contiguous slots,
-//      per-row copies for gathered slots; double buffered;
+// One kernel per (d, output dtype, n = 2^W, norm bits B, norm mode), like the
+// encoder.  A warp decodes warp tiles of RW = 32/L rows, L = d/16 lanes per
+// row, 8 angle pairs per lane, each warp with its own pipeline:
+//   1. a kNS-stage cp.async ring stages the tile's records (angle / norm /
+//      header segments, each a whole number of 16-byte chunks): one chunk per
+//      lane for contiguous slots, per-row copies for gathered slots;
 //   2. lane l unpacks its 8 consecutive codes (pairs 8l..8l+7) and rebuilds each
 //      pair from its bin-centre angle by table lookup: the table holds
 //      (cos phi_k + sin phi_k, cos phi_k - sin phi_k) / sqrt(d), i.e. the
@@ -23,83 +24,84 @@ namespace tac {
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles of records in flight
 
-template <int D, typename TOut>
+template <int D, typename TOut, int W, int B>
 struct Dec {
   using G = Geo<D>;
   using OT = RowTile<D, (int)sizeof(TOut)>;
   static constexpr int P = G::P, L = G::L, RW = G::RW;
   static constexpr int ESZ = (int)sizeof(TOut);
-  // one record stage of a warp tile: angle, norm and header segments
+  static constexpr int n = 1 << W;
+  static constexpr int AB = P * W / 8;        // angle record bytes per row
+  static constexpr int NB = P * B / 8;        // norm record bytes per row
+  static constexpr int NA = RW * AB / 16, NN = RW * NB / 16, NH = RW * 8 / 16;
+  static constexpr int NCH = NA + NN + NH;
+  static constexpr int ROUNDS = (NCH + 31) / 32;
+  // one record stage of a warp tile: angle | norm | header segments
   static constexpr int R_ANG = 0;
-  static constexpr int R_NRM = RW * P;                      // angle records <= P bytes per row
-  static constexpr int R_HDR = R_NRM + RW * P;              // norm records <= P bytes per row
+  static constexpr int R_NRM = RW * AB;
+  static constexpr int R_HDR = R_NRM + RW * NB;
   static constexpr int REC_W = R_HDR + RW * 8 + 16;         // + slack for 3-word angle reads
+  // Output chunk map: 32 consecutive 16-byte chunks cover RPQ rows.
+  static constexpr int CPR = OT::CPR, RPQ = 32 / CPR, CHUNKS = OT::CHUNKS;
   // per-warp shared memory region
   static constexpr int W_REC = 0;                           // kNS record stages
   static constexpr int W_TP = W_REC + kNS * REC_W;          // transpose rows
   static constexpr int W_OUT = W_TP + G::TP_W;              // output rows
-  static constexpr int W_JOB = W_OUT + OT::BYTES;           // current job (DecWarpJob)
-  static constexpr int WARP_B = W_JOB + 128;
-  static constexpr int OFF_TAB = kWarps * WARP_B;           // centre tables, every n
-  static constexpr int SMEM = OFF_TAB + kTabEntries * 8;
-  static_assert(REC_W % 16 == 0 && W_OUT % 16 == 0 && W_JOB % 16 == 0, "alignment");
+  static constexpr int WARP_B = W_OUT + OT::BYTES;
+  static constexpr int OFF_TAB = kWarps * WARP_B;           // centre table of this n
+  static constexpr int SMEM = OFF_TAB + n * 8;
+  static_assert(REC_W % 16 == 0 && W_TP % 16 == 0 && W_OUT % 16 == 0 && WARP_B % 16 == 0, "alignment");
+  static_assert(32 % CPR == 0 && RW % RPQ == 0, "chunk map");
 };
 
-struct DecWarpJob {
-  void* y;
-  int64_t rows;
-  int64_t stride;  // elements
-  int32_t t0, end, variant, pad_;
-};
-static_assert(sizeof(DecWarpJob) <= 128, "DecWarpJob");
-
-// Stage the records of warp tile (row0, nrows) of a job into `stage`.
-// Contiguous slots: 16-byte cp.async chunks of the three plane segments (a
-// segment of a full tile is a multiple of 16 bytes; a tail tile's last chunk is
-// zero-filled).  Gathered slots: lane r < nrows copies row r's record with plain loads.
-template <int D, typename TOut>
-__device__ __forceinline__ void stage_records(const uint8_t* codes, const uint8_t* norms, const uint8_t* hdr,
-                                              const int64_t* slot, int64_t capacity, int64_t row0, int nrows,
-                                              int AB, int NB, uint8_t* stage, int lane) {
-  using C = Dec<D, TOut>;
-  if (slot == nullptr) {
+// Stage the records of a tail tile (nrows < RW) or of gathered slots into
+// `stage`.  Contiguous slots: 16-byte cp.async chunks of the three segments,
+// the last chunk of each zero-filled past the tile.  Gathered slots: lane
+// r < nrows copies row r's record with plain loads; an out-of-range slot
+// decodes as an all-zero record.
+template <int AB, int NB, int R_NRM, int R_HDR>
+__device__ __noinline__ void stage_records_slow(const DecJob& J, int64_t row0, int nrows, uint8_t* stage,
+                                                int lane) {
+  if (J.slot == nullptr) {
     const int ba = nrows * AB, bn = nrows * NB, bh = nrows * 8;
     const int ca = (ba + 15) >> 4, cn = (bn + 15) >> 4, ch = (bh + 15) >> 4;
-    const uint8_t* ga = codes + row0 * AB;
-    const uint8_t* gn = norms + row0 * NB;
-    const uint8_t* gh = hdr + row0 * 8;
+    const uint8_t* ga = J.codes + row0 * AB;
+    const uint8_t* gn = J.norms + row0 * NB;
+    const uint8_t* gh = J.hdr + row0 * 8;
     for (int q = lane; q < ca + cn + ch; q += 32) {
       if (q < ca) {
         const int rem = ba - 16 * q;
-        cp_async16(stage + C::R_ANG + 16 * q, ga + 16 * q, rem >= 16 ? 16 : rem);
+        cp_async16(stage + 16 * q, ga + 16 * q, rem >= 16 ? 16 : rem);
       } else if (q < ca + cn) {
         const int qq = q - ca, rem = bn - 16 * qq;
-        cp_async16(stage + C::R_NRM + 16 * qq, gn + 16 * qq, rem >= 16 ? 16 : rem);
+        cp_async16(stage + R_NRM + 16 * qq, gn + 16 * qq, rem >= 16 ? 16 : rem);
       } else {
         const int qq = q - ca - cn, rem = bh - 16 * qq;
-        cp_async16(stage + C::R_HDR + 16 * qq, gh + 16 * qq, rem >= 16 ? 16 : rem);
+        cp_async16(stage + R_HDR + 16 * qq, gh + 16 * qq, rem >= 16 ? 16 : rem);
       }
     }
   } else if (lane < nrows) {
-    const int64_t s = slot[row0 + lane];
-    uint8_t* da = stage + C::R_ANG + lane * AB;
-    uint8_t* dn = stage + C::R_NRM + lane * NB;
-    float2* dh = reinterpret_cast<float2*>(stage + C::R_HDR) + lane;
-    if (s < 0 || s >= capacity) {  // out-of-range slot: decodes as an all-zero record
+    const int64_t s = J.slot[row0 + lane];
+    uint8_t* da = stage + lane * AB;
+    uint8_t* dn = stage + R_NRM + lane * NB;
+    float2* dh = reinterpret_cast<float2*>(stage + R_HDR) + lane;
+    if (s < 0 || s >= J.capacity) {
       for (int q = 0; q < AB; ++q) da[q] = 0;
       for (int q = 0; q < NB; ++q) dn[q] = 0;
       *dh = make_float2(0.f, 0.f);
       return;
     }
-    const uint8_t* sa = codes + s * AB;
-    const uint8_t* sn = norms + s * NB;
-    if ((AB & 3) == 0) {
-      for (int q = 0; q < AB / 4; ++q) reinterpret_cast<uint32_t*>(da)[q] = __ldg(reinterpret_cast<const uint32_t*>(sa) + q);
+    const uint8_t* sa = J.codes + s * AB;
+    const uint8_t* sn = J.norms + s * NB;
+    if constexpr ((AB & 3) == 0) {
+      for (int q = 0; q < AB / 4; ++q)
+        reinterpret_cast<uint32_t*>(da)[q] = __ldg(reinterpret_cast<const uint32_t*>(sa) + q);
     } else {
       for (int q = 0; q < AB; ++q) da[q] = __ldg(sa + q);
     }
-    for (int q = 0; q < NB / 4; ++q) reinterpret_cast<uint32_t*>(dn)[q] = __ldg(reinterpret_cast<const uint32_t*>(sn) + q);
-    *dh = __ldg(reinterpret_cast<const float2*>(hdr) + s);
+    for (int q = 0; q < NB / 4; ++q)
+      reinterpret_cast<uint32_t*>(dn)[q] = __ldg(reinterpret_cast<const uint32_t*>(sn) + q);
+    *dh = __ldg(reinterpret_cast<const float2*>(J.hdr) + s);
   }
 }
 
@@ -124,18 +126,16 @@ __device__ __forceinline__ uint64_t load_bytes(const uint8_t* p) {
 
 // Decode this lane's 8 pairs of warp-tile row r and stage the output row segment.
 template <int D, typename TOut, int W, int B, int MODE>
-__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab_all, int lane,
+__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab, int lane,
                                             const uint2 (&msk)[8]) {
-  using C = Dec<D, TOut>;
+  using C = Dec<D, TOut, W, B>;
   using G = Geo<D>;
   using OT = typename C::OT;
-  constexpr int P = C::P, L = C::L;
+  constexpr int L = C::L;
   constexpr int n = 1 << W;
-  constexpr int AB = P * W / 8;
-  constexpr int NB = P * B / 8;
+  constexpr int AB = C::AB, NB = C::NB;
   constexpr int Lq = (1 << B) - 1;
   const int r = lane / L, l = lane % L;
-  const float2* ttab = ttab_all + tab_offset(W);
 
   const uint64_t acc_a = load_bytes<W>(rec + C::R_ANG + r * AB + l * W);
   const uint64_t acc_n = load_bytes<B>(rec + C::R_NRM + r * NB + l * B);
@@ -144,6 +144,8 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
 
   // Dequantization (the inverse of Eq. 2): linear r^ = r_min + c (r_max - r_min)/L,
   // log r^ = 2^(l_min + c (l_max - l_min)/L); r_max == r_min gives r^ = r_min.
+  // The code enters as the float f = 1 + c 2^-B (its bits placed in the mantissa
+  // of 1.0), so base + c step = fma(f, 2^B step, base - 2^B step).
   const bool spread = hmax > hmin;
   float base, step;
   if constexpr (MODE == TAC_NORM_LINEAR) {
@@ -153,16 +155,18 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
     base = lg2_approx(hmin);
     step = spread ? (lg2_approx(hmax) - base) * (1.0f / (float)Lq) : 0.f;
   }
+  const float S = step * (float)(1 << B);
+  const float base2 = base - S;
 
   float2 v[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     const uint32_t k = (uint32_t)(acc_a >> (j * W)) & (uint32_t)(n - 1);
-    const uint32_t c = (uint32_t)(acc_n >> (j * B)) & (uint32_t)Lq;
-    float rh = __fmaf_rn(__uint2float_rn(c), step, base);
+    const uint32_t cb = (uint32_t)(acc_n >> (j * B)) & (uint32_t)Lq;
+    const float f = __uint_as_float(0x3F800000u | (cb << (23 - B)));
+    float rh = __fmaf_rn(f, S, base2);
     if constexpr (MODE != TAC_NORM_LINEAR) rh = ex2_approx(rh);
-    const float2 t = ttab[k];
-    v[j] = make_float2(rh * t.x, rh * t.y);
+    v[j] = mul2(make_float2(rh, rh), ttab[k]);
   }
   // Butterfly stages on pair-index bits 0..2 (this lane holds pairs 8l..8l+7).
   butterfly8<8>(v);
@@ -193,22 +197,20 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
   }
 }
 
-template <int D, typename TOut>
+template <int D, typename TOut, int W, int B, int MODE>
 __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_constant__ DecParams p) {
-  using C = Dec<D, TOut>;
+  using C = Dec<D, TOut, W, B>;
   using OT = typename C::OT;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
 
-  // Centre tables for every n = 2..256: (cos + sin, cos - sin)(2 pi k / n) / sqrt(d).
+  // Centre table of this n: (cos + sin, cos - sin)(2 pi k / n) / sqrt(d).
   float2* ttab = reinterpret_cast<float2*>(smem + C::OFF_TAB);
   const float sc = sqrtf(2.f / (float)D);  // sqrt2 / sqrt(d)
-  for (int idx = tid; idx < kTabEntries - 2; idx += kThreads) {
-    const int w = 31 - __clz(idx + 2);
-    const int k = idx - tab_offset(w);
-    const float2 cs = cos_sin_q8(centre_q8(k, 1 << w), 1 << w);  // (cos psi, sin psi), psi = phi + pi/4
-    ttab[idx] = make_float2(sc * cs.y, sc * cs.x);
+  for (int k = tid; k < C::n; k += kThreads) {
+    const float2 cs = cos_sin_q8(centre_q8(k, C::n), C::n);  // (cos psi, sin psi), psi = phi + pi/4
+    ttab[k] = make_float2(sc * cs.y, sc * cs.x);
   }
   __syncthreads();
 
@@ -217,28 +219,60 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
   if (t >= p.ntiles) return;
   uint8_t* wsm = smem + warp * C::WARP_B;
 
-  // Prefetch cursor: the job of the next warp tile whose records are staged.
+  // ---- prefetch cursor: the job of the next warp tile whose records are staged ----
   int pj = find_job(p, t);
-  int p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
+  int p_t0 = 0, p_end = 0;
+  int64_t p_rows = 0;
+  bool p_dense = true;
+  const uint8_t* i_src[C::ROUNDS];  // this lane's record chunk(s) at tile 0 of the job
+  int i_step[C::ROUNDS];            // bytes between consecutive tiles of its plane
+  auto set_issue_job = [&]() {
+    const DecJob& J = p.job[pj];
+    p_t0 = J.tile0;
+    p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
+    p_rows = J.rows;
+    p_dense = J.slot == nullptr;
+#pragma unroll
+    for (int q = 0; q < C::ROUNDS; ++q) {
+      const int ch = q * 32 + lane;
+      if (ch < C::NA) { i_src[q] = J.codes + 16 * ch; i_step[q] = C::RW * C::AB; }
+      else if (ch < C::NA + C::NN) { i_src[q] = J.norms + 16 * (ch - C::NA); i_step[q] = C::RW * C::NB; }
+      else { i_src[q] = J.hdr + 16 * (ch - C::NA - C::NN); i_step[q] = C::RW * 8; }
+    }
+  };
+  set_issue_job();
   auto issue = [&](int tt, int stg) {
     if (tt < p.ntiles) {
       while (tt >= p_end) {
         ++pj;
-        p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
+        set_issue_job();
       }
-      const DecJob& J = p.job[pj];
-      const int64_t row0 = (int64_t)(tt - J.tile0) * C::RW;
-      const int nrows = (int)min((int64_t)C::RW, J.rows - row0);
-      stage_records<D, TOut>(J.codes, J.norms, J.hdr, J.slot, J.capacity, row0, nrows, C::P * J.w / 8,
-                             C::P * J.b / 8, wsm + C::W_REC + stg * C::REC_W, lane);
+      const int rel = tt - p_t0;
+      const int64_t row0 = (int64_t)rel * C::RW;
+      uint8_t* stage = wsm + C::W_REC + stg * C::REC_W;
+      if (p_dense && row0 + C::RW <= p_rows) {
+#pragma unroll
+        for (int q = 0; q < C::ROUNDS; ++q) {
+          const int ch = q * 32 + lane;
+          if (ch < C::NCH) cp_async16(stage + 16 * ch, i_src[q] + (int64_t)rel * i_step[q], 16);
+        }
+      } else {
+        stage_records_slow<C::AB, C::NB, C::R_NRM, C::R_HDR>(p.job[pj], row0, (int)min((int64_t)C::RW, p_rows - row0),
+                                                            stage, lane);
+      }
     }
     cp_async_commit();
   };
 #pragma unroll
   for (int s = 0; s < kNS - 1; ++s) issue(t + s * Gw, s);
 
-  DecWarpJob* wj = reinterpret_cast<DecWarpJob*>(wsm + C::W_JOB);
-  int cj = -1, c_end = 0;
+  // ---- compute cursor ----
+  int c_t0 = 0, c_end = 0;
+  int64_t c_rows = 0, c_sb = 0;
+  // Output chunk q of a lane is row q*RPQ + lane/CPR, bytes (lane % CPR)*16.
+  const int lane_cr = lane / C::CPR;
+  const uint8_t* const out_src = wsm + C::W_OUT + lane_cr * OT::STRIDE + (lane % C::CPR) * 16;
+  uint8_t* o_dst = nullptr;  // this lane's first output chunk of the job's row 0
   uint2 msk[8];
 #pragma unroll
   for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
@@ -252,47 +286,31 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
       if (ns >= kNS) ns -= kNS;
       issue(t + (kNS - 1) * Gw, ns);
     }
-    if (t >= c_end) {  // next job: copy its descriptor to shared memory
-      cj = (cj < 0) ? find_job(p, t) : cj + 1;
-      while (cj + 1 < p.njobs && p.job[cj + 1].tile0 <= t) ++cj;
+    if (t >= c_end) {  // next job
+      const int cj = find_job(p, t);
       const DecJob& J = p.job[cj];
+      c_t0 = J.tile0;
       c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
-      if (lane == 0) {
-        wj->y = J.y; wj->rows = J.rows; wj->stride = J.stride; wj->t0 = J.tile0; wj->end = c_end;
-        wj->variant = (J.w - 1) * 4 + (J.b == 8 ? 2 : 0) + (J.mode == TAC_NORM_LOG ? 1 : 0);
-      }
+      c_rows = J.rows;
+      c_sb = J.stride * C::ESZ;
+      o_dst = reinterpret_cast<uint8_t*>(J.y) + lane_cr * c_sb + (lane % C::CPR) * 16;
       const int l = lane % C::L;
 #pragma unroll
       for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
-      __syncwarp();
     }
     const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;
-
-#define TAC_DEC_CASE(WW)                                                                              \
-  case (WW - 1) * 4 + 0: decode_body<D, TOut, WW, 4, TAC_NORM_LINEAR>(rec, wsm, ttab, lane, msk); break;  \
-  case (WW - 1) * 4 + 1: decode_body<D, TOut, WW, 4, TAC_NORM_LOG>(rec, wsm, ttab, lane, msk); break;     \
-  case (WW - 1) * 4 + 2: decode_body<D, TOut, WW, 8, TAC_NORM_LINEAR>(rec, wsm, ttab, lane, msk); break;  \
-  case (WW - 1) * 4 + 3: decode_body<D, TOut, WW, 8, TAC_NORM_LOG>(rec, wsm, ttab, lane, msk); break;
-    switch (wj->variant) {
-      TAC_DEC_CASE(1) TAC_DEC_CASE(2) TAC_DEC_CASE(3) TAC_DEC_CASE(4)
-      TAC_DEC_CASE(5) TAC_DEC_CASE(6) TAC_DEC_CASE(7) TAC_DEC_CASE(8)
-      default: break;
-    }
-#undef TAC_DEC_CASE
+    decode_body<D, TOut, W, B, MODE>(rec, wsm, ttab, lane, msk);
     __syncwarp();
     // Write the warp tile's rows: 16-byte chunks, coalesced.
     {
-      const int64_t row0 = (int64_t)(t - wj->t0) * C::RW;
-      const int nrows = (int)min((int64_t)C::RW, wj->rows - row0);
-      uint8_t* y = reinterpret_cast<uint8_t*>(wj->y);
-      const int64_t sb = wj->stride * C::ESZ;
+      const int64_t row0 = (int64_t)(t - c_t0) * C::RW;
+      const int64_t left = c_rows - row0 - lane_cr;
+      uint8_t* dst = o_dst + row0 * c_sb;
 #pragma unroll
-      for (int q = 0; q < OT::CHUNKS; ++q) {
-        const int id = q * 32 + lane;
-        const int rr = id / OT::CPR, col = (id % OT::CPR) * 16;
-        if (rr < nrows)
-          *reinterpret_cast<uint4*>(y + (row0 + rr) * sb + col) =
-              *reinterpret_cast<const uint4*>(wsm + C::W_OUT + rr * OT::STRIDE + col);
+      for (int q = 0; q < C::CHUNKS; ++q) {
+        if (q * C::RPQ < left)
+          *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(out_src + q * C::RPQ * OT::STRIDE);
+        dst += C::RPQ * c_sb;
       }
     }
     stage = (stage + 1 == kNS) ? 0 : stage + 1;
@@ -300,10 +318,10 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
   cp_async_wait<0>();
 }
 
-template <int D, typename TOut>
-static cudaError_t launch_decode_t(const DecParams& p, int grid_cap, cudaStream_t st) {
-  using C = Dec<D, TOut>;
-  auto kern = decode_kernel<D, TOut>;
+template <int D, typename TOut, int W, int B, int MODE>
+static cudaError_t launch_decode_v(const DecParams& p, int grid_cap, cudaStream_t st) {
+  using C = Dec<D, TOut, W, B>;
+  auto kern = decode_kernel<D, TOut, W, B, MODE>;
   static int configured[64] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -324,6 +342,22 @@ static cudaError_t launch_decode_t(const DecParams& p, int grid_cap, cudaStream_
   return cudaGetLastError();
 }
 
+template <int D, typename TOut>
+static cudaError_t launch_decode_t(const DecParams& p, int w, int b, int mode, int sms, cudaStream_t st) {
+#define TAC_DEC_CASE(WW)                                                                         \
+  case (WW - 1) * 4 + 0: return launch_decode_v<D, TOut, WW, 4, TAC_NORM_LINEAR>(p, sms, st);    \
+  case (WW - 1) * 4 + 1: return launch_decode_v<D, TOut, WW, 4, TAC_NORM_LOG>(p, sms, st);       \
+  case (WW - 1) * 4 + 2: return launch_decode_v<D, TOut, WW, 8, TAC_NORM_LINEAR>(p, sms, st);    \
+  case (WW - 1) * 4 + 3: return launch_decode_v<D, TOut, WW, 8, TAC_NORM_LOG>(p, sms, st);
+  switch ((w - 1) * 4 + (b == 8 ? 2 : 0) + (mode == TAC_NORM_LOG ? 1 : 0)) {
+    TAC_DEC_CASE(1) TAC_DEC_CASE(2) TAC_DEC_CASE(3) TAC_DEC_CASE(4)
+    TAC_DEC_CASE(5) TAC_DEC_CASE(6) TAC_DEC_CASE(7) TAC_DEC_CASE(8)
+    default: break;
+  }
+#undef TAC_DEC_CASE
+  return cudaErrorInvalidValue;
+}
+
 // Instances: the build compiles this file once per (d, dtype) with
 // -DTAC_INST_D=<d> -DTAC_INST_BF16=1|-DTAC_INST_F32=1 so they compile in parallel;
 // without those flags every instance is compiled here.
@@ -337,45 +371,35 @@ static cudaError_t launch_decode_t(const DecParams& p, int grid_cap, cudaStream_
 #ifndef TAC_INST_F32
 #define TAC_INST_F32 0
 #endif
+#define TAC_DEC_INSTANCE(DD, NAME, T)                                                                 \
+  cudaError_t launch_decode_##DD##_##NAME(const DecParams& p, int w, int b, int mode, int sms,       \
+                                          cudaStream_t st) {                                         \
+    return launch_decode_t<DD, T>(p, w, b, mode, sms, st);                                           \
+  }
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 16 && TAC_INST_BF16)
-cudaError_t launch_decode_16_bf16(const DecParams& p, int sms, cudaStream_t st) {
-  return launch_decode_t<16, __nv_bfloat16>(p, sms, st);
-}
+TAC_DEC_INSTANCE(16, bf16, __nv_bfloat16)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 32 && TAC_INST_BF16)
-cudaError_t launch_decode_32_bf16(const DecParams& p, int sms, cudaStream_t st) {
-  return launch_decode_t<32, __nv_bfloat16>(p, sms, st);
-}
+TAC_DEC_INSTANCE(32, bf16, __nv_bfloat16)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 64 && TAC_INST_BF16)
-cudaError_t launch_decode_64_bf16(const DecParams& p, int sms, cudaStream_t st) {
-  return launch_decode_t<64, __nv_bfloat16>(p, sms, st);
-}
+TAC_DEC_INSTANCE(64, bf16, __nv_bfloat16)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 128 && TAC_INST_BF16)
-cudaError_t launch_decode_128_bf16(const DecParams& p, int sms, cudaStream_t st) {
-  return launch_decode_t<128, __nv_bfloat16>(p, sms, st);
-}
+TAC_DEC_INSTANCE(128, bf16, __nv_bfloat16)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 16 && TAC_INST_F32)
-cudaError_t launch_decode_16_f32(const DecParams& p, int sms, cudaStream_t st) {
-  return launch_decode_t<16, float>(p, sms, st);
-}
+TAC_DEC_INSTANCE(16, f32, float)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 32 && TAC_INST_F32)
-cudaError_t launch_decode_32_f32(const DecParams& p, int sms, cudaStream_t st) {
-  return launch_decode_t<32, float>(p, sms, st);
-}
+TAC_DEC_INSTANCE(32, f32, float)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 64 && TAC_INST_F32)
-cudaError_t launch_decode_64_f32(const DecParams& p, int sms, cudaStream_t st) {
-  return launch_decode_t<64, float>(p, sms, st);
-}
+TAC_DEC_INSTANCE(64, f32, float)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 128 && TAC_INST_F32)
-cudaError_t launch_decode_128_f32(const DecParams& p, int sms, cudaStream_t st) {
-  return launch_decode_t<128, float>(p, sms, st);
-}
+TAC_DEC_INSTANCE(128, f32, float)
 #endif
+#undef TAC_DEC_INSTANCE
 
 }  // namespace tac

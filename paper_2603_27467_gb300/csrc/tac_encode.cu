@@ -1,5 +1,9 @@
 // TurboAngle encode kernel for sm_103a (Alg. 1 + Sec. 3.3 / Eq. 2 of arXiv 2603.27467).
 //
+// One kernel per (d, input dtype, n = 2^W, norm bits B, norm mode): a launch
+// encodes a batch of jobs that share the codebook shape, so every record size
+// is a compile-time constant and the instruction footprint is one body.
+//
 // Work is split into warp tiles: L = d/16 lanes share a row, each lane owns 8
 // angle pairs (16 elements), so a warp encodes RW = 32/L rows at a time.  Every
 // warp runs its own pipeline (no block-wide barrier in the main loop):
@@ -18,53 +22,81 @@
 //      (max error 0.0038 rad: Rajan, Wang, Inkol, Joyal, "Efficient
 //      approximations for the arctangent function", IEEE SPM 2006), then the sign
 //      of the cross product of (E, O) with the edge direction.  The test is
-//      certified by a rigorous bound on the fp32 error; pairs inside it are
-//      re-decided by the warp in fp64 from the staged input (exact sums);
+//      certified by a rigorous bound on the fp32 error; the pairs it does not
+//      certify are re-decided by the warp from error-free double-float sums of
+//      the staged input (no fp64: the FP64 pipe is a small fraction of fp32 here);
 //   4. Eq. 2 norm codes (linear, or on log2 r) against the stored fp32 (r_min, r_max);
 //   5. each lane packs its 8 codes LSB-first; the warp stages its records in
-//      shared memory and writes them with 16-byte stores (contiguous slots) or
-//      per row (scatter-append slots).
+//      shared memory and writes them with one 16-byte store per lane (contiguous
+//      slots) or per row (scatter-append slots).
 #include "tac_common.cuh"
 
 namespace tac {
 
-// fp64 edge directions (cos psi_e, sin psi_e) for every n = 2..256, read
-// warp-uniformly by the exact-decision path.
-__constant__ cx::EdgeTable g_edge_dir = cx::make_edge_table();
+// Edge directions (cos psi_e, sin psi_e) for every n = 2..256 as double-float
+// pairs (c = ch + cl, s = sh + sl), read warp-uniformly by the exact path.
+namespace cx {
+struct DF4 { float ch, cl, sh, sl; };
+struct DFEdgeTable { DF4 v[kTabEntries]; };
+constexpr DFEdgeTable make_df_edge_table() {
+  DFEdgeTable t{};
+  for (int idx = 0; idx < kTabEntries - 2; ++idx) {
+    int w = 1;
+    while ((1 << (w + 1)) - 2 <= idx) ++w;
+    const int n = 1 << w, e = idx - ((1 << w) - 2);
+    const CS d = cos_sin_q8(8 * e + 4 + n, n);
+    const float ch = (float)d.c, sh = (float)d.s;
+    t.v[idx] = DF4{ch, (float)(d.c - (double)ch), sh, (float)(d.s - (double)sh)};
+  }
+  return t;
+}
+}  // namespace cx
+__constant__ cx::DFEdgeTable g_edge_df = cx::make_df_edge_table();
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles in flight
 
-template <int D, typename TIn>
+template <int D, typename TIn, int W, int B>
 struct Enc {
   using G = Geo<D>;
   using IT = RowTile<D, (int)sizeof(TIn)>;
   static constexpr int P = G::P, L = G::L, RW = G::RW;
   static constexpr int ESZ = (int)sizeof(TIn);
+  static constexpr int n = 1 << W;
+  static constexpr int AB = P * W / 8;        // angle record bytes per row
+  static constexpr int NB = P * B / 8;        // norm record bytes per row
+  // A warp tile's records: RW*AB = 32 W and RW*NB = 32 B bytes, RW*8 header
+  // bytes: every segment is a whole number of 16-byte chunks.
+  static constexpr int NA = RW * AB / 16, NN = RW * NB / 16, NH = RW * 8 / 16;
+  static constexpr int NCH = NA + NN + NH;
+  static constexpr int ROUNDS = (NCH + 31) / 32;
+  // Input chunk map: 32 consecutive 16-byte chunks cover RPQ rows.
+  static constexpr int CPR = IT::CPR, RPQ = 32 / CPR, CHUNKS = IT::CHUNKS;
   // per-warp shared memory region
   static constexpr int W_IN = 0;                            // kNS input stages
   static constexpr int W_TP = W_IN + kNS * IT::BYTES;       // transpose rows
-  static constexpr int W_ANG = W_TP + G::TP_W;              // staged angle records (<= P bytes/row)
-  static constexpr int W_NRM = W_ANG + RW * P;              // staged norm records (<= P bytes/row)
-  static constexpr int W_HDR = W_NRM + RW * P;              // staged headers
-  static constexpr int W_JOB = (W_HDR + RW * 8 + 15) / 16 * 16;  // current job (WarpJob)
-  static constexpr int WARP_B = W_JOB + 128;
-  static constexpr int OFF_TAB = kWarps * WARP_B;           // fp32 edge tables, every n
-  static constexpr int SMEM = OFF_TAB + kTabEntries * 8;
+  static constexpr int W_ANG = W_TP + G::TP_W;              // staged records: angle | norm | header
+  static constexpr int W_NRM = W_ANG + RW * AB;
+  static constexpr int W_HDR = W_NRM + RW * NB;
+  static constexpr int W_JOB = W_HDR + RW * 8;              // current job (WarpJob)
+  static constexpr int WARP_B = W_JOB + 64;
+  static constexpr int OFF_TAB = kWarps * WARP_B;           // fp32 edge table of this n
+  static constexpr int SMEM = OFF_TAB + n * 8;
+  static_assert((RW * AB) % 16 == 0 && (RW * NB) % 16 == 0 && (RW * 8) % 16 == 0, "record segments");
+  static_assert(W_TP % 16 == 0 && W_ANG % 16 == 0 && W_JOB % 16 == 0 && WARP_B % 16 == 0, "alignment");
+  static_assert(32 % CPR == 0 && RW % RPQ == 0, "chunk map");
 };
 
-// The job a warp is encoding, copied from the kernel parameters into the warp's
-// shared region when the warp reaches a new job (keeps it out of registers).
+// The job a warp is encoding as far as the rare paths need it (exact
+// re-decision, tail tiles and scatter), kept in the warp's shared region.
 struct WarpJob {
   uint8_t* codes;
   uint8_t* norms;
   uint8_t* hdr;
   const int64_t* slot;
   int64_t capacity;
-  int64_t rows;
-  int32_t t0, end, variant, ab, nb, pad_;
   uint32_t signs[4];
 };
-static_assert(sizeof(WarpJob) <= 128, "WarpJob");
+static_assert(sizeof(WarpJob) <= 64, "WarpJob");
 
 // Store the low NBYTES (<= 8) bytes of (hi:lo) at a shared address aligned to gcd(NBYTES, 8).
 template <int NBYTES>
@@ -83,55 +115,88 @@ __device__ __forceinline__ void store_bytes(uint8_t* dst, uint32_t lo, uint32_t 
   }
 }
 
+// Error-free transformation: s + e == a + b exactly (Knuth's TwoSum).
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+  s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
 // Exact re-decision of pair i of warp-tile row rr by the whole warp (all lanes
-// call it with the same arguments).  E_i, O_i are summed in fp64 from the staged
-// input (each term is an exactly representable signed input element), the
-// candidate edge comes from an fp32 atan2 of the exact values and the edge test
-// is evaluated in fp64 against an fp64 edge direction.  Returns k in every lane.
-template <int D, typename TIn>
-__device__ __forceinline__ int exact_angle_code(const uint32_t* signs, int w, const uint8_t* in, int rr, int i,
-                                             int lane) {
-  using C = Enc<D, TIn>;
+// call it with the same arguments); returns k in every lane.  E_i = sum_j
+// +-x_2j and O_i = sum_j +-x_2j+1 (each term an exactly representable signed
+// input element) are accumulated as double-float values with TwoSum; their
+// relative error is of order 64 u^2, far inside the 1e-5 rad band the angle
+// parity tolerates.  The candidate edge comes from an fp32 atan2 of the sums
+// (an error near a bin centre picks a neighbouring edge, whose test gives the
+// same bin), the edge test m = E cos psi - O sin psi is evaluated in
+// double-float against the double-float edge direction.
+template <int D, typename TIn, int W, int B>
+__device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uint8_t* in, int rr, int i,
+                                                int lane) {
+  using C = Enc<D, TIn, W, B>;
   using IT = typename C::IT;
-  const int n = 1 << w;
-  double Ep = 0.0, Op = 0.0;
+  constexpr int n = 1 << W;
+  float eh = 0.f, el = 0.f, oh = 0.f, ol = 0.f;
   const uint8_t* row = in + rr * IT::STRIDE;
-  for (int jj = lane; jj < C::P; jj += 32) {
-    const int j0 = 2 * jj, j1 = 2 * jj + 1;
-    float x0, x1;
-    if constexpr (C::ESZ == 2) {
-      const uint32_t u = *reinterpret_cast<const uint32_t*>(row + 4 * jj);
-      x0 = bf16lo(u); x1 = bf16hi(u);
-    } else {
-      const float2 u = *reinterpret_cast<const float2*>(row + 8 * jj);
-      x0 = u.x; x1 = u.y;
+#pragma unroll
+  for (int j0 = 0; j0 < C::P; j0 += 32) {
+    const int jj = j0 + lane;
+    if (jj < C::P) {
+      const int e0 = 2 * jj, e1 = 2 * jj + 1;
+      float x0, x1;
+      if constexpr (C::ESZ == 2) {
+        const uint32_t u = *reinterpret_cast<const uint32_t*>(row + 4 * jj);
+        x0 = bf16lo(u); x1 = bf16hi(u);
+      } else {
+        const float2 u = *reinterpret_cast<const float2*>(row + 8 * jj);
+        x0 = u.x; x1 = u.y;
+      }
+      const bool neg = __popc((unsigned)(i & jj)) & 1;
+      if (((signs[e0 >> 5] >> (e0 & 31)) & 1u) != (uint32_t)neg) x0 = -x0;
+      if (((signs[e1 >> 5] >> (e1 & 31)) & 1u) != (uint32_t)neg) x1 = -x1;
+      float t;
+      two_sum(eh, x0, eh, t); el = __fadd_rn(el, t);
+      two_sum(oh, x1, oh, t); ol = __fadd_rn(ol, t);
     }
-    if ((signs[j0 >> 5] >> (j0 & 31)) & 1u) x0 = -x0;
-    if ((signs[j1 >> 5] >> (j1 & 31)) & 1u) x1 = -x1;
-    const bool neg = __popc((unsigned)(i & jj)) & 1;
-    Ep += neg ? -(double)x0 : (double)x0;
-    Op += neg ? -(double)x1 : (double)x1;
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
-    Ep += __shfl_xor_sync(0xffffffffu, Ep, off);
-    Op += __shfl_xor_sync(0xffffffffu, Op, off);
+    const float a = __shfl_xor_sync(0xffffffffu, eh, off), b = __shfl_xor_sync(0xffffffffu, el, off);
+    const float c = __shfl_xor_sync(0xffffffffu, oh, off), d = __shfl_xor_sync(0xffffffffu, ol, off);
+    float t;
+    two_sum(eh, a, eh, t); el = __fadd_rn(__fadd_rn(el, b), t);
+    two_sum(oh, c, oh, t); ol = __fadd_rn(__fadd_rn(ol, d), t);
   }
-  if (Ep == 0.0 && Op == 0.0) return 0;  // pair (0, 0) -> bin 0
-  const float th = atan2f((float)(Ep - Op), (float)(Ep + Op));
+  two_sum(eh, el, eh, el);  // renormalize: eh == 0 now means E == 0
+  two_sum(oh, ol, oh, ol);
+  if (eh == 0.f && oh == 0.f) return 0;  // pair (0, 0) -> bin 0
+  const float th = atan2f(__fsub_rn(eh, oh), __fadd_rn(eh, oh));
   const int e = ((int)floorf(th * ((float)n * 0.15915494309189535f))) & (n - 1);
-  const cx::CS ab = g_edge_dir.v[tab_offset(w) + e];
-  const double m = fma(Ep, ab.c, -(Op * ab.s));
-  return (e + (m >= 0.0 ? 1 : 0)) & (n - 1);
+  const cx::DF4 dir = g_edge_df.v[tab_offset(W) + e];
+  const float p1 = __fmul_rn(eh, dir.ch), q1 = __fmaf_rn(eh, dir.ch, -p1);
+  const float p2 = __fmul_rn(oh, dir.sh), q2 = __fmaf_rn(oh, dir.sh, -p2);
+  float dd, t;
+  two_sum(p1, -p2, dd, t);
+  float rest = __fadd_rn(t, __fsub_rn(q1, q2));
+  rest = __fmaf_rn(eh, dir.cl, rest);
+  rest = __fmaf_rn(el, dir.ch, rest);
+  rest = __fmaf_rn(-oh, dir.sl, rest);
+  rest = __fmaf_rn(-ol, dir.sh, rest);
+  const float m = __fadd_rn(dd, rest);
+  return (e + (m >= 0.f ? 1 : 0)) & (n - 1);
 }
 
-// Patch code i (W bits) of a staged angle record.
-__device__ __forceinline__ void patch_code(uint8_t* rec, int i, int W, int k) {
-  for (int t = 0; t < W; ++t) {
-    const int bit = i * W + t;
-    const uint8_t mask = (uint8_t)(1u << (bit & 7));
-    if ((k >> t) & 1) rec[bit >> 3] |= mask; else rec[bit >> 3] &= (uint8_t)~mask;
-  }
+// Patch code i (W bits) of a staged angle record (one lane).
+template <int W>
+__device__ __forceinline__ void patch_code(uint8_t* rec, int i, int k) {
+  const int bit = i * W, b0 = bit >> 3, sh = bit & 7;
+  const uint32_t mask = ((1u << W) - 1u) << sh;
+  uint32_t v = rec[b0];
+  if (sh + W > 8) v |= (uint32_t)rec[b0 + 1] << 8;
+  v = (v & ~mask) | ((uint32_t)k << sh);
+  rec[b0] = (uint8_t)v;
+  if (sh + W > 8) rec[b0 + 1] = (uint8_t)(v >> 8);
 }
 
 // Alg. 1 bin of the pair (E, O) (butterfly halves, y = (E + O, E - O)) for
@@ -162,19 +227,19 @@ __device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et
 // Encode this lane's 8 pairs of warp-tile row r (lane l of the row) and stage
 // the records; W = log2 n, B = norm bits, MODE = TAC_NORM_LINEAR / TAC_NORM_LOG.
 template <int D, typename TIn, int W, int B, int MODE>
-__device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const float2* etab, int nrows,
+__device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const float2* et, int nrows,
                                           int lane, const uint2 (&msk)[8], const uint32_t* signs) {
   // (for bf16 only msk[m].x is used; the .y words are constant zero)
-  using C = Enc<D, TIn>;
+  using C = Enc<D, TIn, W, B>;
   using G = Geo<D>;
   using IT = typename C::IT;
   constexpr int P = C::P, L = C::L;
   constexpr int n = 1 << W;
-  constexpr int AB = P * W / 8;           // angle record bytes
-  constexpr int NB = P * B / 8;           // norm record bytes
+  constexpr int AB = C::AB, NB = C::NB;
   constexpr int Lq = (1 << B) - 1;
   const int r = lane / L, l = lane % L;
   const bool live = r < nrows;
+  static_assert(P == 8 * L, "geometry");
 
   // ---- load 8 pairs (i = l + L*m), apply D, widen ----
   float2 v[8];
@@ -256,14 +321,12 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   const float sthr = rthr * rthr;
 
   // ---- pass 2: angle codes (Alg. 1), norm codes (Eq. 2), packing ----
-  const float2* et = etab + tab_offset(W);
-  uint32_t alo = 0, ahi = 0, nlo = 0, nhi = 0;
-  float mmin = __int_as_float(0x7f800000);
+  uint32_t alo = 0, ahi = 0, nlo = 0, nhi = 0, fm = 0;
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     float m;
     const uint32_t k = edge_test<W>(v[j].x, v[j].y, et, m);
-    mmin = fminf(mmin, fabsf(m));
+    fm |= (fabsf(m) < tau ? 1u : 0u) << j;      // not certified by the bound
     float f;
     if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_approx(s[j]);
     else f = lg2_approx(fmaxf(s[j], sfloor));
@@ -274,16 +337,11 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
     else { alo |= k << sa; ahi |= k >> (32 - sa); }
     if (sn < 32) nlo |= c << sn; else nhi |= c << (sn - 32);
   }
-  uint32_t fm = 0;
-  if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; }
-  else if (mmin < tau || lmin_s < sthr) {  // rare: name the uncertified pairs
+  if (lmin_s < sthr) {  // rare: small-norm pairs
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      float m;
-      edge_test<W>(v[j].x, v[j].y, et, m);
-      if (fabsf(m) < tau || s[j] < sthr) fm |= 1u << j;
-    }
+    for (int j = 0; j < 8; ++j) fm |= (s[j] < sthr ? 1u : 0u) << j;
   }
+  if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; fm = 0; }
   if (!live) fm = 0;
 
   // ---- stage the records ----
@@ -305,72 +363,61 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
       const int j = __ffs(mm) - 1;
       mm &= mm - 1;
       const int i = 8 * ol + j;
-      const int kk = exact_angle_code<D, TIn>(signs, W, in, rr, i, lane);
-      if (lane == 0) patch_code(wsm + C::W_ANG + rr * AB, i, W, kk);
+      const int kk = exact_angle_code<D, TIn, W, B>(signs, in, rr, i, lane);
+      if (lane == 0) patch_code<W>(wsm + C::W_ANG + rr * AB, i, kk);
     }
     __syncwarp();
   }
 }
 
-// Write the warp tile's staged records (nrows rows from row0) to the planes.
-__device__ __forceinline__ void warp_copy_out(uint8_t* codes, uint8_t* norms, uint8_t* hdr, const int64_t* slot,
-                                              int64_t capacity, const uint8_t* sang, const uint8_t* snrm,
-                                              const uint8_t* shdr, int64_t row0, int nrows, int RW, int AB, int NB,
-                                              int lane) {
-  if (slot == nullptr) {
-    uint8_t* ga = codes + row0 * AB;
-    uint8_t* gn = norms + row0 * NB;
-    uint8_t* gh = hdr + row0 * 8;
-    if (nrows == RW) {  // full tile: each plane segment is a 16-byte multiple (32 w, 32 b, 8 RW bytes)
-      const int na = RW * AB / 16, nn = RW * NB / 16, nh = RW / 2;
-      if (lane < na) reinterpret_cast<uint4*>(ga)[lane] = reinterpret_cast<const uint4*>(sang)[lane];
-      if (lane < nn) reinterpret_cast<uint4*>(gn)[lane] = reinterpret_cast<const uint4*>(snrm)[lane];
-      if (lane < nh) reinterpret_cast<uint4*>(gh)[lane] = reinterpret_cast<const uint4*>(shdr)[lane];
-    } else {
-      for (int q = lane; q < nrows * AB; q += 32) ga[q] = sang[q];
-      for (int q = lane; q < nrows * NB; q += 32) gn[q] = snrm[q];
-      for (int q = lane; q < nrows * 8; q += 32) gh[q] = shdr[q];
-    }
+// Records of a tail tile (nrows < RW) or of scattered slots, from the staged
+// records to the planes.
+template <int AB, int NB>
+__device__ __noinline__ void copy_out_slow(const WarpJob* wj, const uint8_t* sang, const uint8_t* snrm,
+                                           const uint8_t* shdr, int64_t row0, int nrows, int lane) {
+  if (wj->slot == nullptr) {
+    uint8_t* ga = wj->codes + row0 * AB;
+    uint8_t* gn = wj->norms + row0 * NB;
+    uint8_t* gh = wj->hdr + row0 * 8;
+    for (int q = lane; q < nrows * AB; q += 32) ga[q] = sang[q];
+    for (int q = lane; q < nrows * NB; q += 32) gn[q] = snrm[q];
+    for (int q = lane; q < nrows * 8; q += 32) gh[q] = shdr[q];
   } else if (lane < nrows) {
-    const int64_t s = slot[row0 + lane];
-    if (s < 0 || s >= capacity) return;  // out-of-range slots are skipped
-    uint8_t* ga = codes + s * AB;
-    uint8_t* gn = norms + s * NB;
+    const int64_t s = wj->slot[row0 + lane];
+    if (s < 0 || s >= wj->capacity) return;  // out-of-range slots are skipped
+    uint8_t* ga = wj->codes + s * AB;
+    uint8_t* gn = wj->norms + s * NB;
     const uint8_t* a = sang + lane * AB;
     const uint8_t* nn = snrm + lane * NB;
-    if ((AB & 15) == 0) {
+    if constexpr ((AB & 15) == 0) {
       for (int q = 0; q < AB / 16; ++q) reinterpret_cast<uint4*>(ga)[q] = reinterpret_cast<const uint4*>(a)[q];
-    } else if ((AB & 7) == 0) {
+    } else if constexpr ((AB & 7) == 0) {
       for (int q = 0; q < AB / 8; ++q) reinterpret_cast<uint2*>(ga)[q] = reinterpret_cast<const uint2*>(a)[q];
-    } else if ((AB & 3) == 0) {
+    } else if constexpr ((AB & 3) == 0) {
       for (int q = 0; q < AB / 4; ++q) reinterpret_cast<uint32_t*>(ga)[q] = reinterpret_cast<const uint32_t*>(a)[q];
     } else {
       for (int q = 0; q < AB; ++q) ga[q] = a[q];
     }
-    if ((NB & 7) == 0) {
+    if constexpr ((NB & 7) == 0) {
       for (int q = 0; q < NB / 8; ++q) reinterpret_cast<uint2*>(gn)[q] = reinterpret_cast<const uint2*>(nn)[q];
     } else {
       for (int q = 0; q < NB / 4; ++q) reinterpret_cast<uint32_t*>(gn)[q] = reinterpret_cast<const uint32_t*>(nn)[q];
     }
-    reinterpret_cast<float2*>(hdr)[s] = reinterpret_cast<const float2*>(shdr)[lane];
+    reinterpret_cast<float2*>(wj->hdr)[s] = reinterpret_cast<const float2*>(shdr)[lane];
   }
 }
 
-template <int D, typename TIn>
+template <int D, typename TIn, int W, int B, int MODE>
 __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_constant__ EncParams p) {
-  using C = Enc<D, TIn>;
+  using C = Enc<D, TIn, W, B>;
   using IT = typename C::IT;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
 
-  // fp32 edge tables for every n = 2..256 (shared by the CTA).
+  // fp32 edge table of this n (shared by the CTA).
   float2* etab = reinterpret_cast<float2*>(smem + C::OFF_TAB);
-  for (int idx = tid; idx < kTabEntries - 2; idx += kThreads) {
-    const int w = 31 - __clz(idx + 2);
-    const int e = idx - tab_offset(w);
-    etab[idx] = cos_sin_q8(edge_q8(e, 1 << w), 1 << w);
-  }
+  for (int e = tid; e < C::n; e += kThreads) etab[e] = cos_sin_q8(edge_q8(e, C::n), C::n);
   __syncthreads();
 
   const int Gw = gridDim.x * kWarps;
@@ -378,32 +425,40 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
   if (t >= p.ntiles) return;
   uint8_t* wsm = smem + warp * C::WARP_B;
 
-
-  // Prefetch cursor (job of the next warp tile to load) and its registers.
+  // ---- prefetch cursor: the job of the next warp tile to load ----
+  // Lane chunk q of a tile is row q*RPQ + lane/CPR, bytes (lane % CPR)*16.
+  const int lane_cr = lane / C::CPR;
+  uint8_t* const in_dst = wsm + C::W_IN + lane_cr * IT::STRIDE + (lane % C::CPR) * 16;
   int pj = find_job(p, t);
-  int p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
-  int p_t0 = p.job[pj].tile0;
-  const uint8_t* p_x = reinterpret_cast<const uint8_t*>(p.job[pj].x);
-  int64_t p_rows = p.job[pj].rows, p_sb = p.job[pj].stride * C::ESZ;
+  int p_t0 = 0, p_end = 0;
+  int64_t p_left0 = 0, p_sb = 0;     // rows of the job from this lane's first row; row stride (bytes)
+  const uint8_t* p_x = nullptr;      // job base (a valid address for zero-fill chunks)
+  const uint8_t* p_src = nullptr;    // this lane's first chunk of the job's row 0
+  auto set_issue_job = [&]() {
+    const EncJob& J = p.job[pj];
+    p_t0 = J.tile0;
+    p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
+    p_left0 = J.rows - lane_cr;
+    p_sb = J.stride * C::ESZ;
+    p_x = reinterpret_cast<const uint8_t*>(J.x);
+    p_src = p_x + lane_cr * p_sb + (lane % C::CPR) * 16;
+  };
+  set_issue_job();
   auto issue = [&](int tt, int stg) {
     if (tt < p.ntiles) {
       while (tt >= p_end) {  // monotone: a warp's tiles only move forward
         ++pj;
-        p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
-        p_t0 = p.job[pj].tile0;
-        p_x = reinterpret_cast<const uint8_t*>(p.job[pj].x);
-        p_rows = p.job[pj].rows;
-        p_sb = p.job[pj].stride * C::ESZ;
+        set_issue_job();
       }
       const int64_t row0 = (int64_t)(tt - p_t0) * C::RW;
-      uint8_t* dst = wsm + C::W_IN + stg * IT::BYTES;
+      const int64_t left = p_left0 - row0;
+      const uint8_t* src = p_src + row0 * p_sb;
+      uint8_t* dst = in_dst + stg * IT::BYTES;
 #pragma unroll
-      for (int q = 0; q < IT::CHUNKS; ++q) {
-        const int id = q * 32 + lane;            // chunk id -> (row, column) of the warp tile
-        const int cr = id / IT::CPR, ccol = (id % IT::CPR) * 16;
-        const int64_t row = row0 + cr;
-        const bool ok = row < p_rows;
-        cp_async16(dst + cr * IT::STRIDE + ccol, ok ? p_x + row * p_sb + ccol : p_x, ok ? 16 : 0);
+      for (int q = 0; q < C::CHUNKS; ++q) {
+        const bool ok = q * C::RPQ < left;
+        cp_async16(dst + q * C::RPQ * IT::STRIDE, ok ? src : p_x, ok ? 16 : 0);
+        src += C::RPQ * p_sb;
       }
     }
     cp_async_commit();
@@ -411,9 +466,17 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
 #pragma unroll
   for (int s = 0; s < kNS - 1; ++s) issue(t + s * Gw, s);
 
-  // Compute cursor: the current job lives in the warp's shared region.
+  // ---- compute cursor ----
   WarpJob* wj = reinterpret_cast<WarpJob*>(wsm + C::W_JOB);
-  int cj = -1, c_end = 0;
+  int c_t0 = 0, c_end = 0;
+  int64_t c_rows = 0;
+  bool c_dense = true;
+  // copy-out: this lane's 16-byte chunk(s) of a full tile, at tile 0 of the job,
+  // and the bytes between consecutive tiles of its plane
+  uint8_t* o_dst[C::ROUNDS];
+  int o_step[C::ROUNDS];
+#pragma unroll
+  for (int q = 0; q < C::ROUNDS; ++q) { o_dst[q] = nullptr; o_step[q] = 0; }
   uint2 msk[8];
 #pragma unroll
   for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
@@ -427,16 +490,22 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
       if (ns >= kNS) ns -= kNS;
       issue(t + (kNS - 1) * Gw, ns);
     }
-    if (t >= c_end) {  // next job: copy its descriptor to shared memory
-      cj = (cj < 0) ? find_job(p, t) : cj + 1;
-      while (cj + 1 < p.njobs && p.job[cj + 1].tile0 <= t) ++cj;
+    if (t >= c_end) {  // next job
+      const int cj = find_job(p, t);
       const EncJob& J = p.job[cj];
+      c_t0 = J.tile0;
       c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
+      c_rows = J.rows;
+      c_dense = J.slot == nullptr;
+#pragma unroll
+      for (int q = 0; q < C::ROUNDS; ++q) {
+        const int ch = q * 32 + lane;
+        if (ch < C::NA) { o_dst[q] = J.codes + 16 * ch; o_step[q] = C::RW * C::AB; }
+        else if (ch < C::NA + C::NN) { o_dst[q] = J.norms + 16 * (ch - C::NA); o_step[q] = C::RW * C::NB; }
+        else { o_dst[q] = J.hdr + 16 * (ch - C::NA - C::NN); o_step[q] = C::RW * 8; }
+      }
       if (lane == 0) {
-        wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot;
-        wj->capacity = J.capacity; wj->rows = J.rows; wj->t0 = J.tile0; wj->end = c_end;
-        wj->variant = (J.w - 1) * 4 + (J.b == 8 ? 2 : 0) + (J.mode == TAC_NORM_LOG ? 1 : 0);
-        wj->ab = C::P * J.w / 8; wj->nb = C::P * J.b / 8;
+        wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot; wj->capacity = J.capacity;
 #pragma unroll
         for (int q = 0; q < 4; ++q) wj->signs[q] = J.signs[q];
       }
@@ -445,25 +514,24 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
       for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
       __syncwarp();
     }
-    const int64_t row0 = (int64_t)(t - wj->t0) * C::RW;
-    const int nrows = (int)min((int64_t)C::RW, wj->rows - row0);
-    const int variant = wj->variant;
+    const int rel = t - c_t0;
+    const int64_t row0 = (int64_t)rel * C::RW;
+    const int64_t left = c_rows - row0;
+    const int nrows = left < C::RW ? (int)left : C::RW;
     const uint8_t* in = wsm + C::W_IN + stage * IT::BYTES;
-
-#define TAC_ENC_CASE(WW)                                                                                       \
-  case (WW - 1) * 4 + 0: tile_body<D, TIn, WW, 4, TAC_NORM_LINEAR>(in, wsm, etab, nrows, lane, msk, wj->signs); break; \
-  case (WW - 1) * 4 + 1: tile_body<D, TIn, WW, 4, TAC_NORM_LOG>(in, wsm, etab, nrows, lane, msk, wj->signs); break;    \
-  case (WW - 1) * 4 + 2: tile_body<D, TIn, WW, 8, TAC_NORM_LINEAR>(in, wsm, etab, nrows, lane, msk, wj->signs); break; \
-  case (WW - 1) * 4 + 3: tile_body<D, TIn, WW, 8, TAC_NORM_LOG>(in, wsm, etab, nrows, lane, msk, wj->signs); break;
-    switch (variant) {
-      TAC_ENC_CASE(1) TAC_ENC_CASE(2) TAC_ENC_CASE(3) TAC_ENC_CASE(4)
-      TAC_ENC_CASE(5) TAC_ENC_CASE(6) TAC_ENC_CASE(7) TAC_ENC_CASE(8)
-      default: break;
-    }
-#undef TAC_ENC_CASE
+    tile_body<D, TIn, W, B, MODE>(in, wsm, etab, nrows, lane, msk, wj->signs);
     __syncwarp();
-    warp_copy_out(wj->codes, wj->norms, wj->hdr, wj->slot, wj->capacity, wsm + C::W_ANG, wsm + C::W_NRM,
-                  wsm + C::W_HDR, row0, nrows, C::RW, wj->ab, wj->nb, lane);
+    if (c_dense && nrows == C::RW) {
+#pragma unroll
+      for (int q = 0; q < C::ROUNDS; ++q) {
+        const int ch = q * 32 + lane;
+        if (ch < C::NCH)
+          *reinterpret_cast<uint4*>(o_dst[q] + (int64_t)rel * o_step[q]) =
+              *reinterpret_cast<const uint4*>(wsm + C::W_ANG + 16 * ch);
+      }
+    } else {
+      copy_out_slow<C::AB, C::NB>(wj, wsm + C::W_ANG, wsm + C::W_NRM, wsm + C::W_HDR, row0, nrows, lane);
+    }
     stage = (stage + 1 == kNS) ? 0 : stage + 1;
   }
   cp_async_wait<0>();
@@ -472,10 +540,10 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
 // ---------------------------------------------------------------------------
 // Host-side launch helpers (called from tac_api.cu).
 // ---------------------------------------------------------------------------
-template <int D, typename TIn>
-static cudaError_t launch_encode_t(const EncParams& p, int grid_cap, cudaStream_t st) {
-  using C = Enc<D, TIn>;
-  auto kern = encode_kernel<D, TIn>;
+template <int D, typename TIn, int W, int B, int MODE>
+static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_t st) {
+  using C = Enc<D, TIn, W, B>;
+  auto kern = encode_kernel<D, TIn, W, B, MODE>;
   static int configured[64] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -496,6 +564,22 @@ static cudaError_t launch_encode_t(const EncParams& p, int grid_cap, cudaStream_
   return cudaGetLastError();
 }
 
+template <int D, typename TIn>
+static cudaError_t launch_encode_t(const EncParams& p, int w, int b, int mode, int sms, cudaStream_t st) {
+#define TAC_ENC_CASE(WW)                                                                         \
+  case (WW - 1) * 4 + 0: return launch_encode_v<D, TIn, WW, 4, TAC_NORM_LINEAR>(p, sms, st);     \
+  case (WW - 1) * 4 + 1: return launch_encode_v<D, TIn, WW, 4, TAC_NORM_LOG>(p, sms, st);        \
+  case (WW - 1) * 4 + 2: return launch_encode_v<D, TIn, WW, 8, TAC_NORM_LINEAR>(p, sms, st);     \
+  case (WW - 1) * 4 + 3: return launch_encode_v<D, TIn, WW, 8, TAC_NORM_LOG>(p, sms, st);
+  switch ((w - 1) * 4 + (b == 8 ? 2 : 0) + (mode == TAC_NORM_LOG ? 1 : 0)) {
+    TAC_ENC_CASE(1) TAC_ENC_CASE(2) TAC_ENC_CASE(3) TAC_ENC_CASE(4)
+    TAC_ENC_CASE(5) TAC_ENC_CASE(6) TAC_ENC_CASE(7) TAC_ENC_CASE(8)
+    default: break;
+  }
+#undef TAC_ENC_CASE
+  return cudaErrorInvalidValue;
+}
+
 // Instances: the build compiles this file once per (d, dtype) with
 // -DTAC_INST_D=<d> -DTAC_INST_BF16=1|-DTAC_INST_F32=1 so they compile in parallel;
 // without those flags every instance is compiled here.
@@ -509,45 +593,35 @@ static cudaError_t launch_encode_t(const EncParams& p, int grid_cap, cudaStream_
 #ifndef TAC_INST_F32
 #define TAC_INST_F32 0
 #endif
+#define TAC_ENC_INSTANCE(DD, NAME, T)                                                                 \
+  cudaError_t launch_encode_##DD##_##NAME(const EncParams& p, int w, int b, int mode, int sms,       \
+                                          cudaStream_t st) {                                         \
+    return launch_encode_t<DD, T>(p, w, b, mode, sms, st);                                           \
+  }
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 16 && TAC_INST_BF16)
-cudaError_t launch_encode_16_bf16(const EncParams& p, int sms, cudaStream_t st) {
-  return launch_encode_t<16, __nv_bfloat16>(p, sms, st);
-}
+TAC_ENC_INSTANCE(16, bf16, __nv_bfloat16)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 32 && TAC_INST_BF16)
-cudaError_t launch_encode_32_bf16(const EncParams& p, int sms, cudaStream_t st) {
-  return launch_encode_t<32, __nv_bfloat16>(p, sms, st);
-}
+TAC_ENC_INSTANCE(32, bf16, __nv_bfloat16)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 64 && TAC_INST_BF16)
-cudaError_t launch_encode_64_bf16(const EncParams& p, int sms, cudaStream_t st) {
-  return launch_encode_t<64, __nv_bfloat16>(p, sms, st);
-}
+TAC_ENC_INSTANCE(64, bf16, __nv_bfloat16)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 128 && TAC_INST_BF16)
-cudaError_t launch_encode_128_bf16(const EncParams& p, int sms, cudaStream_t st) {
-  return launch_encode_t<128, __nv_bfloat16>(p, sms, st);
-}
+TAC_ENC_INSTANCE(128, bf16, __nv_bfloat16)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 16 && TAC_INST_F32)
-cudaError_t launch_encode_16_f32(const EncParams& p, int sms, cudaStream_t st) {
-  return launch_encode_t<16, float>(p, sms, st);
-}
+TAC_ENC_INSTANCE(16, f32, float)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 32 && TAC_INST_F32)
-cudaError_t launch_encode_32_f32(const EncParams& p, int sms, cudaStream_t st) {
-  return launch_encode_t<32, float>(p, sms, st);
-}
+TAC_ENC_INSTANCE(32, f32, float)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 64 && TAC_INST_F32)
-cudaError_t launch_encode_64_f32(const EncParams& p, int sms, cudaStream_t st) {
-  return launch_encode_t<64, float>(p, sms, st);
-}
+TAC_ENC_INSTANCE(64, f32, float)
 #endif
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 128 && TAC_INST_F32)
-cudaError_t launch_encode_128_f32(const EncParams& p, int sms, cudaStream_t st) {
-  return launch_encode_t<128, float>(p, sms, st);
-}
+TAC_ENC_INSTANCE(128, f32, float)
 #endif
+#undef TAC_ENC_INSTANCE
 
 }  // namespace tac
