@@ -10,10 +10,22 @@
 namespace tac {
 
 constexpr int kThreads = 256;      // threads per CTA
+constexpr int kMinBlocks = 3;      // resident CTAs per SM the kernels are built for (24 warps)
 constexpr int kPairsPerThread = 8; // each thread owns 8 consecutive angle pairs (16 elements)
 constexpr int kMaxW = 8;           // log2 n <= 8 (n <= 256)
 constexpr int kTabEntries = 512;   // sum_{w=1..8} 2^w = 510, padded
 constexpr float kU = 5.9604644775390625e-08f;  // fp32 unit roundoff 2^-24
+
+// Lookup tables indexed by a per-pair code are replicated: entry e of copy c
+// sits at index e*R + c and lane l reads copy l % R, so the 16 lanes a 64-bit
+// shared load serves at a time spread over 16 bank pairs (conflict-free for
+// R = 16; for smaller R two or four lanes share a bank pair).  R is the largest
+// power of two <= 16 with n * R * 8 <= the byte budget.
+__host__ __device__ constexpr int tab_copies(int n, int budget) {
+  int r = 16;
+  while (r > 1 && n * r * 8 > budget) r >>= 1;
+  return r;
+}
 
 // Offset of the table for n = 2^w inside a table holding every w = 1..8 back to back.
 __host__ __device__ constexpr int tab_offset(int w) { return (1 << w) - 2; }
@@ -277,6 +289,17 @@ __device__ __forceinline__ float lg2_approx(float x) {
 }
 __device__ __forceinline__ float ex2_approx(float x) {
   float r; asm("ex2.approx.f32 %0, %1;" : "=f"(r) : "f"(x)); return r;
+}
+// Flush-to-zero forms (subnormal inputs and results read as zero): the callers
+// keep their arguments and results in the normal range.
+__device__ __forceinline__ float sqrt_ftz(float x) {
+  float r; asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x)); return r;
+}
+__device__ __forceinline__ float lg2_ftz(float x) {
+  float r; asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x)); return r;
+}
+__device__ __forceinline__ float ex2_ftz(float x) {
+  float r; asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x)); return r;
 }
 __device__ __forceinline__ float min3(float a, float b, float c) {
   float r; asm("min.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c)); return r;

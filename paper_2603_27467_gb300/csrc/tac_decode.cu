@@ -15,9 +15,9 @@
 //      (E_i, O_i) = r^_i * T[k_i] on packed fp32 pairs (FADD2/FFMA2): the low
 //      pair-index bits in registers, an intra-warp shared-memory transpose, the
 //      high bits;
-//   3. D is a sign XOR on the output bits (after bf16 round-to-nearest-even, or
-//      on fp32); rows are staged in shared memory and written with coalesced
-//      16-byte stores.
+//   3. rows are staged in shared memory (bf16 round-to-nearest-even, or fp32)
+//      and written with coalesced 16-byte stores; D is a sign XOR on the output
+//      bits of each chunk as it is stored.
 #include "tac_common.cuh"
 
 namespace tac {
@@ -48,8 +48,9 @@ struct Dec {
   static constexpr int W_TP = W_REC + kNS * REC_W;          // transpose rows
   static constexpr int W_OUT = W_TP + G::TP_W;              // output rows
   static constexpr int WARP_B = W_OUT + OT::BYTES;
-  static constexpr int OFF_TAB = kWarps * WARP_B;           // centre table of this n
-  static constexpr int SMEM = OFF_TAB + n * 8;
+  static constexpr int TABR = tab_copies(n, 16384);          // centre table copies
+  static constexpr int OFF_TAB = kWarps * WARP_B;           // centre table of this n (TABR copies)
+  static constexpr int SMEM = OFF_TAB + n * TABR * 8;
   static_assert(REC_W % 16 == 0 && W_TP % 16 == 0 && W_OUT % 16 == 0 && WARP_B % 16 == 0, "alignment");
   static_assert(32 % CPR == 0 && RW % RPQ == 0, "chunk map");
 };
@@ -124,10 +125,10 @@ __device__ __forceinline__ uint64_t load_bytes(const uint8_t* p) {
   }
 }
 
-// Decode this lane's 8 pairs of warp-tile row r and stage the output row segment.
+// Decode this lane's 8 pairs of warp-tile row r and stage the output row
+// segment (ttab: this lane's copy of the replicated centre table).
 template <int D, typename TOut, int W, int B, int MODE>
-__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab, int lane,
-                                            const uint2 (&msk)[8]) {
+__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab, int lane) {
   using C = Dec<D, TOut, W, B>;
   using G = Geo<D>;
   using OT = typename C::OT;
@@ -165,8 +166,8 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
     const uint32_t cb = (uint32_t)(acc_n >> (j * B)) & (uint32_t)Lq;
     const float f = __uint_as_float(0x3F800000u | (cb << (23 - B)));
     float rh = __fmaf_rn(f, S, base2);
-    if constexpr (MODE != TAC_NORM_LINEAR) rh = ex2_approx(rh);
-    v[j] = mul2(make_float2(rh, rh), ttab[k]);
+    if constexpr (MODE != TAC_NORM_LINEAR) rh = ex2_ftz(rh);
+    v[j] = mul2(make_float2(rh, rh), ttab[k * C::TABR]);
   }
   // Butterfly stages on pair-index bits 0..2 (this lane holds pairs 8l..8l+7).
   butterfly8<8>(v);
@@ -183,22 +184,22 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
     // Stages on pair-index bits 3..log2(P)-1 (this lane now holds pairs l + L*m).
     butterfly8<8, 8 / L>(v);
   }
-  // D, convert, stage the row: pair i = l + L*m is element pair (2i, 2i+1).
+  // Convert and stage the row (D is applied in the copy-out): pair i = l + L*m
+  // is element pair (2i, 2i+1).
   uint8_t* orow = wsm + C::W_OUT + r * OT::STRIDE + 2 * C::ESZ * l;
 #pragma unroll
   for (int m = 0; m < 8; ++m) {
     if constexpr (C::ESZ == 2) {
       const __nv_bfloat162 bb = __floats2bfloat162_rn(v[m].x, v[m].y);
-      *reinterpret_cast<uint32_t*>(orow + 4 * L * m) = (*reinterpret_cast<const uint32_t*>(&bb)) ^ msk[m].x;
+      *reinterpret_cast<__nv_bfloat162*>(orow + 4 * L * m) = bb;
     } else {
-      *reinterpret_cast<uint2*>(orow + 8 * L * m) =
-          make_uint2(__float_as_uint(v[m].x) ^ msk[m].x, __float_as_uint(v[m].y) ^ msk[m].y);
+      *reinterpret_cast<float2*>(orow + 8 * L * m) = v[m];
     }
   }
 }
 
 template <int D, typename TOut, int W, int B, int MODE>
-__global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_constant__ DecParams p) {
+__global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecParams p) {
   using C = Dec<D, TOut, W, B>;
   using OT = typename C::OT;
   extern __shared__ __align__(128) uint8_t smem[];
@@ -210,27 +211,34 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
   const float sc = sqrtf(2.f / (float)D);  // sqrt2 / sqrt(d)
   for (int k = tid; k < C::n; k += kThreads) {
     const float2 cs = cos_sin_q8(centre_q8(k, C::n), C::n);  // (cos psi, sin psi), psi = phi + pi/4
-    ttab[k] = make_float2(sc * cs.y, sc * cs.x);
+#pragma unroll
+    for (int c = 0; c < C::TABR; ++c) ttab[k * C::TABR + c] = make_float2(sc * cs.y, sc * cs.x);
   }
   __syncthreads();
 
-  const int Gw = gridDim.x * kWarps;
-  int t = blockIdx.x * kWarps + warp;
-  if (t >= p.ntiles) return;
+  // Each warp owns a contiguous range of warp tiles (balanced to +-1 tile).
+  const int Gw = gridDim.x * kWarps, gw = blockIdx.x * kWarps + warp;
+  const int per = p.ntiles / Gw, extra = p.ntiles % Gw;
+  int t = gw * per + min(gw, extra);
+  const int t_end = t + per + (gw < extra ? 1 : 0);
+  if (t >= t_end) return;
   uint8_t* wsm = smem + warp * C::WARP_B;
 
-  // ---- prefetch cursor: the job of the next warp tile whose records are staged ----
-  int pj = find_job(p, t);
-  int p_t0 = 0, p_end = 0;
-  int64_t p_rows = 0;
+  // ---- prefetch cursor: the next warp tile whose records are staged ----
+  int it = t;                    // next tile to issue
+  int pj = find_job(p, t);       // its job
+  int p_end = 0;
+  int64_t i_row0 = 0;            // the tile's first row within its job
+  int64_t i_left = 0;            // rows of the job from i_row0
   bool p_dense = true;
-  const uint8_t* i_src[C::ROUNDS];  // this lane's record chunk(s) at tile 0 of the job
+  const uint8_t* i_src[C::ROUNDS];  // this lane's record chunk(s) of the tile
   int i_step[C::ROUNDS];            // bytes between consecutive tiles of its plane
   auto set_issue_job = [&]() {
     const DecJob& J = p.job[pj];
-    p_t0 = J.tile0;
     p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
-    p_rows = J.rows;
+    const int rel = it - J.tile0;
+    i_row0 = (int64_t)rel * C::RW;
+    i_left = J.rows - i_row0;
     p_dense = J.slot == nullptr;
 #pragma unroll
     for (int q = 0; q < C::ROUNDS; ++q) {
@@ -238,81 +246,105 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
       if (ch < C::NA) { i_src[q] = J.codes + 16 * ch; i_step[q] = C::RW * C::AB; }
       else if (ch < C::NA + C::NN) { i_src[q] = J.norms + 16 * (ch - C::NA); i_step[q] = C::RW * C::NB; }
       else { i_src[q] = J.hdr + 16 * (ch - C::NA - C::NN); i_step[q] = C::RW * 8; }
+      i_src[q] += (int64_t)rel * i_step[q];
     }
   };
   set_issue_job();
-  auto issue = [&](int tt, int stg) {
-    if (tt < p.ntiles) {
-      while (tt >= p_end) {
-        ++pj;
+  auto issue = [&](int stg) {
+    if (it < t_end) {
+      if (it >= p_end) {  // a warp's tiles only move forward
+        while (it >= p_end) { ++pj; p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles; }
         set_issue_job();
       }
-      const int rel = tt - p_t0;
-      const int64_t row0 = (int64_t)rel * C::RW;
       uint8_t* stage = wsm + C::W_REC + stg * C::REC_W;
-      if (p_dense && row0 + C::RW <= p_rows) {
+      if (p_dense && i_left >= C::RW) {
 #pragma unroll
         for (int q = 0; q < C::ROUNDS; ++q) {
           const int ch = q * 32 + lane;
-          if (ch < C::NCH) cp_async16(stage + 16 * ch, i_src[q] + (int64_t)rel * i_step[q], 16);
+          if (ch < C::NCH) cp_async16(stage + 16 * ch, i_src[q], 16);
         }
       } else {
-        stage_records_slow<C::AB, C::NB, C::R_NRM, C::R_HDR>(p.job[pj], row0, (int)min((int64_t)C::RW, p_rows - row0),
+        stage_records_slow<C::AB, C::NB, C::R_NRM, C::R_HDR>(p.job[pj], i_row0, (int)min((int64_t)C::RW, i_left),
                                                             stage, lane);
       }
+#pragma unroll
+      for (int q = 0; q < C::ROUNDS; ++q) i_src[q] += i_step[q];
+      i_row0 += C::RW;
+      i_left -= C::RW;
+      ++it;
     }
     cp_async_commit();
   };
 #pragma unroll
-  for (int s = 0; s < kNS - 1; ++s) issue(t + s * Gw, s);
+  for (int s = 0; s < kNS - 1; ++s) issue(s);
 
   // ---- compute cursor ----
-  int c_t0 = 0, c_end = 0;
-  int64_t c_rows = 0, c_sb = 0;
+  int c_end = t;                 // first tile after the current job (forces a job load)
+  int64_t c_left = 0;            // rows of the job from the current tile's row 0
+  int64_t c_step = 0;            // output bytes between consecutive tiles (RW rows)
+  int64_t c_qstep = 0;           // output bytes between a lane's consecutive chunks (RPQ rows)
   // Output chunk q of a lane is row q*RPQ + lane/CPR, bytes (lane % CPR)*16.
   const int lane_cr = lane / C::CPR;
   const uint8_t* const out_src = wsm + C::W_OUT + lane_cr * OT::STRIDE + (lane % C::CPR) * 16;
-  uint8_t* o_dst = nullptr;  // this lane's first output chunk of the job's row 0
-  uint2 msk[8];
-#pragma unroll
-  for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
+  uint8_t* o_dst = nullptr;      // this lane's first output chunk of the current tile
+  uint4 dmask = make_uint4(0u, 0u, 0u, 0u);  // D of Sec. 2 on this lane's 16 output bytes (sign bits)
 
   int stage = 0;
-  for (; t < p.ntiles; t += Gw) {
+  for (; t < t_end; ++t) {
     cp_async_wait<kNS - 2>();   // this warp tile's records have landed
     __syncwarp();               // ... and every lane is done with the previous tile
     {
       int ns = stage + kNS - 1;
       if (ns >= kNS) ns -= kNS;
-      issue(t + (kNS - 1) * Gw, ns);
+      issue(ns);
     }
     if (t >= c_end) {  // next job
       const int cj = find_job(p, t);
       const DecJob& J = p.job[cj];
-      c_t0 = J.tile0;
       c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
-      c_rows = J.rows;
-      c_sb = J.stride * C::ESZ;
-      o_dst = reinterpret_cast<uint8_t*>(J.y) + lane_cr * c_sb + (lane % C::CPR) * 16;
-      const int l = lane % C::L;
+      const int64_t row0 = (int64_t)(t - J.tile0) * C::RW;
+      c_left = J.rows - row0;
+      const int64_t sb = J.stride * C::ESZ;
+      c_step = C::RW * sb;
+      c_qstep = C::RPQ * sb;
+      o_dst = reinterpret_cast<uint8_t*>(J.y) + (row0 + lane_cr) * sb + (lane % C::CPR) * 16;
+      // the lane's chunk holds elements e0 .. e0 + 16/ESZ - 1 of every row it writes
+      const int e0 = (lane % C::CPR) * (16 / C::ESZ);
+      uint32_t mw[4];
 #pragma unroll
-      for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
+      for (int q = 0; q < 4; ++q) {
+        if constexpr (C::ESZ == 2) {
+          const int e = e0 + 2 * q;
+          mw[q] = (((J.signs[e >> 5] >> (e & 31)) & 1u) << 15) | (((J.signs[(e + 1) >> 5] >> ((e + 1) & 31)) & 1u) << 31);
+        } else {
+          const int e = e0 + q;
+          mw[q] = ((J.signs[e >> 5] >> (e & 31)) & 1u) << 31;
+        }
+      }
+      dmask = make_uint4(mw[0], mw[1], mw[2], mw[3]);
     }
     const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;
-    decode_body<D, TOut, W, B, MODE>(rec, wsm, ttab, lane, msk);
+    decode_body<D, TOut, W, B, MODE>(rec, wsm, ttab + (lane % C::TABR), lane);
     __syncwarp();
-    // Write the warp tile's rows: 16-byte chunks, coalesced.
-    {
-      const int64_t row0 = (int64_t)(t - c_t0) * C::RW;
-      const int64_t left = c_rows - row0 - lane_cr;
-      uint8_t* dst = o_dst + row0 * c_sb;
+    // Apply D and write the warp tile's rows: 16-byte chunks, coalesced.
+    if (c_left >= C::RW) {
 #pragma unroll
       for (int q = 0; q < C::CHUNKS; ++q) {
-        if (q * C::RPQ < left)
-          *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(out_src + q * C::RPQ * OT::STRIDE);
-        dst += C::RPQ * c_sb;
+        uint4 v = *reinterpret_cast<const uint4*>(out_src + q * C::RPQ * OT::STRIDE);
+        v.x ^= dmask.x; v.y ^= dmask.y; v.z ^= dmask.z; v.w ^= dmask.w;
+        *reinterpret_cast<uint4*>(o_dst + q * c_qstep) = v;
       }
+    } else {
+#pragma unroll
+      for (int q = 0; q < C::CHUNKS; ++q)
+        if (q * C::RPQ + lane_cr < c_left) {
+          uint4 v = *reinterpret_cast<const uint4*>(out_src + q * C::RPQ * OT::STRIDE);
+          v.x ^= dmask.x; v.y ^= dmask.y; v.z ^= dmask.z; v.w ^= dmask.w;
+          *reinterpret_cast<uint4*>(o_dst + q * c_qstep) = v;
+        }
     }
+    o_dst += c_step;
+    c_left -= C::RW;
     stage = (stage + 1 == kNS) ? 0 : stage + 1;
   }
   cp_async_wait<0>();

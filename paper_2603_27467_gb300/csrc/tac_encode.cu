@@ -79,8 +79,9 @@ struct Enc {
   static constexpr int W_HDR = W_NRM + RW * NB;
   static constexpr int W_JOB = W_HDR + RW * 8;              // current job (WarpJob)
   static constexpr int WARP_B = W_JOB + 64;
-  static constexpr int OFF_TAB = kWarps * WARP_B;           // fp32 edge table of this n
-  static constexpr int SMEM = OFF_TAB + n * 8;
+  static constexpr int TABR = tab_copies(n, 8192);           // edge table copies
+  static constexpr int OFF_TAB = kWarps * WARP_B;           // fp32 edge table of this n (TABR copies)
+  static constexpr int SMEM = OFF_TAB + n * TABR * 8;
   static_assert((RW * AB) % 16 == 0 && (RW * NB) % 16 == 0 && (RW * 8) % 16 == 0, "record segments");
   static_assert(W_TP % 16 == 0 && W_ANG % 16 == 0 && W_JOB % 16 == 0 && WARP_B % 16 == 0, "alignment");
   static_assert(32 % CPR == 0 && RW % RPQ == 0, "chunk map");
@@ -122,14 +123,49 @@ __device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
   e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
 }
 
+// Candidate edge for the pair (E, O) (butterfly halves, y = (E + O, E - O))
+// and n = 2^W: Alg. 1's angle theta = pi/4 - angle(E, O) from the
+// octant-reduced arctangent polynomial, in bins, floored (M + n/8 - angle,
+// rounded down onto the integer grid of M = 1.5 * 2^23).  The true bin is the
+// candidate or the next one whenever the polynomial's error (0.0038 rad) is
+// below half a bin, i.e. for every n <= 256.
+template <int W>
+__device__ __forceinline__ int candidate_edge(float E, float O) {
+  constexpr int n = 1 << W;
+  constexpr float nb = (float)n * 0.15915494309189535f;  // bins per radian
+  constexpr float c1 = (0.78539816f + 0.273f) * nb;       // atan(t) ~ t (pi/4 + 0.273 (1 - t))
+  constexpr float c2 = 0.273f * nb;
+  const float aE = fabsf(E), aO = fabsf(O);
+  const float mx = fmaxf(aE, aO), mn = fminf(aE, aO);
+  const float t = mn * rcp_approx(mx);
+  const float phi = t * __fmaf_rn(t, -c2, c1);                 // octant angle, bins
+  float fb = (aO > aE) ? (0.25f * n - phi) : phi;              // angle of (|E|, |O|)
+  fb = (E < 0.f) ? (0.5f * n - fb) : fb;                       // angle of (E, |O|)
+  const float ab = __uint_as_float(__float_as_uint(fb) ^ (__float_as_uint(O) & 0x80000000u));
+  return __float_as_int(__fadd_rd(12582912.0f + 0.125f * n, -ab)) & (n - 1);
+}
+
+// Alg. 1 bin of the pair (E, O) for n = 2^W by the edge test: the candidate
+// edge, then the sign of the cross product with the edge direction (et: this
+// lane's copy of the replicated table, R copies).  Returns k; m is the signed
+// cross product (its magnitude is the certification margin).
+template <int W, int R>
+__device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et, float& m) {
+  constexpr int n = 1 << W;
+  const int e = candidate_edge<W>(E, O);
+  const float2 dir = et[e * R];
+  m = __fmaf_rn(E, dir.x, -__fmul_rn(O, dir.y));
+  return (uint32_t)(e + 1 + (__float_as_int(m) >> 31)) & (uint32_t)(n - 1);
+}
+
 // Exact re-decision of pair i of warp-tile row rr by the whole warp (all lanes
 // call it with the same arguments); returns k in every lane.  E_i = sum_j
 // +-x_2j and O_i = sum_j +-x_2j+1 (each term an exactly representable signed
 // input element) are accumulated as double-float values with TwoSum; their
 // relative error is of order 64 u^2, far inside the 1e-5 rad band the angle
-// parity tolerates.  The candidate edge comes from an fp32 atan2 of the sums
-// (an error near a bin centre picks a neighbouring edge, whose test gives the
-// same bin), the edge test m = E cos psi - O sin psi is evaluated in
+// parity tolerates.  The candidate edge comes from the polynomial on the sums
+// rounded to fp32 (scaled by a power of two when tiny, so the reciprocal sees
+// a normal number), the edge test m = E cos psi - O sin psi is evaluated in
 // double-float against the double-float edge direction.
 template <int D, typename TIn, int W, int B>
 __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uint8_t* in, int rr, int i,
@@ -171,8 +207,11 @@ __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uin
   two_sum(eh, el, eh, el);  // renormalize: eh == 0 now means E == 0
   two_sum(oh, ol, oh, ol);
   if (eh == 0.f && oh == 0.f) return 0;  // pair (0, 0) -> bin 0
-  const float th = atan2f(__fsub_rn(eh, oh), __fadd_rn(eh, oh));
-  const int e = ((int)floorf(th * ((float)n * 0.15915494309189535f))) & (n - 1);
+  if (fmaxf(fabsf(eh), fabsf(oh)) < 1e-30f) {  // exact power-of-two rescale
+    eh *= 18446744073709551616.f; el *= 18446744073709551616.f;
+    oh *= 18446744073709551616.f; ol *= 18446744073709551616.f;
+  }
+  const int e = candidate_edge<W>(eh, oh);
   const cx::DF4 dir = g_edge_df.v[tab_offset(W) + e];
   const float p1 = __fmul_rn(eh, dir.ch), q1 = __fmaf_rn(eh, dir.ch, -p1);
   const float p2 = __fmul_rn(oh, dir.sh), q2 = __fmaf_rn(oh, dir.sh, -p2);
@@ -197,31 +236,6 @@ __device__ __forceinline__ void patch_code(uint8_t* rec, int i, int k) {
   v = (v & ~mask) | ((uint32_t)k << sh);
   rec[b0] = (uint8_t)v;
   if (sh + W > 8) rec[b0 + 1] = (uint8_t)(v >> 8);
-}
-
-// Alg. 1 bin of the pair (E, O) (butterfly halves, y = (E + O, E - O)) for
-// n = 2^W by the edge test: candidate edge from the arctangent polynomial, then
-// the sign of the cross product with the edge direction.  Returns k; m is the
-// signed cross product (its magnitude is the certification margin).
-template <int W>
-__device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et, float& m) {
-  constexpr int n = 1 << W;
-  constexpr float nb = (float)n * 0.15915494309189535f;  // bins per radian
-  constexpr float c1 = (0.78539816f + 0.273f) * nb;       // atan(t) ~ t (pi/4 + 0.273 (1 - t))
-  constexpr float c2 = 0.273f * nb;
-  const float aE = fabsf(E), aO = fabsf(O);
-  const float mx = fmaxf(aE, aO), mn = fminf(aE, aO);
-  const float t = mn * rcp_approx(mx);
-  const float phi = t * __fmaf_rn(t, -c2, c1);                 // octant angle, bins
-  float fb = (aO > aE) ? (0.25f * n - phi) : phi;              // angle of (|E|, |O|)
-  fb = (E < 0.f) ? (0.5f * n - fb) : fb;                       // angle of (E, |O|)
-  const float ab = __uint_as_float(__float_as_uint(fb) ^ (__float_as_uint(O) & 0x80000000u));
-  // theta = pi/4 - angle(E, O): round(v - 1/2) is the candidate edge index
-  const float vm = (0.125f * n - 0.5f) - ab;
-  const int e = __float_as_int(vm + 12582912.0f) & (n - 1);
-  const float2 dir = et[e];
-  m = __fmaf_rn(E, dir.x, -__fmul_rn(O, dir.y));
-  return (uint32_t)(e + 1 + (__float_as_int(m) >> 31)) & (uint32_t)(n - 1);
 }
 
 // Encode this lane's 8 pairs of warp-tile row r (lane l of the row) and stage
@@ -282,10 +296,12 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   const float lmin_s = min3(min3(s[0], s[1], s[2]), min3(s[3], s[4], s[5]), fminf(s[6], s[7]));
   float smin = lmin_s;
   float smax = max3(max3(s[0], s[1], s[2]), max3(s[3], s[4], s[5]), fmaxf(s[6], s[7]));
+  float ssum = ((s[0] + s[1]) + (s[2] + s[3])) + ((s[4] + s[5]) + (s[6] + s[7]));
 #pragma unroll
   for (int off = 1; off < L; off <<= 1) {
     smin = fminf(smin, __shfl_xor_sync(0xffffffffu, smin, off));
     smax = fmaxf(smax, __shfl_xor_sync(0xffffffffu, smax, off));
+    ssum += __shfl_xor_sync(0xffffffffu, ssum, off);
   }
   const bool zero_row = !(smax > 0.f);
 
@@ -310,26 +326,43 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
                    sc, 0.5f);
     if (!(hmax > hmin) || !(sc <= 3.0e38f)) { qs = 0.f; qo = 0.5f; }
   }
-  // Certification bound: |dE|, |dO| <= (log2 d - 1) u ||x||_1, ||x||_1 <= sqrt(d smax);
-  // edge direction (<= 1 ulp), product and fma add <= 4 u (|E| + |O|) <= 4 u sqrt(2 smax).
+  // Certification bound on the cross product m = E c - O s.  The butterfly's
+  // log2 d - 1 rounded stages give |dE| <= (log2 d - 1) u ||x_even||_1 and
+  // |dO| <= (log2 d - 1) u ||x_odd||_1 (first order), so with c^2 + s^2 = 1
+  //   |dm| <= (log2 d - 1) u sqrt(||x_even||_1^2 + ||x_odd||_1^2)
+  //        <= (log2 d - 1) u sqrt(d/2) ||x||_2 = (log2 d - 1) u sqrt(S),
+  // S = sum_i (E_i^2 + O_i^2) = d ||x||_2^2 / 2 (the factor 1.01 covers the
+  // rounding of the computed S and the second-order terms).  The edge direction
+  // (<= 1 ulp), the product and the fma add <= 4 u (|E| + |O|) <= 4 u sqrt(2 smax).
   const float rmx = sqrt_approx(smax);
-  const float ty = (float)(G::LOGD - 1) * kU * 1.002f * sqrt_approx((float)D) * rmx;
+  const float ty = (float)(G::LOGD - 1) * kU * 1.01f * sqrt_approx(ssum);
   const float tau = ty + 5.f * kU * 1.4143f * rmx;
+  // Per-pair norm functions run on s * sigma, sigma = 4^-k an exact power of two
+  // with smax * sigma in [1, 4): sqrt(s) = 2^k sqrt(s sigma), log2 s =
+  // log2(s sigma) + 2k, so the flush-to-zero hardware forms see normal numbers
+  // (pairs below the log floor are clamped to it first).
+  const int ek = ((int)((__float_as_uint(smax) >> 23) & 0xFFu) - 127) >> 1;
+  const int kk = ek < -62 ? -62 : (ek > 63 ? 63 : ek);
+  const float sigma = __uint_as_float((uint32_t)(127 - 2 * kk) << 23);
+  if constexpr (MODE == TAC_NORM_LINEAR) qs *= __uint_as_float((uint32_t)(127 + kk) << 23);
+  else qo = __fmaf_rn((float)(2 * kk), qs, qo);
+  const float sfl = sfloor * sigma;
   // Pairs whose norm is so small that the fp32 angle may be off by a quarter bin
   // are re-decided too: sqrt(s) < 4 n ty / pi.
   const float rthr = ty * (4.f * (float)n / 3.14159265f);
   const float sthr = rthr * rthr;
 
   // ---- pass 2: angle codes (Alg. 1), norm codes (Eq. 2), packing ----
-  uint32_t alo = 0, ahi = 0, nlo = 0, nhi = 0, fm = 0;
+  uint32_t alo = 0, ahi = 0, nlo = 0, nhi = 0;
+  float mmin = __int_as_float(0x7f800000);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     float m;
-    const uint32_t k = edge_test<W>(v[j].x, v[j].y, et, m);
-    fm |= (fabsf(m) < tau ? 1u : 0u) << j;      // not certified by the bound
+    const uint32_t k = edge_test<W, C::TABR>(v[j].x, v[j].y, et, m);
+    mmin = fminf(mmin, fabsf(m));
     float f;
-    if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_approx(s[j]);
-    else f = lg2_approx(fmaxf(s[j], sfloor));
+    if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_ftz(s[j] * sigma);
+    else f = lg2_ftz(fmaxf(s[j] * sigma, sfl));
     const uint32_t c = min(__float2uint_rd(__fmaf_rn(f, qs, qo)), (uint32_t)Lq);
     const int sa = j * W, sn = j * B;
     if (sa + W <= 32) alo |= k << sa;
@@ -337,11 +370,16 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
     else { alo |= k << sa; ahi |= k >> (32 - sa); }
     if (sn < 32) nlo |= c << sn; else nhi |= c << (sn - 32);
   }
-  if (lmin_s < sthr) {  // rare: small-norm pairs
+  uint32_t fm = 0;
+  if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; }
+  else if (mmin < tau || lmin_s < sthr) {  // rare: name the uncertified pairs
 #pragma unroll
-    for (int j = 0; j < 8; ++j) fm |= (s[j] < sthr ? 1u : 0u) << j;
+    for (int j = 0; j < 8; ++j) {
+      float m;
+      edge_test<W, C::TABR>(v[j].x, v[j].y, et, m);
+      if (fabsf(m) < tau || s[j] < sthr) fm |= 1u << j;
+    }
   }
-  if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; fm = 0; }
   if (!live) fm = 0;
 
   // ---- stage the records ----
@@ -408,7 +446,7 @@ __device__ __noinline__ void copy_out_slow(const WarpJob* wj, const uint8_t* san
 }
 
 template <int D, typename TIn, int W, int B, int MODE>
-__global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_constant__ EncParams p) {
+__global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __grid_constant__ EncParams p) {
   using C = Enc<D, TIn, W, B>;
   using IT = typename C::IT;
   extern __shared__ __align__(128) uint8_t smem[];
@@ -417,62 +455,80 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
 
   // fp32 edge table of this n (shared by the CTA).
   float2* etab = reinterpret_cast<float2*>(smem + C::OFF_TAB);
-  for (int e = tid; e < C::n; e += kThreads) etab[e] = cos_sin_q8(edge_q8(e, C::n), C::n);
+  for (int e = tid; e < C::n; e += kThreads) {
+    const float2 cs = cos_sin_q8(edge_q8(e, C::n), C::n);
+#pragma unroll
+    for (int c = 0; c < C::TABR; ++c) etab[e * C::TABR + c] = cs;
+  }
   __syncthreads();
 
-  const int Gw = gridDim.x * kWarps;
-  int t = blockIdx.x * kWarps + warp;
-  if (t >= p.ntiles) return;
+  // Each warp owns a contiguous range of warp tiles (balanced to +-1 tile), so
+  // it meets a new job at most a few times per launch and walks its planes
+  // with pointer increments.
+  const int Gw = gridDim.x * kWarps, gw = blockIdx.x * kWarps + warp;
+  const int per = p.ntiles / Gw, extra = p.ntiles % Gw;
+  int t = gw * per + min(gw, extra);
+  const int t_end = t + per + (gw < extra ? 1 : 0);
+  if (t >= t_end) return;
   uint8_t* wsm = smem + warp * C::WARP_B;
 
-  // ---- prefetch cursor: the job of the next warp tile to load ----
+  // ---- prefetch cursor: the next warp tile to load ----
   // Lane chunk q of a tile is row q*RPQ + lane/CPR, bytes (lane % CPR)*16.
   const int lane_cr = lane / C::CPR;
   uint8_t* const in_dst = wsm + C::W_IN + lane_cr * IT::STRIDE + (lane % C::CPR) * 16;
-  int pj = find_job(p, t);
-  int p_t0 = 0, p_end = 0;
-  int64_t p_left0 = 0, p_sb = 0;     // rows of the job from this lane's first row; row stride (bytes)
-  const uint8_t* p_x = nullptr;      // job base (a valid address for zero-fill chunks)
-  const uint8_t* p_src = nullptr;    // this lane's first chunk of the job's row 0
+  int it = t;                    // next tile to issue
+  int pj = find_job(p, t);       // its job
+  int p_end = 0;                 // first tile after that job
+  int64_t i_left = 0;            // rows of the job from the tile's row 0
+  int64_t i_step = 0;            // bytes between consecutive tiles (RW rows)
+  int64_t i_qstep = 0;           // bytes between a lane's consecutive chunks (RPQ rows)
+  const uint8_t* i_src = nullptr;  // this lane's first chunk of the tile
   auto set_issue_job = [&]() {
     const EncJob& J = p.job[pj];
-    p_t0 = J.tile0;
     p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles;
-    p_left0 = J.rows - lane_cr;
-    p_sb = J.stride * C::ESZ;
-    p_x = reinterpret_cast<const uint8_t*>(J.x);
-    p_src = p_x + lane_cr * p_sb + (lane % C::CPR) * 16;
+    const int64_t sb = J.stride * C::ESZ;
+    const int64_t row0 = (int64_t)(it - J.tile0) * C::RW;
+    i_left = J.rows - row0;
+    i_step = C::RW * sb;
+    i_qstep = C::RPQ * sb;
+    i_src = reinterpret_cast<const uint8_t*>(J.x) + (row0 + lane_cr) * sb + (lane % C::CPR) * 16;
   };
   set_issue_job();
-  auto issue = [&](int tt, int stg) {
-    if (tt < p.ntiles) {
-      while (tt >= p_end) {  // monotone: a warp's tiles only move forward
-        ++pj;
+  auto issue = [&](int stg) {
+    if (it < t_end) {
+      if (it >= p_end) {  // a warp's tiles only move forward
+        while (it >= p_end) { ++pj; p_end = (pj + 1 < p.njobs) ? p.job[pj + 1].tile0 : p.ntiles; }
         set_issue_job();
       }
-      const int64_t row0 = (int64_t)(tt - p_t0) * C::RW;
-      const int64_t left = p_left0 - row0;
-      const uint8_t* src = p_src + row0 * p_sb;
       uint8_t* dst = in_dst + stg * IT::BYTES;
+      if (i_left >= C::RW) {
 #pragma unroll
-      for (int q = 0; q < C::CHUNKS; ++q) {
-        const bool ok = q * C::RPQ < left;
-        cp_async16(dst + q * C::RPQ * IT::STRIDE, ok ? src : p_x, ok ? 16 : 0);
-        src += C::RPQ * p_sb;
+        for (int q = 0; q < C::CHUNKS; ++q) cp_async16(dst + q * C::RPQ * IT::STRIDE, i_src + q * i_qstep, 16);
+      } else {  // the job's last tile: rows past its end are zero-filled
+        const uint8_t* x0 = reinterpret_cast<const uint8_t*>(p.job[pj].x);
+#pragma unroll
+        for (int q = 0; q < C::CHUNKS; ++q) {
+          const bool ok = q * C::RPQ + lane_cr < i_left;
+          cp_async16(dst + q * C::RPQ * IT::STRIDE, ok ? i_src + q * i_qstep : x0, ok ? 16 : 0);
+        }
       }
+      i_src += i_step;
+      i_left -= C::RW;
+      ++it;
     }
     cp_async_commit();
   };
 #pragma unroll
-  for (int s = 0; s < kNS - 1; ++s) issue(t + s * Gw, s);
+  for (int s = 0; s < kNS - 1; ++s) issue(s);
 
   // ---- compute cursor ----
   WarpJob* wj = reinterpret_cast<WarpJob*>(wsm + C::W_JOB);
-  int c_t0 = 0, c_end = 0;
-  int64_t c_rows = 0;
+  int c_end = t;                 // first tile after the current job (forces a job load)
+  int64_t c_row0 = 0;            // the tile's first row within its job
+  int64_t c_left = 0;            // rows of the job from c_row0
   bool c_dense = true;
-  // copy-out: this lane's 16-byte chunk(s) of a full tile, at tile 0 of the job,
-  // and the bytes between consecutive tiles of its plane
+  // copy-out: this lane's 16-byte chunk(s) of the current tile and the bytes
+  // between consecutive tiles of its plane
   uint8_t* o_dst[C::ROUNDS];
   int o_step[C::ROUNDS];
 #pragma unroll
@@ -482,20 +538,21 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
   for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
 
   int stage = 0;
-  for (; t < p.ntiles; t += Gw) {
+  for (; t < t_end; ++t) {
     cp_async_wait<kNS - 2>();   // this warp tile has landed
     __syncwarp();               // ... and every lane is done with the previous one
     {
       int ns = stage + kNS - 1;
       if (ns >= kNS) ns -= kNS;
-      issue(t + (kNS - 1) * Gw, ns);
+      issue(ns);
     }
     if (t >= c_end) {  // next job
       const int cj = find_job(p, t);
       const EncJob& J = p.job[cj];
-      c_t0 = J.tile0;
       c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
-      c_rows = J.rows;
+      const int rel = t - J.tile0;
+      c_row0 = (int64_t)rel * C::RW;
+      c_left = J.rows - c_row0;
       c_dense = J.slot == nullptr;
 #pragma unroll
       for (int q = 0; q < C::ROUNDS; ++q) {
@@ -503,6 +560,7 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
         if (ch < C::NA) { o_dst[q] = J.codes + 16 * ch; o_step[q] = C::RW * C::AB; }
         else if (ch < C::NA + C::NN) { o_dst[q] = J.norms + 16 * (ch - C::NA); o_step[q] = C::RW * C::NB; }
         else { o_dst[q] = J.hdr + 16 * (ch - C::NA - C::NN); o_step[q] = C::RW * 8; }
+        o_dst[q] += (int64_t)rel * o_step[q];
       }
       if (lane == 0) {
         wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot; wj->capacity = J.capacity;
@@ -514,24 +572,24 @@ __global__ void __launch_bounds__(kThreads, 3) encode_kernel(const __grid_consta
       for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
       __syncwarp();
     }
-    const int rel = t - c_t0;
-    const int64_t row0 = (int64_t)rel * C::RW;
-    const int64_t left = c_rows - row0;
-    const int nrows = left < C::RW ? (int)left : C::RW;
+    const int nrows = c_left < C::RW ? (int)c_left : C::RW;
     const uint8_t* in = wsm + C::W_IN + stage * IT::BYTES;
-    tile_body<D, TIn, W, B, MODE>(in, wsm, etab, nrows, lane, msk, wj->signs);
+    tile_body<D, TIn, W, B, MODE>(in, wsm, etab + (lane % C::TABR), nrows, lane, msk, wj->signs);
     __syncwarp();
     if (c_dense && nrows == C::RW) {
 #pragma unroll
       for (int q = 0; q < C::ROUNDS; ++q) {
         const int ch = q * 32 + lane;
         if (ch < C::NCH)
-          *reinterpret_cast<uint4*>(o_dst[q] + (int64_t)rel * o_step[q]) =
-              *reinterpret_cast<const uint4*>(wsm + C::W_ANG + 16 * ch);
+          *reinterpret_cast<uint4*>(o_dst[q]) = *reinterpret_cast<const uint4*>(wsm + C::W_ANG + 16 * ch);
       }
     } else {
-      copy_out_slow<C::AB, C::NB>(wj, wsm + C::W_ANG, wsm + C::W_NRM, wsm + C::W_HDR, row0, nrows, lane);
+      copy_out_slow<C::AB, C::NB>(wj, wsm + C::W_ANG, wsm + C::W_NRM, wsm + C::W_HDR, c_row0, nrows, lane);
     }
+#pragma unroll
+    for (int q = 0; q < C::ROUNDS; ++q) o_dst[q] += o_step[q];
+    c_row0 += C::RW;
+    c_left -= C::RW;
     stage = (stage + 1 == kNS) ? 0 : stage + 1;
   }
   cp_async_wait<0>();
