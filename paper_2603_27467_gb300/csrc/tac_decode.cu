@@ -15,9 +15,9 @@
 //      (E_i, O_i) = r^_i * T[k_i] on packed fp32 pairs (FADD2/FFMA2): the low
 //      pair-index bits in registers, an intra-warp shared-memory transpose, the
 //      high bits;
-//   3. rows are staged in shared memory (bf16 round-to-nearest-even, or fp32)
-//      and written with coalesced 16-byte stores; D is a sign XOR on the output
-//      bits of each chunk as it is stored.
+//   3. D is a sign XOR on the output bits (after bf16 round-to-nearest-even, or
+//      on fp32); each lane stores its pairs straight from registers: the L
+//      lanes of a row write L consecutive pairs, whole 32-byte sectors.
 #include "tac_common.cuh"
 
 namespace tac {
@@ -27,7 +27,6 @@ constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles of recor
 template <int D, typename TOut, int W, int B>
 struct Dec {
   using G = Geo<D>;
-  using OT = RowTile<D, (int)sizeof(TOut)>;
   static constexpr int P = G::P, L = G::L, RW = G::RW;
   static constexpr int ESZ = (int)sizeof(TOut);
   static constexpr int n = 1 << W;
@@ -41,18 +40,14 @@ struct Dec {
   static constexpr int R_NRM = RW * AB;
   static constexpr int R_HDR = R_NRM + RW * NB;
   static constexpr int REC_W = R_HDR + RW * 8 + 16;         // + slack for 3-word angle reads
-  // Output chunk map: 32 consecutive 16-byte chunks cover RPQ rows.
-  static constexpr int CPR = OT::CPR, RPQ = 32 / CPR, CHUNKS = OT::CHUNKS;
   // per-warp shared memory region
   static constexpr int W_REC = 0;                           // kNS record stages
   static constexpr int W_TP = W_REC + kNS * REC_W;          // transpose rows
-  static constexpr int W_OUT = W_TP + G::TP_W;              // output rows
-  static constexpr int WARP_B = W_OUT + OT::BYTES;
+  static constexpr int WARP_B = W_TP + G::TP_W;
   static constexpr int TABR = tab_copies(n, 16384);          // centre table copies
   static constexpr int OFF_TAB = kWarps * WARP_B;           // centre table of this n (TABR copies)
   static constexpr int SMEM = OFF_TAB + n * TABR * 8;
-  static_assert(REC_W % 16 == 0 && W_TP % 16 == 0 && W_OUT % 16 == 0 && WARP_B % 16 == 0, "alignment");
-  static_assert(32 % CPR == 0 && RW % RPQ == 0, "chunk map");
+  static_assert(REC_W % 16 == 0 && W_TP % 16 == 0 && WARP_B % 16 == 0, "alignment");
 };
 
 // Stage the records of a tail tile (nrows < RW) or of gathered slots into
@@ -125,13 +120,14 @@ __device__ __forceinline__ uint64_t load_bytes(const uint8_t* p) {
   }
 }
 
-// Decode this lane's 8 pairs of warp-tile row r and stage the output row
-// segment (ttab: this lane's copy of the replicated centre table).
+// Decode this lane's 8 pairs of warp-tile row r and store them (ttab: this
+// lane's copy of the replicated centre table; orow: the lane's first output
+// pair, element 2l of its row; live: the row exists).
 template <int D, typename TOut, int W, int B, int MODE>
-__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab, int lane) {
+__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab, int lane,
+                                            const uint2 (&msk)[8], uint8_t* orow, bool live) {
   using C = Dec<D, TOut, W, B>;
   using G = Geo<D>;
-  using OT = typename C::OT;
   constexpr int L = C::L;
   constexpr int n = 1 << W;
   constexpr int AB = C::AB, NB = C::NB;
@@ -184,16 +180,19 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
     // Stages on pair-index bits 3..log2(P)-1 (this lane now holds pairs l + L*m).
     butterfly8<8, 8 / L>(v);
   }
-  // Convert and stage the row (D is applied in the copy-out): pair i = l + L*m
-  // is element pair (2i, 2i+1).
-  uint8_t* orow = wsm + C::W_OUT + r * OT::STRIDE + 2 * C::ESZ * l;
+  // D, convert, store: pair i = l + L*m is element pair (2i, 2i+1).  The L
+  // lanes of a row store L consecutive pairs (a whole 32-byte sector for bf16),
+  // so every store instruction writes full sectors.
+  if (live) {
 #pragma unroll
-  for (int m = 0; m < 8; ++m) {
-    if constexpr (C::ESZ == 2) {
-      const __nv_bfloat162 bb = __floats2bfloat162_rn(v[m].x, v[m].y);
-      *reinterpret_cast<__nv_bfloat162*>(orow + 4 * L * m) = bb;
-    } else {
-      *reinterpret_cast<float2*>(orow + 8 * L * m) = v[m];
+    for (int m = 0; m < 8; ++m) {
+      if constexpr (C::ESZ == 2) {
+        const __nv_bfloat162 bb = __floats2bfloat162_rn(v[m].x, v[m].y);
+        *reinterpret_cast<uint32_t*>(orow + 4 * L * m) = (*reinterpret_cast<const uint32_t*>(&bb)) ^ msk[m].x;
+      } else {
+        *reinterpret_cast<uint2*>(orow + 8 * L * m) =
+            make_uint2(__float_as_uint(v[m].x) ^ msk[m].x, __float_as_uint(v[m].y) ^ msk[m].y);
+      }
     }
   }
 }
@@ -201,7 +200,6 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
 template <int D, typename TOut, int W, int B, int MODE>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecParams p) {
   using C = Dec<D, TOut, W, B>;
-  using OT = typename C::OT;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
@@ -282,12 +280,11 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
   int c_end = t;                 // first tile after the current job (forces a job load)
   int64_t c_left = 0;            // rows of the job from the current tile's row 0
   int64_t c_step = 0;            // output bytes between consecutive tiles (RW rows)
-  int64_t c_qstep = 0;           // output bytes between a lane's consecutive chunks (RPQ rows)
-  // Output chunk q of a lane is row q*RPQ + lane/CPR, bytes (lane % CPR)*16.
-  const int lane_cr = lane / C::CPR;
-  const uint8_t* const out_src = wsm + C::W_OUT + lane_cr * OT::STRIDE + (lane % C::CPR) * 16;
-  uint8_t* o_dst = nullptr;      // this lane's first output chunk of the current tile
-  uint4 dmask = make_uint4(0u, 0u, 0u, 0u);  // D of Sec. 2 on this lane's 16 output bytes (sign bits)
+  const int r = lane / C::L, l = lane % C::L;
+  uint8_t* o_row = nullptr;      // this lane's first output pair in the current tile
+  uint2 msk[8];
+#pragma unroll
+  for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
 
   int stage = 0;
   for (; t < t_end; ++t) {
@@ -306,44 +303,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
       c_left = J.rows - row0;
       const int64_t sb = J.stride * C::ESZ;
       c_step = C::RW * sb;
-      c_qstep = C::RPQ * sb;
-      o_dst = reinterpret_cast<uint8_t*>(J.y) + (row0 + lane_cr) * sb + (lane % C::CPR) * 16;
-      // the lane's chunk holds elements e0 .. e0 + 16/ESZ - 1 of every row it writes
-      const int e0 = (lane % C::CPR) * (16 / C::ESZ);
-      uint32_t mw[4];
+      o_row = reinterpret_cast<uint8_t*>(J.y) + (row0 + r) * sb + 2 * C::ESZ * l;
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        if constexpr (C::ESZ == 2) {
-          const int e = e0 + 2 * q;
-          mw[q] = (((J.signs[e >> 5] >> (e & 31)) & 1u) << 15) | (((J.signs[(e + 1) >> 5] >> ((e + 1) & 31)) & 1u) << 31);
-        } else {
-          const int e = e0 + q;
-          mw[q] = ((J.signs[e >> 5] >> (e & 31)) & 1u) << 31;
-        }
-      }
-      dmask = make_uint4(mw[0], mw[1], mw[2], mw[3]);
+      for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
     }
     const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;
-    decode_body<D, TOut, W, B, MODE>(rec, wsm, ttab + (lane % C::TABR), lane);
-    __syncwarp();
-    // Apply D and write the warp tile's rows: 16-byte chunks, coalesced.
-    if (c_left >= C::RW) {
-#pragma unroll
-      for (int q = 0; q < C::CHUNKS; ++q) {
-        uint4 v = *reinterpret_cast<const uint4*>(out_src + q * C::RPQ * OT::STRIDE);
-        v.x ^= dmask.x; v.y ^= dmask.y; v.z ^= dmask.z; v.w ^= dmask.w;
-        *reinterpret_cast<uint4*>(o_dst + q * c_qstep) = v;
-      }
-    } else {
-#pragma unroll
-      for (int q = 0; q < C::CHUNKS; ++q)
-        if (q * C::RPQ + lane_cr < c_left) {
-          uint4 v = *reinterpret_cast<const uint4*>(out_src + q * C::RPQ * OT::STRIDE);
-          v.x ^= dmask.x; v.y ^= dmask.y; v.z ^= dmask.z; v.w ^= dmask.w;
-          *reinterpret_cast<uint4*>(o_dst + q * c_qstep) = v;
-        }
-    }
-    o_dst += c_step;
+    decode_body<D, TOut, W, B, MODE>(rec, wsm, ttab + (lane % C::TABR), lane, msk, o_row, r < c_left);
+    o_row += c_step;
     c_left -= C::RW;
     stage = (stage + 1 == kNS) ? 0 : stage + 1;
   }

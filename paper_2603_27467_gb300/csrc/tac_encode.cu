@@ -364,11 +364,12 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
     if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_ftz(s[j] * sigma);
     else f = lg2_ftz(fmaxf(s[j] * sigma, sfl));
     const uint32_t c = min(__float2uint_rd(__fmaf_rn(f, qs, qo)), (uint32_t)Lq);
+    // fields are disjoint and k < n, c <= Lq: the adds are ORs (one IMAD each)
     const int sa = j * W, sn = j * B;
-    if (sa + W <= 32) alo |= k << sa;
-    else if (sa >= 32) ahi |= k << (sa - 32);
-    else { alo |= k << sa; ahi |= k >> (32 - sa); }
-    if (sn < 32) nlo |= c << sn; else nhi |= c << (sn - 32);
+    if (sa + W <= 32) alo += k << sa;
+    else if (sa >= 32) ahi += k << (sa - 32);
+    else { alo += k << sa; ahi += k >> (32 - sa); }
+    if (sn < 32) nlo += c << sn; else nhi += c << (sn - 32);
   }
   uint32_t fm = 0;
   if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; }
