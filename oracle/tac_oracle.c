@@ -40,6 +40,10 @@
  *      (q = 0 for every (layer, kv) in "shared" mode, the paper's single D).
  *   R9 Bit packing: each vector's codes form one LSB-first bitstream (code i at bit
  *      i*w); a vector's stream starts on a byte boundary.
+ *   R16 fp32 norm storage (mode 2, the angle-only configuration whose rates count
+ *      angle bits only, Sec. 3.1 and Tables 1-4): each pair norm r_i is stored as
+ *      the fp32 value nearest to it (its 32 bits are the "norm code", b = 32) and
+ *      decode uses that value as r^; there is no min/max header in this mode.
  */
 #include <math.h>
 #include <stddef.h>
@@ -128,6 +132,14 @@ static int32_t angle_code(double y0, double y1, int n, double* edge_dist) {
   return (int32_t)k;
 }
 
+/* fp32 bit pattern of the float nearest to v (reading R16). */
+static int32_t fp32_bits(double v) {
+  float f = (float)v;
+  int32_t b;
+  memcpy(&b, &f, sizeof b);
+  return b;
+}
+
 /* Eq. 2 with clamp (reading R4); returns the pre-round value in *pre. */
 static int32_t norm_code(double val, double lo, double hi, int b, double* pre) {
   int32_t L = (1 << b) - 1;
@@ -144,7 +156,8 @@ static int32_t norm_code(double val, double lo, double hi, int b, double* pre) {
  * Encode (Alg. 1 + Sec. 3.3 / Eq. 2).
  *   x        rows x d doubles (the input vectors, converted exactly from bf16/fp32)
  *   s        d signs (+-1), the diagonal D
- *   n        angle bins; b norm bits; mode 0 = linear, 1 = log-space
+ *   n        angle bins; b norm bits; mode 0 = linear, 1 = log-space,
+ *            2 = fp32 norms (b = 32, reading R16)
  *   k_out    rows x d/2 angle indices
  *   c_out    rows x d/2 norm codes
  *   hdr_out  rows x 2 floats: stored (r_min, r_max)
@@ -155,7 +168,8 @@ static int32_t norm_code(double val, double lo, double hi, int b, double* pre) {
 int orc_encode(const double* x, int64_t rows, int d, const int8_t* s, int n, int b, int mode,
                int32_t* k_out, int32_t* c_out, float* hdr_out, double* edge_out, double* pre_out,
                double* r_out) {
-  if (d < 2 || (d & (d - 1)) || n < 1 || b < 1 || b > 16 || (mode != 0 && mode != 1)) return 1;
+  if (d < 2 || (d & (d - 1)) || n < 1) return 1;
+  if (!((mode == 0 || mode == 1) && b >= 1 && b <= 16) && !(mode == 2 && b == 32)) return 1;
   const int P = d / 2;
   double* H = (double*)malloc(sizeof(double) * (size_t)d * d);
   double* y = (double*)malloc(sizeof(double) * (size_t)d);
@@ -176,7 +190,14 @@ int orc_encode(const double* x, int64_t rows, int d, const int8_t* s, int n, int
       if (r[i] > rmax) rmax = r[i];
     }
     double* pre = pre_out ? pre_out + row * P : NULL;
-    if (mode == 0) {
+    if (mode == 2) {                                         /* reading R16 */
+      hdr_out[2 * row] = (float)rmin;
+      hdr_out[2 * row + 1] = (float)rmax;
+      for (int i = 0; i < P; ++i) {
+        c_out[row * P + i] = fp32_bits(r[i]);
+        if (pre) pre[i] = 0.0;
+      }
+    } else if (mode == 0) {
       float hmin = (float)rmin, hmax = (float)rmax;        /* Sec. 3.3: fp32 min/max */
       hdr_out[2 * row] = hmin;
       hdr_out[2 * row + 1] = hmax;
@@ -217,9 +238,10 @@ int orc_encode(const double* x, int64_t rows, int d, const int8_t* s, int n, int
  */
 int orc_decode(const int32_t* k, const int32_t* c, const float* hdr, int64_t rows, int d,
                const int8_t* s, int n, int b, int mode, double* y_out) {
-  if (d < 2 || (d & (d - 1)) || n < 1 || b < 1 || b > 16 || (mode != 0 && mode != 1)) return 1;
+  if (d < 2 || (d & (d - 1)) || n < 1) return 1;
+  if (!((mode == 0 || mode == 1) && b >= 1 && b <= 16) && !(mode == 2 && b == 32)) return 1;
   const int P = d / 2;
-  const double L = (double)((1 << b) - 1);
+  const double L = mode == 2 ? 1.0 : (double)((1 << b) - 1);
   double* H = (double*)malloc(sizeof(double) * (size_t)d * d);
   double* yh = (double*)malloc(sizeof(double) * (size_t)d);
   if (!H || !yh) { free(H); free(yh); return 2; }
@@ -228,7 +250,11 @@ int orc_decode(const int32_t* k, const int32_t* c, const float* hdr, int64_t row
     double hmin = (double)hdr[2 * row], hmax = (double)hdr[2 * row + 1];
     for (int i = 0; i < P; ++i) {
       double ci = (double)c[row * P + i], rh;
-      if (hmax == hmin) rh = hmin;
+      if (mode == 2) {                                       /* reading R16 */
+        float f;
+        memcpy(&f, &c[row * P + i], sizeof f);
+        rh = (double)f;
+      } else if (hmax == hmin) rh = hmin;
       else if (mode == 0) rh = hmin + ci * (hmax - hmin) / L;
       else {
         double lmin = log2(hmin), lmax = log2(hmax);
@@ -255,7 +281,7 @@ int orc_decode(const int32_t* k, const int32_t* c, const float* hdr, int64_t row
 /* Reading R9: pack `count` codes of `bits` bits per row into an LSB-first
  * bitstream; row stride = ceil(count*bits/8) bytes. */
 int orc_pack(const int32_t* codes, int64_t rows, int count, int bits, uint8_t* out) {
-  if (bits < 1 || bits > 16) return 1;
+  if (bits < 1 || bits > 32) return 1;
   size_t stride = ((size_t)count * bits + 7) / 8;
   memset(out, 0, stride * (size_t)rows);
   for (int64_t r = 0; r < rows; ++r) {
@@ -272,7 +298,7 @@ int orc_pack(const int32_t* codes, int64_t rows, int count, int bits, uint8_t* o
 }
 
 int orc_unpack(const uint8_t* in, int64_t rows, int count, int bits, int32_t* codes) {
-  if (bits < 1 || bits > 16) return 1;
+  if (bits < 1 || bits > 32) return 1;
   size_t stride = ((size_t)count * bits + 7) / 8;
   for (int64_t r = 0; r < rows; ++r) {
     const uint8_t* p = in + (size_t)r * stride;

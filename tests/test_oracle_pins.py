@@ -126,7 +126,7 @@ def _x_from_y(orc, y, s):
     return orc.transform(y, np.ones(d, dtype=np.int8)) * s
 
 
-@pytest.mark.parametrize("n", [8, 16, 64, 256])
+@pytest.mark.parametrize("n", [8, 16, 48, 56, 64, 256])
 def test_angle_worked_examples(orc, n):
     d = 64  # 1/sqrt(64) = 1/8: x = D H y is exact
     s = orc.signs(3, 0, 0, d)
@@ -158,7 +158,7 @@ def test_angle_n2_halfplane_and_n4_nearest_axis(orc):
     assert np.array_equal(k4, axis.astype(np.int32))               # n = 4: nearest axis
 
 
-@pytest.mark.parametrize("n", [16, 64, 256])
+@pytest.mark.parametrize("n", [16, 48, 56, 64, 256])
 def test_angle_error_bound(orc, n):
     """|theta^ - theta| <= pi/n (wrapped) for every pair, theta^ = 2 pi k / n."""
     d = 128
@@ -279,7 +279,7 @@ def test_degenerate_rows(orc):
 # ---------------------------------------------------------------------------
 # Decode (Sec. 3.1) and whole round trips
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("n", [8, 64, 256])
+@pytest.mark.parametrize("n", [8, 48, 56, 64, 256])
 def test_exact_round_trip_at_bin_centres(orc, n):
     """y with every angle on a bin centre and norms in {1, 2}: encode gives the
     known codes and decode returns x (1-bit linear norms are exact here)."""
@@ -301,7 +301,7 @@ def test_exact_round_trip_at_bin_centres(orc, n):
     assert np.allclose(xh, x, atol=1e-12)
 
 
-@pytest.mark.parametrize("n", [16, 64, 256])
+@pytest.mark.parametrize("n", [16, 56, 64, 256])
 def test_decode_pair_error_bound(orc, n):
     """With (nearly) unquantized norms the reconstruction error of each pair is
     at most the chord of half a bin, 2 r sin(pi / 2n), and H is orthonormal so
@@ -320,6 +320,55 @@ def test_decode_pair_error_bound(orc, n):
 
 
 # ---------------------------------------------------------------------------
+# fp32 norm storage (reading R16: the angle-only configuration of Sec. 3.1 and
+# Tables 1-4, "each pair norm r_i is stored in fp32")
+# ---------------------------------------------------------------------------
+def test_fp32_norms_store_exact_norms(orc):
+    """Pairs built from scaled Pythagorean triples have exactly representable
+    norms (3-4-5, 5-12-13, 8-15-17); x = D H y is exact at d = 64.  The stored
+    norm code is the fp32 bit pattern of that norm, and decode equals an
+    independent reconstruction D H y^ (test-local butterfly) from the stored
+    norm and the bin-centre angle."""
+    d, n = 64, 56
+    triples = [(3, 4, 5), (5, 12, 13), (8, 15, 17), (-3, 4, 5), (4, -3, 5), (-12, -5, 13)]
+    rng = np.random.default_rng(2)
+    y = np.zeros((8, d))
+    rr = np.zeros((8, d // 2))
+    for row in range(8):
+        for i in range(d // 2):
+            a, b, c = triples[rng.integers(len(triples))]
+            sc = 2.0 ** int(rng.integers(-4, 4))
+            y[row, 2 * i], y[row, 2 * i + 1], rr[row, i] = a * sc, b * sc, c * sc
+    s = orc.signs(1, 2, 1, d)
+    x = _x_from_y(orc, y, s)
+    out = orc.encode(x, s, n, 32, 2)
+    assert np.array_equal(out["c"].view(np.float32).astype(np.float64), rr)
+    xh = orc.decode(out["k"], out["c"], out["hdr"], s, n, 32, 2)
+    phi = 2 * np.pi * out["k"] / n
+    yh = np.zeros((8, d))
+    yh[:, 0::2], yh[:, 1::2] = rr * np.cos(phi), rr * np.sin(phi)
+    want = _butterfly(yh) / math.sqrt(d) * s
+    assert np.allclose(xh, want, rtol=0, atol=1e-12 * np.abs(want).max())
+
+
+@pytest.mark.parametrize("n", [48, 64, 256])
+def test_fp32_norms_pair_error_bound(orc, n):
+    """fp32 norms: each pair's reconstruction error is at most the chord of half
+    a bin, 2 r sin(pi/2n), plus the fp32 rounding of r (2^-24 r)."""
+    d = 128
+    rng = np.random.default_rng(30 + n)
+    x = rng.standard_normal((40, d)) * np.exp(rng.normal(0, 1, d))
+    s = orc.signs(0, 5, 0, d)
+    out = orc.encode(x, s, n, 32, 2)
+    xh = orc.decode(out["k"], out["c"], out["hdr"], s, n, 32, 2)
+    r = out["r"]
+    bound = np.sqrt(np.sum((2 * r * math.sin(math.pi / (2 * n)) + r * 2.0**-24) ** 2, axis=1))
+    assert np.all(np.linalg.norm(xh - x, axis=1) <= bound * (1 + 1e-9) + 1e-12)
+    # 16 bits per element: one fp32 per pair (Sec. 3.1)
+    assert orc.pack(out["c"][:1], 32).nbytes * 8 / d == 16
+
+
+# ---------------------------------------------------------------------------
 # Packing (reading R9) and rates (Eq. 1, Eq. 3)
 # ---------------------------------------------------------------------------
 def test_pack_layout_by_hand(orc):
@@ -332,10 +381,10 @@ def test_pack_layout_by_hand(orc):
     assert out.tolist() == [[0xC3]]
 
 
-@pytest.mark.parametrize("bits", [1, 3, 4, 5, 6, 7, 8])
+@pytest.mark.parametrize("bits", [1, 3, 4, 5, 6, 7, 8, 32])
 def test_pack_round_trip(orc, bits):
     rng = np.random.default_rng(bits)
-    codes = rng.integers(0, 1 << bits, size=(17, 64))
+    codes = rng.integers(-(1 << 31), 1 << 31, size=(17, 64)) if bits == 32 else rng.integers(0, 1 << bits, size=(17, 64))
     assert np.array_equal(orc.unpack(orc.pack(codes, bits), 64, bits), codes)
 
 
