@@ -10,17 +10,20 @@
  *     k_i = floor(n theta_i / 2 pi + 1/2) mod n                      (Alg. 1)
  *     c_i = round((r_i - r_min)/(r_max - r_min) (2^b - 1))           (Eq. 2, linear)
  *           or Eq. 2 applied to log2 r_i                              (Sec. 3.3, log-space)
- *     stored: k_i (log2 n bits each), c_i (b bits each), (r_min, r_max) as fp32.
+ *     stored: k_i (ceil(log2 n) bits each), c_i (b bits each), (r_min, r_max) as fp32;
+ *     or, with TAC_NORM_FP32 (the angle-only configuration of Sec. 3.1 / Tables 1-4),
+ *     r_i itself as fp32 (b = 32) and no (r_min, r_max).
  *   decode (Sec. 3.1): y^_2i = r^_i cos(2 pi k_i / n), y^_2i+1 = r^_i sin(2 pi k_i / n),
  *     x^ = D H y^, with r^_i the dequantized norm (r_min + c (r_max - r_min)/(2^b - 1), or
  *     the same in log2 space).
  *
  * Record layout ("three planes", caller-owned device memory, one record slot per row):
- *   angle plane   slot s at  codes + s * tac_angle_row_bytes(cfg):  d/2 codes of log2(n) bits,
- *                 one LSB-first bitstream per row (code i occupies bits [i*w, i*w + w)).
- *   norm plane    slot s at  norms + s * tac_norm_row_bytes(cfg):   d/2 codes of b bits, same order.
+ *   angle plane   slot s at  codes + s * tac_angle_row_bytes(cfg):  d/2 codes of w = ceil(log2 n)
+ *                 bits, one LSB-first bitstream per row (code i occupies bits [i*w, i*w + w)).
+ *   norm plane    slot s at  norms + s * tac_norm_row_bytes(cfg):   d/2 codes of b bits, same order
+ *                 (TAC_NORM_FP32: d/2 little-endian floats r_i).
  *   header plane  slot s at  norms + tac_header_offset(cfg, capacity) + 8*s:
- *                 float r_min, float r_max (little endian).
+ *                 float r_min, float r_max (little endian); absent with TAC_NORM_FP32.
  *
  * Conventions shared by every entry point:
  *   - All device pointers must be 16-byte aligned; rows are row_stride elements
@@ -53,7 +56,9 @@ typedef enum {
   TAC_E_CUDA = 3
 } tac_status;
 
-typedef enum { TAC_NORM_LINEAR = 0, TAC_NORM_LOG = 1 } tac_norm_mode;
+/* Norm storage: Eq. 2 linear, Eq. 2 on log2 r (Sec. 3.3), or the pair norms as fp32
+ * (Sec. 3.1: "each pair norm r_i is stored in fp32"; norm_bits must be 32). */
+typedef enum { TAC_NORM_LINEAR = 0, TAC_NORM_LOG = 1, TAC_NORM_FP32 = 2 } tac_norm_mode;
 typedef enum { TAC_BF16 = 0, TAC_FP32 = 1 } tac_dtype;
 
 #define TAC_MAX_D 128
@@ -66,8 +71,8 @@ typedef enum { TAC_BF16 = 0, TAC_FP32 = 1 } tac_dtype;
  */
 typedef struct {
   int32_t d;          /* head dimension: 16, 32, 64 or 128 */
-  int32_t n_angle;    /* angle bins n: a power of two, 2..256 */
-  int32_t norm_bits;  /* b: 4 or 8 */
+  int32_t n_angle;    /* angle bins n: a power of two 2..256, or 48 or 56 (Table 1) */
+  int32_t norm_bits;  /* b: 4 or 8 (linear / log), 32 (TAC_NORM_FP32) */
   int32_t norm_mode;  /* tac_norm_mode */
   uint32_t signs[TAC_MAX_D / 32]; /* D: bit j of the little-endian word array set <=> s_j = -1
                                      (from tac_make_signs); bits >= d are ignored */
@@ -115,15 +120,17 @@ typedef struct {
  */
 int tac_make_signs(uint64_t seed, int layer, int kv, int shared, int d, uint32_t* out_words);
 
-/* Bytes per row of each plane (Sec. 3.1 rate: log2(n) bits per pair; Eq. 3 norm bits
- * per pair; 64 bits of header per vector).  Return -1 for an invalid cfg. */
-int64_t tac_angle_row_bytes(const tac_layer_cfg* cfg);   /* d/2 * log2(n) / 8 */
+/* Bytes per row of each plane (Sec. 3.1 rate: log2(n) bits per pair, stored in
+ * ceil(log2 n) bits; Eq. 3 norm bits per pair; 64 bits of header per vector).
+ * Return -1 for an invalid cfg. */
+int64_t tac_angle_row_bytes(const tac_layer_cfg* cfg);   /* d/2 * ceil(log2 n) / 8 */
 int64_t tac_norm_row_bytes(const tac_layer_cfg* cfg);    /* d/2 * b / 8 */
 /* Byte offset of the header plane inside `norms` for a cache of `capacity` slots:
  * capacity * tac_norm_row_bytes rounded up to a multiple of 16. */
 int64_t tac_header_offset(const tac_layer_cfg* cfg, int64_t capacity);
 int64_t tac_codes_bytes(const tac_layer_cfg* cfg, int64_t capacity); /* angle plane size */
-int64_t tac_norms_bytes(const tac_layer_cfg* cfg, int64_t capacity); /* norm + header planes */
+/* norm + header planes: tac_header_offset + 8 * capacity (no header with TAC_NORM_FP32) */
+int64_t tac_norms_bytes(const tac_layer_cfg* cfg, int64_t capacity);
 
 /* Eq. 1: (1/L) sum_l (log2 n_K^l + log2 n_V^l) / 4.  Returns NaN if an n is < 1. */
 double tac_avg_angle_bits(int num_layers, const int* n_k, const int* n_v);

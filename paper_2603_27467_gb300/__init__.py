@@ -19,7 +19,7 @@ from dataclasses import dataclass, field
 import numpy as np
 
 __all__ = [
-    "TAC_OK", "TAC_E_INVAL", "TAC_E_UNSUPPORTED", "TAC_E_CUDA", "NORM_LINEAR", "NORM_LOG",
+    "TAC_OK", "TAC_E_INVAL", "TAC_E_UNSUPPORTED", "TAC_E_CUDA", "NORM_LINEAR", "NORM_LOG", "NORM_FP32",
     "BF16", "FP32", "TacError", "LayerCfg", "EncodeJob", "DecodeJob", "library_path", "load",
     "make_signs", "layer_cfg", "angle_row_bytes", "norm_row_bytes", "header_offset",
     "codes_bytes", "norms_bytes", "avg_angle_bits", "total_bits", "encode", "decode",
@@ -27,7 +27,7 @@ __all__ = [
 ]
 
 TAC_OK, TAC_E_INVAL, TAC_E_UNSUPPORTED, TAC_E_CUDA = 0, 1, 2, 3
-NORM_LINEAR, NORM_LOG = 0, 1
+NORM_LINEAR, NORM_LOG, NORM_FP32 = 0, 1, 2
 BF16, FP32 = 0, 1
 MAX_D = 128
 MAX_JOBS = 96  # TAC_MAX_JOBS: jobs per kernel launch
@@ -252,12 +252,15 @@ class Cache:
         return Cache(cfg, capacity, codes, norms)
 
     def planes(self):
-        """Host views (numpy) of (angle plane, norm plane, header (r_min, r_max))."""
+        """Host views (numpy) of (angle plane, norm plane, header (r_min, r_max));
+        with fp32 norms there is no header plane and the header is None."""
         ab, nb = angle_row_bytes(self.cfg), norm_row_bytes(self.cfg)
         off = header_offset(self.cfg, self.capacity)
         codes = self.codes.cpu().numpy()[: self.capacity * ab].reshape(self.capacity, ab)
         nh = self.norms.cpu().numpy()
         norms = nh[: self.capacity * nb].reshape(self.capacity, nb)
+        if self.cfg.norm_mode == NORM_FP32:
+            return codes, norms, None
         hdr = nh[off: off + 8 * self.capacity].view(np.float32).reshape(self.capacity, 2)
         return codes, norms, hdr
 
@@ -360,11 +363,18 @@ def fwht_debug(x, signs: np.ndarray, d: int, stream=None):
 
 def rates(d: int, n_k, n_v, b_k: int = 8, b_v: int = 4) -> dict:
     """Rate accounting for a per-layer schedule: Eq. 1 angle bits, payload bits
-    (angle + norm bits per pair / 2) and Eq. 3 totals (64/d min-max overhead)."""
+    (angle + norm bits per pair / 2) and Eq. 3 totals (64/d min-max overhead).
+    With b_k = b_v = 32 (fp32 norms, Sec. 3.1) the total is the angle bits plus
+    16 bits per element and there is no min-max overhead; "stored_bits" counts
+    the ceil(log2 n) bits a code of a non-power-of-two n occupies."""
+    import math
     b_angle = avg_angle_bits(n_k, n_v)
     payload = b_angle + (b_k + b_v) / 4.0
-    return {"angle_bits": b_angle, "payload_bits": payload,
-            "total_bits": total_bits(b_angle, (b_k + b_v) / 2.0, d)}
+    fp32 = b_k == 32 and b_v == 32
+    total = payload if fp32 else total_bits(b_angle, (b_k + b_v) / 2.0, d)
+    stored = sum(math.ceil(math.log2(a)) + math.ceil(math.log2(b)) for a, b in zip(n_k, n_v)) / (4.0 * len(n_k))
+    return {"angle_bits": b_angle, "payload_bits": payload, "total_bits": total,
+            "stored_angle_bits": stored}
 
 
 def early_boost(num_layers: int, boosted, n_early=(256, 128), base=(128, 64)):

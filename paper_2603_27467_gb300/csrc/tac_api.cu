@@ -12,59 +12,59 @@
 #include "tac_common.cuh"
 
 namespace tac {
-cudaError_t launch_encode_16_bf16(const EncParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_encode_16_bf16(const EncParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_encode_32_bf16(const EncParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_encode_32_bf16(const EncParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_encode_64_bf16(const EncParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_encode_64_bf16(const EncParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_encode_128_bf16(const EncParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_encode_128_bf16(const EncParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_encode_16_f32(const EncParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_encode_16_f32(const EncParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_encode_32_f32(const EncParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_encode_32_f32(const EncParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_encode_64_f32(const EncParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_encode_64_f32(const EncParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_encode_128_f32(const EncParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_encode_128_f32(const EncParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_decode_16_bf16(const DecParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_decode_16_bf16(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_decode_32_bf16(const DecParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_decode_32_bf16(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_decode_64_bf16(const DecParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_decode_64_bf16(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_decode_128_bf16(const DecParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_decode_128_bf16(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_decode_16_f32(const DecParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_decode_16_f32(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_decode_32_f32(const DecParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_decode_32_f32(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_decode_64_f32(const DecParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_decode_64_f32(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
-cudaError_t launch_decode_128_f32(const DecParams& p, int w, int b, int mode, int sms,
+cudaError_t launch_decode_128_f32(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
 
-static cudaError_t launch_encode(int d, int dtype, int w, int b, int mode, const EncParams& p, int sms,
+static cudaError_t launch_encode(int d, int dtype, int n, int b, int mode, const EncParams& p, int sms,
                                  cudaStream_t st) {
   const bool bf = dtype == TAC_BF16;
   switch (d) {
-    case 16: return bf ? launch_encode_16_bf16(p, w, b, mode, sms, st) : launch_encode_16_f32(p, w, b, mode, sms, st);
-    case 32: return bf ? launch_encode_32_bf16(p, w, b, mode, sms, st) : launch_encode_32_f32(p, w, b, mode, sms, st);
-    case 64: return bf ? launch_encode_64_bf16(p, w, b, mode, sms, st) : launch_encode_64_f32(p, w, b, mode, sms, st);
-    case 128: return bf ? launch_encode_128_bf16(p, w, b, mode, sms, st) : launch_encode_128_f32(p, w, b, mode, sms, st);
+    case 16: return bf ? launch_encode_16_bf16(p, n, b, mode, sms, st) : launch_encode_16_f32(p, n, b, mode, sms, st);
+    case 32: return bf ? launch_encode_32_bf16(p, n, b, mode, sms, st) : launch_encode_32_f32(p, n, b, mode, sms, st);
+    case 64: return bf ? launch_encode_64_bf16(p, n, b, mode, sms, st) : launch_encode_64_f32(p, n, b, mode, sms, st);
+    case 128: return bf ? launch_encode_128_bf16(p, n, b, mode, sms, st) : launch_encode_128_f32(p, n, b, mode, sms, st);
   }
   return cudaErrorInvalidValue;
 }
 
-static cudaError_t launch_decode(int d, int dtype, int w, int b, int mode, const DecParams& p, int sms,
+static cudaError_t launch_decode(int d, int dtype, int n, int b, int mode, const DecParams& p, int sms,
                                  cudaStream_t st) {
   const bool bf = dtype == TAC_BF16;
   switch (d) {
-    case 16: return bf ? launch_decode_16_bf16(p, w, b, mode, sms, st) : launch_decode_16_f32(p, w, b, mode, sms, st);
-    case 32: return bf ? launch_decode_32_bf16(p, w, b, mode, sms, st) : launch_decode_32_f32(p, w, b, mode, sms, st);
-    case 64: return bf ? launch_decode_64_bf16(p, w, b, mode, sms, st) : launch_decode_64_f32(p, w, b, mode, sms, st);
-    case 128: return bf ? launch_decode_128_bf16(p, w, b, mode, sms, st) : launch_decode_128_f32(p, w, b, mode, sms, st);
+    case 16: return bf ? launch_decode_16_bf16(p, n, b, mode, sms, st) : launch_decode_16_f32(p, n, b, mode, sms, st);
+    case 32: return bf ? launch_decode_32_bf16(p, n, b, mode, sms, st) : launch_decode_32_f32(p, n, b, mode, sms, st);
+    case 64: return bf ? launch_decode_64_bf16(p, n, b, mode, sms, st) : launch_decode_64_f32(p, n, b, mode, sms, st);
+    case 128: return bf ? launch_decode_128_bf16(p, n, b, mode, sms, st) : launch_decode_128_f32(p, n, b, mode, sms, st);
   }
   return cudaErrorInvalidValue;
 }
@@ -113,23 +113,25 @@ int check_cfg(const tac_layer_cfg* c, const char* who) {
       return fail(TAC_E_UNSUPPORTED, "%s: d = %d not implemented (16, 32, 64, 128)", who, c->d);
     return fail(TAC_E_INVAL, "%s: d = %d is not a power of two", who, c->d);
   }
-  const int w = log2_exact(c->n_angle);
-  if (w < 0) {
-    if (c->n_angle > 1) return fail(TAC_E_UNSUPPORTED, "%s: n = %d is not a power of two", who, c->n_angle);
-    return fail(TAC_E_INVAL, "%s: n = %d", who, c->n_angle);
-  }
-  if (w < 1 || w > 8) return fail(TAC_E_UNSUPPORTED, "%s: n = %d outside 2..256", who, c->n_angle);
-  if (c->norm_bits != 4 && c->norm_bits != 8) {
+  const int n = c->n_angle;
+  if (n < 2) return fail(TAC_E_INVAL, "%s: n = %d", who, n);
+  const int w = log2_exact(n);
+  if (w < 0 && n != 48 && n != 56)
+    return fail(TAC_E_UNSUPPORTED, "%s: n = %d not implemented (powers of two 2..256, 48, 56)", who, n);
+  if (w > 8) return fail(TAC_E_UNSUPPORTED, "%s: n = %d outside 2..256", who, n);
+  if (c->norm_mode != TAC_NORM_LINEAR && c->norm_mode != TAC_NORM_LOG && c->norm_mode != TAC_NORM_FP32)
+    return fail(TAC_E_INVAL, "%s: norm_mode = %d", who, c->norm_mode);
+  if (c->norm_mode == TAC_NORM_FP32) {
+    if (c->norm_bits != 32) return fail(TAC_E_INVAL, "%s: norm_bits = %d with fp32 norms (must be 32)", who, c->norm_bits);
+  } else if (c->norm_bits != 4 && c->norm_bits != 8) {
     if (c->norm_bits >= 1 && c->norm_bits <= 16)
       return fail(TAC_E_UNSUPPORTED, "%s: norm_bits = %d not implemented (4, 8)", who, c->norm_bits);
     return fail(TAC_E_INVAL, "%s: norm_bits = %d", who, c->norm_bits);
   }
-  if (c->norm_mode != TAC_NORM_LINEAR && c->norm_mode != TAC_NORM_LOG)
-    return fail(TAC_E_INVAL, "%s: norm_mode = %d", who, c->norm_mode);
   return TAC_OK;
 }
 
-int64_t angle_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * log2_exact(c->n_angle) / 8; }
+int64_t angle_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * tac::code_bits(c->n_angle) / 8; }
 int64_t norm_row_bytes(const tac_layer_cfg* c) { return (int64_t)(c->d / 2) * c->norm_bits / 8; }
 int64_t header_offset(const tac_layer_cfg* c, int64_t cap) { return (cap * norm_row_bytes(c) + 15) & ~(int64_t)15; }
 
@@ -223,7 +225,7 @@ int64_t tac_codes_bytes(const tac_layer_cfg* cfg, int64_t capacity) {
 
 int64_t tac_norms_bytes(const tac_layer_cfg* cfg, int64_t capacity) {
   if (check_cfg(cfg, "tac_norms_bytes") || capacity < 0) return -1;
-  return header_offset(cfg, capacity) + 8 * capacity;
+  return header_offset(cfg, capacity) + (cfg->norm_mode == TAC_NORM_FP32 ? 0 : 8 * capacity);
 }
 
 double tac_avg_angle_bits(int num_layers, const int* n_k, const int* n_v) {
@@ -271,8 +273,7 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
   // and up to TAC_MAX_JOBS jobs per launch.
   auto kernel_key = [&](int j) {
     const tac_encode_job& J = jobs[j];
-    return (((J.cfg.d * 4 + J.x.dtype) * 16 + log2_exact(J.cfg.n_angle)) * 16 + J.cfg.norm_bits) * 4 +
-           J.cfg.norm_mode;
+    return (((J.cfg.d * 4 + J.x.dtype) * 512 + J.cfg.n_angle) * 64 + J.cfg.norm_bits) * 4 + J.cfg.norm_mode;
   };
   std::stable_sort(live.begin(), live.end(), [&](int a, int b) { return kernel_key(a) < kernel_key(b); });
   static thread_local tac::EncParams P;
@@ -281,7 +282,7 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
     const int key = kernel_key(live[i]);
     const tac_layer_cfg& c0 = jobs[live[i]].cfg;
     const int d = c0.d, dt = jobs[live[i]].x.dtype;
-    const int w = log2_exact(c0.n_angle), nb = c0.norm_bits, mode = c0.norm_mode;
+    const int na = c0.n_angle, nb = c0.norm_bits, mode = c0.norm_mode;
     std::memset(&P, 0, sizeof(P));
     int64_t tiles = 0;
     while (i < live.size() && P.njobs < TAC_MAX_JOBS && kernel_key(live[i]) == key) {
@@ -299,7 +300,7 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
       E.rows = J.x.rows;
       E.stride = J.x.row_stride;
       copy_signs(E.signs, &J.cfg);
-      E.w = log2_exact(J.cfg.n_angle);
+      E.w = tac::code_bits(J.cfg.n_angle);
       E.b = J.cfg.norm_bits;
       E.mode = J.cfg.norm_mode;
       E.tile0 = (int32_t)tiles;
@@ -309,7 +310,7 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
     }
     if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many rows", who);
     P.ntiles = (int32_t)tiles;
-    cudaError_t e = tac::launch_encode(d, dt, w, nb, mode, P, sms, reinterpret_cast<cudaStream_t>(stream));
+    cudaError_t e = tac::launch_encode(d, dt, na, nb, mode, P, sms, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
   }
   return ok();
@@ -344,8 +345,7 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
   // and up to TAC_MAX_JOBS jobs per launch.
   auto kernel_key = [&](int j) {
     const tac_decode_job& J = jobs[j];
-    return (((J.cfg.d * 4 + J.y.dtype) * 16 + log2_exact(J.cfg.n_angle)) * 16 + J.cfg.norm_bits) * 4 +
-           J.cfg.norm_mode;
+    return (((J.cfg.d * 4 + J.y.dtype) * 512 + J.cfg.n_angle) * 64 + J.cfg.norm_bits) * 4 + J.cfg.norm_mode;
   };
   std::stable_sort(live.begin(), live.end(), [&](int a, int b) { return kernel_key(a) < kernel_key(b); });
   static thread_local tac::DecParams P;
@@ -354,7 +354,7 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
     const int key = kernel_key(live[i]);
     const tac_layer_cfg& c0 = jobs[live[i]].cfg;
     const int d = c0.d, dt = jobs[live[i]].y.dtype;
-    const int w = log2_exact(c0.n_angle), nb = c0.norm_bits, mode = c0.norm_mode;
+    const int na = c0.n_angle, nb = c0.norm_bits, mode = c0.norm_mode;
     std::memset(&P, 0, sizeof(P));
     int64_t tiles = 0;
     while (i < live.size() && P.njobs < TAC_MAX_JOBS && kernel_key(live[i]) == key) {
@@ -372,7 +372,7 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
       E.rows = J.y.rows;
       E.stride = J.y.row_stride;
       copy_signs(E.signs, &J.cfg);
-      E.w = log2_exact(J.cfg.n_angle);
+      E.w = tac::code_bits(J.cfg.n_angle);
       E.b = J.cfg.norm_bits;
       E.mode = J.cfg.norm_mode;
       E.tile0 = (int32_t)tiles;
@@ -382,7 +382,7 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
     }
     if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many rows", who);
     P.ntiles = (int32_t)tiles;
-    cudaError_t e = tac::launch_decode(d, dt, w, nb, mode, P, sms, reinterpret_cast<cudaStream_t>(stream));
+    cudaError_t e = tac::launch_decode(d, dt, na, nb, mode, P, sms, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
   }
   return ok();

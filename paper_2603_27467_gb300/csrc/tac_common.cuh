@@ -12,8 +12,10 @@ namespace tac {
 constexpr int kThreads = 256;      // threads per CTA
 constexpr int kMinBlocks = 3;      // resident CTAs per SM the kernels are built for (24 warps)
 constexpr int kPairsPerThread = 8; // each thread owns 8 consecutive angle pairs (16 elements)
-constexpr int kMaxW = 8;           // log2 n <= 8 (n <= 256)
-constexpr int kTabEntries = 512;   // sum_{w=1..8} 2^w = 510, padded
+constexpr int kMaxW = 8;           // code bits <= 8 (n <= 256)
+// Tables holding one entry per bin for every supported n back to back:
+// n = 2, 4, ..., 256 (510 entries), then n = 48 and n = 56 (Table 1).
+constexpr int kTabEntries = 616;
 constexpr float kU = 5.9604644775390625e-08f;  // fp32 unit roundoff 2^-24
 
 // Lookup tables indexed by a per-pair code are replicated: entry e of copy c
@@ -27,8 +29,23 @@ __host__ __device__ constexpr int tab_copies(int n, int budget) {
   return r;
 }
 
-// Offset of the table for n = 2^w inside a table holding every w = 1..8 back to back.
-__host__ __device__ constexpr int tab_offset(int w) { return (1 << w) - 2; }
+__host__ __device__ constexpr bool is_pow2(int n) { return n > 0 && (n & (n - 1)) == 0; }
+// Code bits for n bins: ceil(log2 n).
+__host__ __device__ constexpr int code_bits(int n) {
+  int w = 0;
+  while ((1 << w) < n) ++w;
+  return w;
+}
+// Offset of the table for n bins inside the table of every supported n.
+__host__ __device__ constexpr int tab_offset_n(int n) { return is_pow2(n) ? n - 2 : (n == 48 ? 510 : 558); }
+// The n of table entry idx and the entry's index within that n's table.
+__host__ __device__ constexpr int tab_n_of(int idx) {
+  if (idx >= 558) return 56;
+  if (idx >= 510) return 48;
+  int w = 1;
+  while ((1 << (w + 1)) - 2 <= idx) ++w;
+  return 1 << w;
+}
 
 // ---------------------------------------------------------------------------
 // Geometry for head dimension D.  P = D/2 angle pairs per row; each lane owns 8
@@ -170,9 +187,9 @@ __device__ __forceinline__ float2 cos_sin_q8(int Q, int n) {
 }
 
 // ---------------------------------------------------------------------------
-// fp64 edge directions for the exact-decision path, built by the host compiler:
-// cos/sin from their Taylor series on [0, pi/4] (|x| <= 0.79: 24 terms reach
-// full double precision) with the same integer octant reduction as above.
+// Edge directions for the exact-decision path, built by the host compiler in
+// fp64: cos/sin from their Taylor series on [0, pi/4] (|x| <= 0.79: 24 terms
+// reach full double precision) with the same integer octant reduction as above.
 // ---------------------------------------------------------------------------
 namespace cx {
 struct CS { double c, s; };
@@ -211,26 +228,15 @@ constexpr CS cos_sin_q8(int Q, int n) {
     default: return CS{s, -c};
   }
 }
-struct EdgeTable { CS v[kTabEntries]; };
-constexpr EdgeTable make_edge_table() {
-  EdgeTable t{};
-  for (int idx = 0; idx < kTabEntries - 2; ++idx) {
-    int w = 1;
-    while ((1 << (w + 1)) - 2 <= idx) ++w;
-    const int n = 1 << w, e = idx - ((1 << w) - 2);
-    t.v[idx] = cos_sin_q8(8 * e + 4 + n, n);
-  }
-  return t;
-}
 }  // namespace cx
 
-// Encode edge table for n = 2^w, entry e: direction psi_e = phi_e + pi/4 of the
+// Encode edge table for n bins, entry e: direction psi_e = phi_e + pi/4 of the
 // edge phi_e = (e + 1/2) 2 pi / n between bins e and e+1, as (cos psi, sin psi).
 // In the pair's butterfly halves (E, O) = ((y0 + y1)/2, (y0 - y1)/2) the sign of
 // E cos psi - O sin psi equals the sign of sin(theta - phi_e) (Alg. 1 angle).
 __device__ __forceinline__ int edge_q8(int e, int n) { return 8 * e + 4 + n; }
 
-// Decode table for n = 2^w, entry k: (cos phi_k + sin phi_k, cos phi_k - sin phi_k)
+// Decode table for n bins, entry k: (cos phi_k + sin phi_k, cos phi_k - sin phi_k)
 // = sqrt2 (sin(phi_k + pi/4), cos(phi_k + pi/4)), phi_k = 2 pi k / n (Sec. 3.1).
 __device__ __forceinline__ int centre_q8(int k, int n) { return 8 * k + n; }
 

@@ -24,22 +24,26 @@ namespace tac {
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles of records in flight
 
-template <int D, typename TOut, int W, int B>
+// Shape of one kernel: n bins (W = ceil(log2 n) bits per code), B norm bits
+// (4, 8, or 32 for fp32 norms), MODE; HB header bytes per row (none for fp32).
+template <int D, typename TOut, int N, int B, int MODE>
 struct Dec {
   using G = Geo<D>;
   static constexpr int P = G::P, L = G::L, RW = G::RW;
   static constexpr int ESZ = (int)sizeof(TOut);
-  static constexpr int n = 1 << W;
+  static constexpr int n = N;
+  static constexpr int W = code_bits(N);
   static constexpr int AB = P * W / 8;        // angle record bytes per row
   static constexpr int NB = P * B / 8;        // norm record bytes per row
-  static constexpr int NA = RW * AB / 16, NN = RW * NB / 16, NH = RW * 8 / 16;
+  static constexpr int HB = (MODE == TAC_NORM_FP32) ? 0 : 8;
+  static constexpr int NA = RW * AB / 16, NN = RW * NB / 16, NH = RW * HB / 16;
   static constexpr int NCH = NA + NN + NH;
   static constexpr int ROUNDS = (NCH + 31) / 32;
   // one record stage of a warp tile: angle | norm | header segments
   static constexpr int R_ANG = 0;
   static constexpr int R_NRM = RW * AB;
   static constexpr int R_HDR = R_NRM + RW * NB;
-  static constexpr int REC_W = R_HDR + RW * 8 + 16;         // + slack for 3-word angle reads
+  static constexpr int REC_W = R_HDR + RW * HB + 16;        // + slack for 3-word angle reads
   // per-warp shared memory region
   static constexpr int W_REC = 0;                           // kNS record stages
   static constexpr int W_TP = W_REC + kNS * REC_W;          // transpose rows
@@ -55,11 +59,11 @@ struct Dec {
 // the last chunk of each zero-filled past the tile.  Gathered slots: lane
 // r < nrows copies row r's record with plain loads; an out-of-range slot
 // decodes as an all-zero record.
-template <int AB, int NB, int R_NRM, int R_HDR>
+template <int AB, int NB, int HB, int R_NRM, int R_HDR>
 __device__ __noinline__ void stage_records_slow(const DecJob& J, int64_t row0, int nrows, uint8_t* stage,
                                                 int lane) {
   if (J.slot == nullptr) {
-    const int ba = nrows * AB, bn = nrows * NB, bh = nrows * 8;
+    const int ba = nrows * AB, bn = nrows * NB, bh = nrows * HB;
     const int ca = (ba + 15) >> 4, cn = (bn + 15) >> 4, ch = (bh + 15) >> 4;
     const uint8_t* ga = J.codes + row0 * AB;
     const uint8_t* gn = J.norms + row0 * NB;
@@ -84,7 +88,7 @@ __device__ __noinline__ void stage_records_slow(const DecJob& J, int64_t row0, i
     if (s < 0 || s >= J.capacity) {
       for (int q = 0; q < AB; ++q) da[q] = 0;
       for (int q = 0; q < NB; ++q) dn[q] = 0;
-      *dh = make_float2(0.f, 0.f);
+      if constexpr (HB > 0) *dh = make_float2(0.f, 0.f);
       return;
     }
     const uint8_t* sa = J.codes + s * AB;
@@ -97,7 +101,7 @@ __device__ __noinline__ void stage_records_slow(const DecJob& J, int64_t row0, i
     }
     for (int q = 0; q < NB / 4; ++q)
       reinterpret_cast<uint32_t*>(dn)[q] = __ldg(reinterpret_cast<const uint32_t*>(sn) + q);
-    *dh = __ldg(reinterpret_cast<const float2*>(J.hdr) + s);
+    if constexpr (HB > 0) *dh = __ldg(reinterpret_cast<const float2*>(J.hdr) + s);
   }
 }
 
@@ -123,18 +127,33 @@ __device__ __forceinline__ uint64_t load_bytes(const uint8_t* p) {
 // Decode this lane's 8 pairs of warp-tile row r and store them (ttab: this
 // lane's copy of the replicated centre table; orow: the lane's first output
 // pair, element 2l of its row; live: the row exists).
-template <int D, typename TOut, int W, int B, int MODE>
+template <int D, typename TOut, int N, int B, int MODE>
 __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab, int lane,
                                             const uint2 (&msk)[8], uint8_t* orow, bool live) {
-  using C = Dec<D, TOut, W, B>;
+  using C = Dec<D, TOut, N, B, MODE>;
   using G = Geo<D>;
   constexpr int L = C::L;
-  constexpr int n = 1 << W;
+  constexpr int n = N, W = C::W;
   constexpr int AB = C::AB, NB = C::NB;
-  constexpr int Lq = (1 << B) - 1;
   const int r = lane / L, l = lane % L;
 
   const uint64_t acc_a = load_bytes<W>(rec + C::R_ANG + r * AB + l * W);
+  // A code of a non-power-of-two n is < n in every record this library
+  // writes; clamping keeps any other record's table reads in bounds.
+  auto code = [&](int j) -> uint32_t {
+    const uint32_t k = (uint32_t)(acc_a >> (j * W)) & (uint32_t)((1 << W) - 1);
+    if constexpr (is_pow2(N)) return k;
+    else return min(k, (uint32_t)(n - 1));
+  };
+  float2 v[8];
+  if constexpr (MODE == TAC_NORM_FP32) {  // r^ = the stored fp32 norm (Sec. 3.1)
+    const float4* rp = reinterpret_cast<const float4*>(rec + C::R_NRM + r * NB + l * 32);
+    const float4 a = rp[0], b = rp[1];
+    const float rr[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = mul2(make_float2(rr[j], rr[j]), ttab[code(j) * C::TABR]);
+  } else {
+  constexpr int Lq = (1 << B) - 1;
   const uint64_t acc_n = load_bytes<B>(rec + C::R_NRM + r * NB + l * B);
   const float2 h = reinterpret_cast<const float2*>(rec + C::R_HDR)[r];
   const float hmin = h.x, hmax = h.y;
@@ -155,15 +174,14 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
   const float S = step * (float)(1 << B);
   const float base2 = base - S;
 
-  float2 v[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    const uint32_t k = (uint32_t)(acc_a >> (j * W)) & (uint32_t)(n - 1);
     const uint32_t cb = (uint32_t)(acc_n >> (j * B)) & (uint32_t)Lq;
     const float f = __uint_as_float(0x3F800000u | (cb << (23 - B)));
     float rh = __fmaf_rn(f, S, base2);
     if constexpr (MODE != TAC_NORM_LINEAR) rh = ex2_ftz(rh);
-    v[j] = mul2(make_float2(rh, rh), ttab[k * C::TABR]);
+    v[j] = mul2(make_float2(rh, rh), ttab[code(j) * C::TABR]);
+  }
   }
   // Butterfly stages on pair-index bits 0..2 (this lane holds pairs 8l..8l+7).
   butterfly8<8>(v);
@@ -197,9 +215,9 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
   }
 }
 
-template <int D, typename TOut, int W, int B, int MODE>
+template <int D, typename TOut, int N, int B, int MODE>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecParams p) {
-  using C = Dec<D, TOut, W, B>;
+  using C = Dec<D, TOut, N, B, MODE>;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
@@ -243,7 +261,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
       const int ch = q * 32 + lane;
       if (ch < C::NA) { i_src[q] = J.codes + 16 * ch; i_step[q] = C::RW * C::AB; }
       else if (ch < C::NA + C::NN) { i_src[q] = J.norms + 16 * (ch - C::NA); i_step[q] = C::RW * C::NB; }
-      else { i_src[q] = J.hdr + 16 * (ch - C::NA - C::NN); i_step[q] = C::RW * 8; }
+      else { i_src[q] = J.hdr + 16 * (ch - C::NA - C::NN); i_step[q] = C::RW * C::HB; }
       i_src[q] += (int64_t)rel * i_step[q];
     }
   };
@@ -262,7 +280,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
           if (ch < C::NCH) cp_async16(stage + 16 * ch, i_src[q], 16);
         }
       } else {
-        stage_records_slow<C::AB, C::NB, C::R_NRM, C::R_HDR>(p.job[pj], i_row0, (int)min((int64_t)C::RW, i_left),
+        stage_records_slow<C::AB, C::NB, C::HB, C::R_NRM, C::R_HDR>(p.job[pj], i_row0, (int)min((int64_t)C::RW, i_left),
                                                             stage, lane);
       }
 #pragma unroll
@@ -308,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
       for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
     }
     const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;
-    decode_body<D, TOut, W, B, MODE>(rec, wsm, ttab + (lane % C::TABR), lane, msk, o_row, r < c_left);
+    decode_body<D, TOut, N, B, MODE>(rec, wsm, ttab + (lane % C::TABR), lane, msk, o_row, r < c_left);
     o_row += c_step;
     c_left -= C::RW;
     stage = (stage + 1 == kNS) ? 0 : stage + 1;
@@ -316,10 +334,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
   cp_async_wait<0>();
 }
 
-template <int D, typename TOut, int W, int B, int MODE>
+template <int D, typename TOut, int N, int B, int MODE>
 static cudaError_t launch_decode_v(const DecParams& p, int grid_cap, cudaStream_t st) {
-  using C = Dec<D, TOut, W, B>;
-  auto kern = decode_kernel<D, TOut, W, B, MODE>;
+  using C = Dec<D, TOut, N, B, MODE>;
+  auto kern = decode_kernel<D, TOut, N, B, MODE>;
   static int configured[64] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -340,19 +358,22 @@ static cudaError_t launch_decode_v(const DecParams& p, int grid_cap, cudaStream_
   return cudaGetLastError();
 }
 
+// One kernel per supported (n, norm bits, mode), as for the encoder.
 template <int D, typename TOut>
-static cudaError_t launch_decode_t(const DecParams& p, int w, int b, int mode, int sms, cudaStream_t st) {
-#define TAC_DEC_CASE(WW)                                                                         \
-  case (WW - 1) * 4 + 0: return launch_decode_v<D, TOut, WW, 4, TAC_NORM_LINEAR>(p, sms, st);    \
-  case (WW - 1) * 4 + 1: return launch_decode_v<D, TOut, WW, 4, TAC_NORM_LOG>(p, sms, st);       \
-  case (WW - 1) * 4 + 2: return launch_decode_v<D, TOut, WW, 8, TAC_NORM_LINEAR>(p, sms, st);    \
-  case (WW - 1) * 4 + 3: return launch_decode_v<D, TOut, WW, 8, TAC_NORM_LOG>(p, sms, st);
-  switch ((w - 1) * 4 + (b == 8 ? 2 : 0) + (mode == TAC_NORM_LOG ? 1 : 0)) {
-    TAC_DEC_CASE(1) TAC_DEC_CASE(2) TAC_DEC_CASE(3) TAC_DEC_CASE(4)
-    TAC_DEC_CASE(5) TAC_DEC_CASE(6) TAC_DEC_CASE(7) TAC_DEC_CASE(8)
-    default: break;
+static cudaError_t launch_decode_t(const DecParams& p, int n, int b, int mode, int sms, cudaStream_t st) {
+#define TAC_DEC_N(NN)                                                                                   \
+  if (n == NN) {                                                                                        \
+    if (mode == TAC_NORM_FP32) return b == 32 ? launch_decode_v<D, TOut, NN, 32, TAC_NORM_FP32>(p, sms, st) \
+                                              : cudaErrorInvalidValue;                                  \
+    if (b == 4) return mode == TAC_NORM_LOG ? launch_decode_v<D, TOut, NN, 4, TAC_NORM_LOG>(p, sms, st)    \
+                                            : launch_decode_v<D, TOut, NN, 4, TAC_NORM_LINEAR>(p, sms, st); \
+    if (b == 8) return mode == TAC_NORM_LOG ? launch_decode_v<D, TOut, NN, 8, TAC_NORM_LOG>(p, sms, st)    \
+                                            : launch_decode_v<D, TOut, NN, 8, TAC_NORM_LINEAR>(p, sms, st); \
+    return cudaErrorInvalidValue;                                                                       \
   }
-#undef TAC_DEC_CASE
+  TAC_DEC_N(2) TAC_DEC_N(4) TAC_DEC_N(8) TAC_DEC_N(16) TAC_DEC_N(32) TAC_DEC_N(64) TAC_DEC_N(128)
+  TAC_DEC_N(256) TAC_DEC_N(48) TAC_DEC_N(56)
+#undef TAC_DEC_N
   return cudaErrorInvalidValue;
 }
 
@@ -370,9 +391,9 @@ static cudaError_t launch_decode_t(const DecParams& p, int w, int b, int mode, i
 #define TAC_INST_F32 0
 #endif
 #define TAC_DEC_INSTANCE(DD, NAME, T)                                                                 \
-  cudaError_t launch_decode_##DD##_##NAME(const DecParams& p, int w, int b, int mode, int sms,       \
+  cudaError_t launch_decode_##DD##_##NAME(const DecParams& p, int n, int b, int mode, int sms,       \
                                           cudaStream_t st) {                                         \
-    return launch_decode_t<DD, T>(p, w, b, mode, sms, st);                                           \
+    return launch_decode_t<DD, T>(p, n, b, mode, sms, st);                                           \
   }
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 16 && TAC_INST_BF16)
 TAC_DEC_INSTANCE(16, bf16, __nv_bfloat16)

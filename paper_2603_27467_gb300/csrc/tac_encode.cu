@@ -33,17 +33,15 @@
 
 namespace tac {
 
-// Edge directions (cos psi_e, sin psi_e) for every n = 2..256 as double-float
+// Edge directions (cos psi_e, sin psi_e) for every supported n as double-float
 // pairs (c = ch + cl, s = sh + sl), read warp-uniformly by the exact path.
 namespace cx {
 struct DF4 { float ch, cl, sh, sl; };
 struct DFEdgeTable { DF4 v[kTabEntries]; };
 constexpr DFEdgeTable make_df_edge_table() {
   DFEdgeTable t{};
-  for (int idx = 0; idx < kTabEntries - 2; ++idx) {
-    int w = 1;
-    while ((1 << (w + 1)) - 2 <= idx) ++w;
-    const int n = 1 << w, e = idx - ((1 << w) - 2);
+  for (int idx = 0; idx < kTabEntries; ++idx) {
+    const int n = tab_n_of(idx), e = idx - tab_offset_n(n);
     const CS d = cos_sin_q8(8 * e + 4 + n, n);
     const float ch = (float)d.c, sh = (float)d.s;
     t.v[idx] = DF4{ch, (float)(d.c - (double)ch), sh, (float)(d.s - (double)sh)};
@@ -55,18 +53,23 @@ __constant__ cx::DFEdgeTable g_edge_df = cx::make_df_edge_table();
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles in flight
 
-template <int D, typename TIn, int W, int B>
+// Shape of one kernel: n bins (W = ceil(log2 n) bits per angle code), B norm
+// bits (4, 8, or 32 for fp32 norms), MODE; HB header bytes per row (8, none
+// for fp32 norms).
+template <int D, typename TIn, int N, int B, int MODE>
 struct Enc {
   using G = Geo<D>;
   using IT = RowTile<D, (int)sizeof(TIn)>;
   static constexpr int P = G::P, L = G::L, RW = G::RW;
   static constexpr int ESZ = (int)sizeof(TIn);
-  static constexpr int n = 1 << W;
+  static constexpr int n = N;
+  static constexpr int W = code_bits(N);
   static constexpr int AB = P * W / 8;        // angle record bytes per row
   static constexpr int NB = P * B / 8;        // norm record bytes per row
-  // A warp tile's records: RW*AB = 32 W and RW*NB = 32 B bytes, RW*8 header
+  static constexpr int HB = (MODE == TAC_NORM_FP32) ? 0 : 8;
+  // A warp tile's records: RW*AB = 32 W and RW*NB = 32 B bytes, RW*HB header
   // bytes: every segment is a whole number of 16-byte chunks.
-  static constexpr int NA = RW * AB / 16, NN = RW * NB / 16, NH = RW * 8 / 16;
+  static constexpr int NA = RW * AB / 16, NN = RW * NB / 16, NH = RW * HB / 16;
   static constexpr int NCH = NA + NN + NH;
   static constexpr int ROUNDS = (NCH + 31) / 32;
   // Input chunk map: 32 consecutive 16-byte chunks cover RPQ rows.
@@ -77,12 +80,12 @@ struct Enc {
   static constexpr int W_ANG = W_TP + G::TP_W;              // staged records: angle | norm | header
   static constexpr int W_NRM = W_ANG + RW * AB;
   static constexpr int W_HDR = W_NRM + RW * NB;
-  static constexpr int W_JOB = W_HDR + RW * 8;              // current job (WarpJob)
+  static constexpr int W_JOB = W_HDR + RW * HB;             // current job (WarpJob)
   static constexpr int WARP_B = W_JOB + 64;
   static constexpr int TABR = tab_copies(n, 8192);           // edge table copies
   static constexpr int OFF_TAB = kWarps * WARP_B;           // fp32 edge table of this n (TABR copies)
   static constexpr int SMEM = OFF_TAB + n * TABR * 8;
-  static_assert((RW * AB) % 16 == 0 && (RW * NB) % 16 == 0 && (RW * 8) % 16 == 0, "record segments");
+  static_assert((RW * AB) % 16 == 0 && (RW * NB) % 16 == 0 && (RW * HB) % 16 == 0, "record segments");
   static_assert(W_TP % 16 == 0 && W_ANG % 16 == 0 && W_JOB % 16 == 0 && WARP_B % 16 == 0, "alignment");
   static_assert(32 % CPR == 0 && RW % RPQ == 0, "chunk map");
 };
@@ -123,15 +126,23 @@ __device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
   e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
 }
 
+// v mod n for v in [-n, 2n).
+template <int N>
+__device__ __forceinline__ int wrap_bin(int v) {
+  if constexpr (is_pow2(N)) return v & (N - 1);
+  else return v < 0 ? v + N : (v >= N ? v - N : v);
+}
+
 // Candidate edge for the pair (E, O) (butterfly halves, y = (E + O, E - O))
-// and n = 2^W: Alg. 1's angle theta = pi/4 - angle(E, O) from the
+// and n bins: Alg. 1's angle theta = pi/4 - angle(E, O) from the
 // octant-reduced arctangent polynomial, in bins, floored (M + n/8 - angle,
-// rounded down onto the integer grid of M = 1.5 * 2^23).  The true bin is the
-// candidate or the next one whenever the polynomial's error (0.0038 rad) is
-// below half a bin, i.e. for every n <= 256.
-template <int W>
+// rounded down onto the integer grid of M = 1.5 * 2^23; for n not a multiple
+// of 8 the shift of M + n/8 onto that grid is below half a bin).  The true bin
+// is the candidate or the next one whenever the polynomial's error (0.0038
+// rad) is below half a bin, i.e. for every n <= 256.
+template <int N>
 __device__ __forceinline__ int candidate_edge(float E, float O) {
-  constexpr int n = 1 << W;
+  constexpr int n = N;
   constexpr float nb = (float)n * 0.15915494309189535f;  // bins per radian
   constexpr float c1 = (0.78539816f + 0.273f) * nb;       // atan(t) ~ t (pi/4 + 0.273 (1 - t))
   constexpr float c2 = 0.273f * nb;
@@ -142,20 +153,27 @@ __device__ __forceinline__ int candidate_edge(float E, float O) {
   float fb = (aO > aE) ? (0.25f * n - phi) : phi;              // angle of (|E|, |O|)
   fb = (E < 0.f) ? (0.5f * n - fb) : fb;                       // angle of (E, |O|)
   const float ab = __uint_as_float(__float_as_uint(fb) ^ (__float_as_uint(O) & 0x80000000u));
-  return __float_as_int(__fadd_rd(12582912.0f + 0.125f * n, -ab)) & (n - 1);
+  const int bits = __float_as_int(__fadd_rd(12582912.0f + 0.125f * n, -ab));
+  if constexpr (is_pow2(N)) {
+    return bits & (n - 1);
+  } else {
+    // 0x4B400000 = bits of M.  A zero pair gives NaN here (its code is decided
+    // by the exact path); the clamp keeps every table index inside [0, n).
+    const int e = wrap_bin<N>(bits - 0x4B400000);
+    return (int)min((uint32_t)e, (uint32_t)(n - 1));
+  }
 }
 
-// Alg. 1 bin of the pair (E, O) for n = 2^W by the edge test: the candidate
+// Alg. 1 bin of the pair (E, O) for n bins by the edge test: the candidate
 // edge, then the sign of the cross product with the edge direction (et: this
 // lane's copy of the replicated table, R copies).  Returns k; m is the signed
 // cross product (its magnitude is the certification margin).
-template <int W, int R>
+template <int N, int R>
 __device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et, float& m) {
-  constexpr int n = 1 << W;
-  const int e = candidate_edge<W>(E, O);
+  const int e = candidate_edge<N>(E, O);
   const float2 dir = et[e * R];
   m = __fmaf_rn(E, dir.x, -__fmul_rn(O, dir.y));
-  return (uint32_t)(e + 1 + (__float_as_int(m) >> 31)) & (uint32_t)(n - 1);
+  return (uint32_t)wrap_bin<N>(e + 1 + (__float_as_int(m) >> 31));
 }
 
 // Exact re-decision of pair i of warp-tile row rr by the whole warp (all lanes
@@ -167,21 +185,22 @@ __device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et
 // rounded to fp32 (scaled by a power of two when tiny, so the reciprocal sees
 // a normal number), the edge test m = E cos psi - O sin psi is evaluated in
 // double-float against the double-float edge direction.
-template <int D, typename TIn, int W, int B>
+template <int D, typename TIn, int N>
 __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uint8_t* in, int rr, int i,
                                                 int lane) {
-  using C = Enc<D, TIn, W, B>;
-  using IT = typename C::IT;
-  constexpr int n = 1 << W;
+  using G = Geo<D>;
+  using IT = RowTile<D, (int)sizeof(TIn)>;
+  constexpr int ESZ = (int)sizeof(TIn);
+  constexpr int P = G::P;
   float eh = 0.f, el = 0.f, oh = 0.f, ol = 0.f;
   const uint8_t* row = in + rr * IT::STRIDE;
 #pragma unroll
-  for (int j0 = 0; j0 < C::P; j0 += 32) {
+  for (int j0 = 0; j0 < P; j0 += 32) {
     const int jj = j0 + lane;
-    if (jj < C::P) {
+    if (jj < P) {
       const int e0 = 2 * jj, e1 = 2 * jj + 1;
       float x0, x1;
-      if constexpr (C::ESZ == 2) {
+      if constexpr (ESZ == 2) {
         const uint32_t u = *reinterpret_cast<const uint32_t*>(row + 4 * jj);
         x0 = bf16lo(u); x1 = bf16hi(u);
       } else {
@@ -211,8 +230,8 @@ __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uin
     eh *= 18446744073709551616.f; el *= 18446744073709551616.f;
     oh *= 18446744073709551616.f; ol *= 18446744073709551616.f;
   }
-  const int e = candidate_edge<W>(eh, oh);
-  const cx::DF4 dir = g_edge_df.v[tab_offset(W) + e];
+  const int e = candidate_edge<N>(eh, oh);
+  const cx::DF4 dir = g_edge_df.v[tab_offset_n(N) + e];
   const float p1 = __fmul_rn(eh, dir.ch), q1 = __fmaf_rn(eh, dir.ch, -p1);
   const float p2 = __fmul_rn(oh, dir.sh), q2 = __fmaf_rn(oh, dir.sh, -p2);
   float dd, t;
@@ -223,7 +242,7 @@ __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uin
   rest = __fmaf_rn(-oh, dir.sl, rest);
   rest = __fmaf_rn(-ol, dir.sh, rest);
   const float m = __fadd_rn(dd, rest);
-  return (e + (m >= 0.f ? 1 : 0)) & (n - 1);
+  return wrap_bin<N>(e + (m >= 0.f ? 1 : 0));
 }
 
 // Patch code i (W bits) of a staged angle record (one lane).
@@ -239,18 +258,20 @@ __device__ __forceinline__ void patch_code(uint8_t* rec, int i, int k) {
 }
 
 // Encode this lane's 8 pairs of warp-tile row r (lane l of the row) and stage
-// the records; W = log2 n, B = norm bits, MODE = TAC_NORM_LINEAR / TAC_NORM_LOG.
-template <int D, typename TIn, int W, int B, int MODE>
+// the records; N bins, B = norm bits, MODE = TAC_NORM_LINEAR / TAC_NORM_LOG /
+// TAC_NORM_FP32 (B = 32: the pair norms themselves, no header).
+template <int D, typename TIn, int N, int B, int MODE>
 __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const float2* et, int nrows,
                                           int lane, const uint2 (&msk)[8], const uint32_t* signs) {
   // (for bf16 only msk[m].x is used; the .y words are constant zero)
-  using C = Enc<D, TIn, W, B>;
+  using C = Enc<D, TIn, N, B, MODE>;
   using G = Geo<D>;
   using IT = typename C::IT;
   constexpr int P = C::P, L = C::L;
-  constexpr int n = 1 << W;
+  constexpr int n = N, W = C::W;
   constexpr int AB = C::AB, NB = C::NB;
-  constexpr int Lq = (1 << B) - 1;
+  constexpr bool FP32N = MODE == TAC_NORM_FP32;
+  constexpr int Lq = FP32N ? 0 : (1 << B) - 1;
   const int r = lane / L, l = lane % L;
   const bool live = r < nrows;
   static_assert(P == 8 * L, "geometry");
@@ -307,8 +328,10 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
 
   // ---- row constants: stored header (Sec. 3.3), Eq. 2 as code = floor(f(s) qs + qo) ----
   constexpr float k2 = 2.0f / (float)D;
-  float hmin, hmax, qs, qo, sfloor = 0.f;
-  if constexpr (MODE == TAC_NORM_LINEAR) {
+  float hmin = 0.f, hmax = 0.f, qs = 0.f, qo = 0.f, sfloor = 0.f;
+  if constexpr (FP32N) {
+    // no header: the norms are stored as they are (Sec. 3.1)
+  } else if constexpr (MODE == TAC_NORM_LINEAR) {
     hmin = sqrt_approx(smin * k2);
     hmax = sqrt_approx(smax * k2);
     const float sc = (float)Lq * rcp_approx(hmax - hmin);
@@ -347,6 +370,7 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   if constexpr (MODE == TAC_NORM_LINEAR) qs *= __uint_as_float((uint32_t)(127 + kk) << 23);
   else qo = __fmaf_rn((float)(2 * kk), qs, qo);
   const float sfl = sfloor * sigma;
+  (void)qs; (void)qo; (void)sfl;
   // Pairs whose norm is so small that the fp32 angle may be off by a quarter bin
   // are re-decided too: sqrt(s) < 4 n ty / pi.
   const float rthr = ty * (4.f * (float)n / 3.14159265f);
@@ -354,22 +378,28 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
 
   // ---- pass 2: angle codes (Alg. 1), norm codes (Eq. 2), packing ----
   uint32_t alo = 0, ahi = 0, nlo = 0, nhi = 0;
+  float rn[FP32N ? 8 : 1];                      // fp32 norms r_j = sqrt(2 s_j / d)
   float mmin = __int_as_float(0x7f800000);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     float m;
-    const uint32_t k = edge_test<W, C::TABR>(v[j].x, v[j].y, et, m);
+    const uint32_t k = edge_test<N, C::TABR>(v[j].x, v[j].y, et, m);
     mmin = fminf(mmin, fabsf(m));
-    float f;
-    if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_ftz(s[j] * sigma);
-    else f = lg2_ftz(fmaxf(s[j] * sigma, sfl));
-    const uint32_t c = min(__float2uint_rd(__fmaf_rn(f, qs, qo)), (uint32_t)Lq);
     // fields are disjoint and k < n, c <= Lq: the adds are ORs (one IMAD each)
-    const int sa = j * W, sn = j * B;
+    const int sa = j * W;
     if (sa + W <= 32) alo += k << sa;
     else if (sa >= 32) ahi += k << (sa - 32);
     else { alo += k << sa; ahi += k >> (32 - sa); }
-    if (sn < 32) nlo += c << sn; else nhi += c << (sn - 32);
+    if constexpr (FP32N) {
+      rn[j] = sqrt_approx(s[j] * k2);
+    } else {
+      float f;
+      if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_ftz(s[j] * sigma);
+      else f = lg2_ftz(fmaxf(s[j] * sigma, sfl));
+      const uint32_t c = min(__float2uint_rd(__fmaf_rn(f, qs, qo)), (uint32_t)Lq);
+      const int sn = j * B;
+      if (sn < 32) nlo += c << sn; else nhi += c << (sn - 32);
+    }
   }
   uint32_t fm = 0;
   if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; }
@@ -377,7 +407,7 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       float m;
-      edge_test<W, C::TABR>(v[j].x, v[j].y, et, m);
+      edge_test<N, C::TABR>(v[j].x, v[j].y, et, m);
       if (fabsf(m) < tau || s[j] < sthr) fm |= 1u << j;
     }
   }
@@ -386,8 +416,14 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   // ---- stage the records ----
   if (live) {
     store_bytes<W>(wsm + C::W_ANG + r * AB + l * W, alo, ahi);
-    store_bytes<B>(wsm + C::W_NRM + r * NB + l * B, nlo, nhi);
-    if (l == 0) reinterpret_cast<float2*>(wsm + C::W_HDR)[r] = make_float2(hmin, hmax);
+    if constexpr (FP32N) {
+      float4* dst = reinterpret_cast<float4*>(wsm + C::W_NRM + r * NB + l * 32);
+      dst[0] = make_float4(rn[0], rn[1], rn[2], rn[3]);
+      dst[1] = make_float4(rn[4], rn[5], rn[6], rn[7]);
+    } else {
+      store_bytes<B>(wsm + C::W_NRM + r * NB + l * B, nlo, nhi);
+      if (l == 0) reinterpret_cast<float2*>(wsm + C::W_HDR)[r] = make_float2(hmin, hmax);
+    }
   }
   __syncwarp();
 
@@ -402,7 +438,7 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
       const int j = __ffs(mm) - 1;
       mm &= mm - 1;
       const int i = 8 * ol + j;
-      const int kk = exact_angle_code<D, TIn, W, B>(signs, in, rr, i, lane);
+      const int kk = exact_angle_code<D, TIn, N>(signs, in, rr, i, lane);
       if (lane == 0) patch_code<W>(wsm + C::W_ANG + rr * AB, i, kk);
     }
     __syncwarp();
@@ -411,7 +447,7 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
 
 // Records of a tail tile (nrows < RW) or of scattered slots, from the staged
 // records to the planes.
-template <int AB, int NB>
+template <int AB, int NB, int HB>
 __device__ __noinline__ void copy_out_slow(const WarpJob* wj, const uint8_t* sang, const uint8_t* snrm,
                                            const uint8_t* shdr, int64_t row0, int nrows, int lane) {
   if (wj->slot == nullptr) {
@@ -420,7 +456,8 @@ __device__ __noinline__ void copy_out_slow(const WarpJob* wj, const uint8_t* san
     uint8_t* gh = wj->hdr + row0 * 8;
     for (int q = lane; q < nrows * AB; q += 32) ga[q] = sang[q];
     for (int q = lane; q < nrows * NB; q += 32) gn[q] = snrm[q];
-    for (int q = lane; q < nrows * 8; q += 32) gh[q] = shdr[q];
+    if constexpr (HB > 0)
+      for (int q = lane; q < nrows * HB; q += 32) gh[q] = shdr[q];
   } else if (lane < nrows) {
     const int64_t s = wj->slot[row0 + lane];
     if (s < 0 || s >= wj->capacity) return;  // out-of-range slots are skipped
@@ -442,13 +479,13 @@ __device__ __noinline__ void copy_out_slow(const WarpJob* wj, const uint8_t* san
     } else {
       for (int q = 0; q < NB / 4; ++q) reinterpret_cast<uint32_t*>(gn)[q] = reinterpret_cast<const uint32_t*>(nn)[q];
     }
-    reinterpret_cast<float2*>(wj->hdr)[s] = reinterpret_cast<const float2*>(shdr)[lane];
+    if constexpr (HB > 0) reinterpret_cast<float2*>(wj->hdr)[s] = reinterpret_cast<const float2*>(shdr)[lane];
   }
 }
 
-template <int D, typename TIn, int W, int B, int MODE>
+template <int D, typename TIn, int N, int B, int MODE>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __grid_constant__ EncParams p) {
-  using C = Enc<D, TIn, W, B>;
+  using C = Enc<D, TIn, N, B, MODE>;
   using IT = typename C::IT;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
@@ -560,7 +597,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
         const int ch = q * 32 + lane;
         if (ch < C::NA) { o_dst[q] = J.codes + 16 * ch; o_step[q] = C::RW * C::AB; }
         else if (ch < C::NA + C::NN) { o_dst[q] = J.norms + 16 * (ch - C::NA); o_step[q] = C::RW * C::NB; }
-        else { o_dst[q] = J.hdr + 16 * (ch - C::NA - C::NN); o_step[q] = C::RW * 8; }
+        else { o_dst[q] = J.hdr + 16 * (ch - C::NA - C::NN); o_step[q] = C::RW * C::HB; }
         o_dst[q] += (int64_t)rel * o_step[q];
       }
       if (lane == 0) {
@@ -575,7 +612,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
     }
     const int nrows = c_left < C::RW ? (int)c_left : C::RW;
     const uint8_t* in = wsm + C::W_IN + stage * IT::BYTES;
-    tile_body<D, TIn, W, B, MODE>(in, wsm, etab + (lane % C::TABR), nrows, lane, msk, wj->signs);
+    tile_body<D, TIn, N, B, MODE>(in, wsm, etab + (lane % C::TABR), nrows, lane, msk, wj->signs);
     __syncwarp();
     if (c_dense && nrows == C::RW) {
 #pragma unroll
@@ -585,7 +622,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
           *reinterpret_cast<uint4*>(o_dst[q]) = *reinterpret_cast<const uint4*>(wsm + C::W_ANG + 16 * ch);
       }
     } else {
-      copy_out_slow<C::AB, C::NB>(wj, wsm + C::W_ANG, wsm + C::W_NRM, wsm + C::W_HDR, c_row0, nrows, lane);
+      copy_out_slow<C::AB, C::NB, C::HB>(wj, wsm + C::W_ANG, wsm + C::W_NRM, wsm + C::W_HDR, c_row0, nrows, lane);
     }
 #pragma unroll
     for (int q = 0; q < C::ROUNDS; ++q) o_dst[q] += o_step[q];
@@ -599,10 +636,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
 // ---------------------------------------------------------------------------
 // Host-side launch helpers (called from tac_api.cu).
 // ---------------------------------------------------------------------------
-template <int D, typename TIn, int W, int B, int MODE>
+template <int D, typename TIn, int N, int B, int MODE>
 static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_t st) {
-  using C = Enc<D, TIn, W, B>;
-  auto kern = encode_kernel<D, TIn, W, B, MODE>;
+  using C = Enc<D, TIn, N, B, MODE>;
+  auto kern = encode_kernel<D, TIn, N, B, MODE>;
   static int configured[64] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -623,19 +660,23 @@ static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_
   return cudaGetLastError();
 }
 
+// One kernel per supported (n, norm bits, mode): n in {2, 4, ..., 256, 48, 56},
+// (B, mode) in {(4, linear), (4, log), (8, linear), (8, log), (32, fp32)}.
 template <int D, typename TIn>
-static cudaError_t launch_encode_t(const EncParams& p, int w, int b, int mode, int sms, cudaStream_t st) {
-#define TAC_ENC_CASE(WW)                                                                         \
-  case (WW - 1) * 4 + 0: return launch_encode_v<D, TIn, WW, 4, TAC_NORM_LINEAR>(p, sms, st);     \
-  case (WW - 1) * 4 + 1: return launch_encode_v<D, TIn, WW, 4, TAC_NORM_LOG>(p, sms, st);        \
-  case (WW - 1) * 4 + 2: return launch_encode_v<D, TIn, WW, 8, TAC_NORM_LINEAR>(p, sms, st);     \
-  case (WW - 1) * 4 + 3: return launch_encode_v<D, TIn, WW, 8, TAC_NORM_LOG>(p, sms, st);
-  switch ((w - 1) * 4 + (b == 8 ? 2 : 0) + (mode == TAC_NORM_LOG ? 1 : 0)) {
-    TAC_ENC_CASE(1) TAC_ENC_CASE(2) TAC_ENC_CASE(3) TAC_ENC_CASE(4)
-    TAC_ENC_CASE(5) TAC_ENC_CASE(6) TAC_ENC_CASE(7) TAC_ENC_CASE(8)
-    default: break;
+static cudaError_t launch_encode_t(const EncParams& p, int n, int b, int mode, int sms, cudaStream_t st) {
+#define TAC_ENC_N(NN)                                                                                   \
+  if (n == NN) {                                                                                        \
+    if (mode == TAC_NORM_FP32) return b == 32 ? launch_encode_v<D, TIn, NN, 32, TAC_NORM_FP32>(p, sms, st) \
+                                              : cudaErrorInvalidValue;                                  \
+    if (b == 4) return mode == TAC_NORM_LOG ? launch_encode_v<D, TIn, NN, 4, TAC_NORM_LOG>(p, sms, st)     \
+                                            : launch_encode_v<D, TIn, NN, 4, TAC_NORM_LINEAR>(p, sms, st); \
+    if (b == 8) return mode == TAC_NORM_LOG ? launch_encode_v<D, TIn, NN, 8, TAC_NORM_LOG>(p, sms, st)     \
+                                            : launch_encode_v<D, TIn, NN, 8, TAC_NORM_LINEAR>(p, sms, st); \
+    return cudaErrorInvalidValue;                                                                       \
   }
-#undef TAC_ENC_CASE
+  TAC_ENC_N(2) TAC_ENC_N(4) TAC_ENC_N(8) TAC_ENC_N(16) TAC_ENC_N(32) TAC_ENC_N(64) TAC_ENC_N(128)
+  TAC_ENC_N(256) TAC_ENC_N(48) TAC_ENC_N(56)
+#undef TAC_ENC_N
   return cudaErrorInvalidValue;
 }
 
@@ -653,9 +694,9 @@ static cudaError_t launch_encode_t(const EncParams& p, int w, int b, int mode, i
 #define TAC_INST_F32 0
 #endif
 #define TAC_ENC_INSTANCE(DD, NAME, T)                                                                 \
-  cudaError_t launch_encode_##DD##_##NAME(const EncParams& p, int w, int b, int mode, int sms,       \
+  cudaError_t launch_encode_##DD##_##NAME(const EncParams& p, int n, int b, int mode, int sms,       \
                                           cudaStream_t st) {                                         \
-    return launch_encode_t<DD, T>(p, w, b, mode, sms, st);                                           \
+    return launch_encode_t<DD, T>(p, n, b, mode, sms, st);                                           \
   }
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 16 && TAC_INST_BF16)
 TAC_ENC_INSTANCE(16, bf16, __nv_bfloat16)

@@ -13,6 +13,8 @@ norm codes    bit-exact wherever the oracle's Eq. 2 pre-round value lies more th
               beta_i from a rounding midpoint, beta_i the propagated bound of the
               fp32 norm, header and Eq. 2 arithmetic; inside, a code may differ by
               one level and is counted (rate reported, must stay <= 1e-4).
+fp32 norms    (mode 2, Sec. 3.1) |r_gpu - r| <= (2/sqrt d) gamma + 4 u r, r the oracle's
+              exact pair norm; there is no header.
 decode        on identical codes: fp32 out |y - v| <= 1e-5 ||x^||;
               bf16 out |y - v| <= ulp_bf16(v)/2 + 1e-3 ||x^||  (v = oracle fp64 output).
 """
@@ -36,19 +38,27 @@ def signs_pm1(words: np.ndarray, d: int) -> np.ndarray:
     return np.array([-1 if (int(words[j // 32]) >> (j % 32)) & 1 else 1 for j in range(d)], dtype=np.int8)
 
 
+def code_bits(n: int) -> int:
+    """Bits of one angle code: ceil(log2 n)."""
+    return int(math.ceil(math.log2(n)))
+
+
+FP32_MODE = 2
+
+
 def gpu_codes(orc, cache, rows: int | None = None, slots: np.ndarray | None = None):
-    """(k, c, hdr) read back from a device cache (optionally only some slots)."""
+    """(k, c, hdr) read back from a device cache (optionally only some slots).
+    With fp32 norms c holds the norms' fp32 bit patterns and hdr is None."""
     cfg = cache.cfg
     codes, norms, hdr = cache.planes()
-    if slots is not None:
-        codes, norms, hdr = codes[slots], norms[slots], hdr[slots]
-    elif rows is not None:
-        codes, norms, hdr = codes[:rows], norms[:rows], hdr[:rows]
+    sel = slots if slots is not None else (slice(0, rows) if rows is not None else slice(None))
+    codes, norms = codes[sel], norms[sel]
+    if hdr is not None:
+        hdr = np.array(hdr[sel], dtype=np.float32)
     P = cfg.d // 2
-    w = int(math.log2(cfg.n_angle))
-    k = orc.unpack(codes, P, w)
+    k = orc.unpack(codes, P, code_bits(cfg.n_angle))
     c = orc.unpack(norms, P, cfg.norm_bits)
-    return k, c, np.array(hdr, dtype=np.float32)
+    return k, c, hdr
 
 
 def _gamma(x64: np.ndarray) -> np.ndarray:
@@ -76,8 +86,18 @@ def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, m
     assert st["angle_mismatch_outside_band"] == 0, (label, np.argwhere(outside)[:5])
     assert st["angle_mismatch"] <= 1e-6 * st["codes"], (label, st)
 
-    # ---- header ----
     gam = _gamma(x64)
+    if mode == FP32_MODE:
+        # ---- fp32 norms: values, not codes ----
+        r = ref["r"]
+        rg = np.ascontiguousarray(c, dtype=np.int32).view(np.float32).astype(np.float64)
+        eps_r = (2.0 / math.sqrt(d)) * gam[:, None] + 4 * U * r + 1e-45
+        err = np.abs(rg - r)
+        st["norm_max_err_over_bound"] = float((err / eps_r).max()) if rows else 0.0
+        assert np.all(err <= eps_r), (label, st)
+        return st
+
+    # ---- header ----
     hmax_o = ref["hdr"][:, 1].astype(np.float64)
     eps_h = (2.0 / math.sqrt(d)) * gam + 4 * U * hmax_o + 1e-45
     dh = np.abs(hdr.astype(np.float64) - ref["hdr"].astype(np.float64))

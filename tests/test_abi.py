@@ -61,6 +61,25 @@ def test_plane_geometry(tac_host):
                     assert tac_host.codes_bytes(cfg, cap) == cap * (d // 2 * w // 8)
 
 
+def test_plane_geometry_extra_shapes(tac_host):
+    """n = 48, 56 (Table 1) store ceil(log2 n) = 6 bits per code; fp32 norms
+    (Sec. 3.1) store 4 bytes per pair and no header plane."""
+    for d in (16, 32, 64, 128):
+        for n in (48, 56):
+            cfg = tac_host.LayerCfg(d, n, 8, 0)
+            assert tac_host.angle_row_bytes(cfg) == d // 2 * 6 // 8
+        for n in (16, 56, 256):
+            cfg = tac_host.LayerCfg(d, n, 32, tac_host.NORM_FP32)
+            assert tac_host.norm_row_bytes(cfg) == d // 2 * 4
+            for cap in (0, 1, 7, 1000):
+                off = tac_host.header_offset(cfg, cap)
+                assert off == (cap * d // 2 * 4 + 15) // 16 * 16
+                assert tac_host.norms_bytes(cfg, cap) == off
+    r = tac_host.rates(128, [56] * 4, [48] * 4, 32, 32)
+    assert abs(r["angle_bits"] - (math.log2(56) + math.log2(48)) / 4) < 1e-12
+    assert abs(r["total_bits"] - (r["angle_bits"] + 16)) < 1e-12 and r["stored_angle_bits"] == 3.0
+
+
 def test_record_bytes_match_rate_accounting(tac_host, orc):
     # Eq. 3 total bits per element x d / 8 = record bytes per row (angle + norm + 8-byte header)
     for n in (16, 64, 256):
@@ -101,10 +120,13 @@ def test_invalid_arguments_rejected_before_launch(tac_host):
         (dict(d=100), tac_host.TAC_E_INVAL),
         (dict(d=256), tac_host.TAC_E_UNSUPPORTED),
         (dict(n=3), tac_host.TAC_E_UNSUPPORTED),
+        (dict(n=24), tac_host.TAC_E_UNSUPPORTED),
         (dict(n=0), tac_host.TAC_E_INVAL),
         (dict(n=512), tac_host.TAC_E_UNSUPPORTED),
         (dict(b=5), tac_host.TAC_E_UNSUPPORTED),
         (dict(b=0), tac_host.TAC_E_INVAL),
+        (dict(b=32), tac_host.TAC_E_INVAL),
+        (dict(mode=2, b=8), tac_host.TAC_E_INVAL),
         (dict(mode=7), tac_host.TAC_E_INVAL),
     ]
     for kw, want in cases:

@@ -19,14 +19,15 @@ def _oracle_cache(tac, orc, cfg, ref):
     """A device cache holding the oracle's own records (for decode on identical codes)."""
     torch = _torch()
     rows = ref["k"].shape[0]
-    w = int(math.log2(cfg.n_angle))
+    w = parity.code_bits(cfg.n_angle)
     cache = tac.Cache.empty(cfg, rows)
     ang = orc.pack(ref["k"], w).reshape(-1)
     nrm = orc.pack(ref["c"], cfg.norm_bits).reshape(-1)
     off = tac.header_offset(cfg, rows)
     nb = np.zeros(tac.norms_bytes(cfg, rows), dtype=np.uint8)
     nb[: nrm.size] = nrm
-    nb[off: off + 8 * rows] = ref["hdr"].astype(np.float32).view(np.uint8).reshape(-1)
+    if cfg.norm_mode != tac.NORM_FP32:
+        nb[off: off + 8 * rows] = ref["hdr"].astype(np.float32).view(np.uint8).reshape(-1)
     if ang.size:
         cache.codes[: ang.size].copy_(torch.from_numpy(ang))
     if nb.size:
@@ -57,7 +58,7 @@ def check_roundtrip(tac, orc, x, d, n, b, mode, seed=0, layer=0, kv=0, label="",
     # end to end: GPU encode -> GPU decode equals the oracle decode of the GPU's codes
     y2 = tac.decode(cache, cfg, dtype=torch.float32)
     torch.cuda.synchronize()
-    v2 = orc.decode(k, c, hdr, s, n, b, mode)
+    v2 = orc.decode(k, c, hdr if hdr is not None else ref["hdr"], s, n, b, mode)
     parity.compare_decode(parity.to_f64(y2), v2, "fp32", label=f"{label} e2e")
     return st
 
@@ -96,6 +97,30 @@ def test_small_d_and_dtypes(tac_gpu, orc, d, dt, b, mode):
     x = x.to(torch.bfloat16 if dt == "bf16" else torch.float32).contiguous()
     for n in (16, 256):
         check_roundtrip(tac_gpu, orc, x, d, n, b, mode, seed=3, layer=2, kv=1, label=f"d{d} {dt} n{n}")
+
+
+@pytest.mark.parametrize("n", [48, 56])
+@pytest.mark.parametrize("b,mode", [(8, 0), (4, 1), (32, 2)])
+def test_non_power_of_two_bins(tac_gpu, orc, n, b, mode):
+    """n = 48, 56 (Table 1): 6-bit codes, bins wrap at n."""
+    w = workloads.CONFIGS["mistral7b"]
+    x = _rows(w, 777, seed=n + b, layer=5, kv=mode % 2)
+    check_roundtrip(tac_gpu, orc, x, 128, n, b, mode, layer=5, kv=mode % 2, label=f"n={n} b={b} m={mode}")
+    wl = workloads.CONFIGS["llama1b"]
+    x = workloads.block(wl, 2, 1, tokens=60, seed=n, device="cuda")
+    check_roundtrip(tac_gpu, orc, x, 64, n, b, mode, seed=1, layer=2, kv=1, label=f"d64 n={n} b={b} m={mode}")
+
+
+@pytest.mark.parametrize("d", [16, 32, 64, 128])
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+def test_fp32_norms(tac_gpu, orc, d, dt):
+    """fp32 pair norms (Sec. 3.1, the angle-only configuration of Tables 1-4)."""
+    torch = _torch()
+    w = workloads.CONFIGS["mistral7b" if d == 128 else "llama1b"]
+    x = workloads.block(w, 3, 0, tokens=50, seed=d, device="cuda")[:, :d]
+    x = x.to(torch.bfloat16 if dt == "bf16" else torch.float32).contiguous()
+    for n in (2, 64, 256, 56):
+        check_roundtrip(tac_gpu, orc, x, d, n, 32, 2, seed=4, layer=3, kv=0, label=f"fp32 norms d{d} {dt} n{n}")
 
 
 def test_d128_fp32_input(tac_gpu, orc):
