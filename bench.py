@@ -67,7 +67,9 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["tac", "reference"], default="tac")
-    ap.add_argument("--config", default="mistral7b", choices=["mistral7b", "llama1b", "append", "longctx"])
+    ap.add_argument("--config", default="mistral7b",
+                    choices=["mistral7b", "llama1b", "append", "longctx", "mistral7b_angle", "mistral7b_norm8",
+                             "tinyllama_n56"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
@@ -150,9 +152,12 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # workloads
 # ---------------------------------------------------------------------------
-def record_bytes(d, n, b):
+def record_bytes(d, n, b, mode=0):
+    """Packed record bytes per row: ceil(log2 n)-bit angle codes, b-bit norms and
+    the 8-byte (r_min, r_max) header (no header with fp32 norms)."""
     import math
-    return d // 2 * int(math.log2(n)) // 8 + d // 2 * b // 8 + 8
+    hdr = 0 if mode == workloads.NORM_FP32 else 8
+    return d // 2 * int(math.ceil(math.log2(n))) // 8 + d // 2 * b // 8 + hdr
 
 
 def config_desc(name):
@@ -164,9 +169,12 @@ def config_desc(name):
                 "codebooks as mistral7b; encode only")
     w = workloads.CONFIGS[name]
     sched = "early-boost" if len(set(w.n_k)) > 1 else "uniform"
+
+    def norms(b, mode):
+        return "fp32" if mode == workloads.NORM_FP32 else f"{b}-bit {'log' if mode == workloads.NORM_LOG else 'linear'}"
     return (f"{name}-shaped KV cache: {w.layers} L x 2 (K,V) x {w.heads} KV heads x {w.tokens} T x d {w.d}, "
             f"{w.dtype}; {sched} n_K={sorted(set(w.n_k))} n_V={sorted(set(w.n_v))}; "
-            f"K {w.b_k}-bit linear / V {w.b_v}-bit log norms")
+            f"K {norms(w.b_k, w.mode_k)} / V {norms(w.b_v, w.mode_v)} norms")
 
 
 class Workset:
@@ -194,7 +202,7 @@ class Workset:
                 self.x_all[bi].copy_(x.view(w.heads, a["seqs"], d).transpose(0, 1).reshape(rows, d))
                 cache = tac.Cache.empty(cfg, cap, device=device)
                 self.enc_jobs.append(tac.EncodeJob(cfg, self.x_all[bi], cache, slots))
-                self.enc_bytes += rows * (2 * d + record_bytes(d, n, b))
+                self.enc_bytes += rows * (2 * d + record_bytes(d, n, b, mode))
             self.tokens = a["seqs"]
             self.y_all = None
             self.rows_per_launch = None   # scattered single-token rows: no traffic figure
@@ -214,7 +222,7 @@ class Workset:
             cache = tac.Cache.empty(cfg, R, device=device)
             self.enc_jobs.append(tac.EncodeJob(cfg, self.x_all[bi], cache))
             self.dec_jobs.append(tac.DecodeJob(cfg, cache, self.y_all[bi]))
-            rb = record_bytes(d, n, b)
+            rb = record_bytes(d, n, b, mode)
             self.enc_bytes += R * (2 * d + rb)
             self.dec_bytes += R * (rb + 2 * d)
         self.tokens = w.tokens
@@ -251,7 +259,7 @@ def run_oracle(w, sample, threads, do_decode=True):
         d, n, b, mode = w.codebook(l, kv)
         s = oracle.signs(0, l, kv, d)
         r = oracle.encode_threads(x, s, n, b, mode, threads)
-        rb = record_bytes(d, n, b)
+        rb = record_bytes(d, n, b, mode)
         nbytes += x.shape[0] * (2 * d + rb)
         if do_decode:
             oracle.decode_threads(r["k"], r["c"], r["hdr"], s, n, b, mode, threads)

@@ -26,7 +26,7 @@ from dataclasses import dataclass
 import numpy as np
 
 K, V = 0, 1
-NORM_LINEAR, NORM_LOG = 0, 1
+NORM_LINEAR, NORM_LOG, NORM_FP32 = 0, 1, 2
 
 
 @dataclass(frozen=True)
@@ -83,6 +83,20 @@ def _make_configs():
     # 5. Long-context decode sweep: 28 L x 4 h x d 128, T 131072 (codebooks swept).
     cfgs["longctx"] = Workload("longctx", 28, 4, 131072, 128, "bf16", 1.0, 0.01, 20.0, 0.0,
                                (64,) * 28, (64,) * 28)
+    # Paper variants (Sec. 3.1 / 3.3, Tables 1-5) on the same value model:
+    #  - Mistral-7B angle-only: fp32 pair norms, early-boost (256, 128) on layers
+    #    0-3 and the K128/V64 baseline elsewhere (Table 3's Mistral row);
+    nk, nv = _boost(32, 4, (256, 128), (128, 64))
+    cfgs["mistral7b_angle"] = Workload("mistral7b_angle", 32, 8, 32768, 128, "bf16", 1.0, 0.01, 20.0, 0.0,
+                                       nk, nv, 32, NORM_FP32, 32, NORM_FP32)
+    #  - Mistral-7B norm8: 8-bit linear norms for K and V (Table 5), codebooks of config 3;
+    nk, nv = _boost(32, 4, (256, 256), (64, 64))
+    cfgs["mistral7b_norm8"] = Workload("mistral7b_norm8", 32, 8, 32768, 128, "bf16", 1.0, 0.01, 20.0, 0.0,
+                                       nk, nv, 8, NORM_LINEAR, 8, NORM_LINEAR)
+    #  - TinyLlama-shaped (22 L x 4 KV heads x d 64) with the non-power-of-two n = 56
+    #    of Table 1 on every layer, fp32 norms.
+    cfgs["tinyllama_n56"] = Workload("tinyllama_n56", 22, 4, 32768, 64, "bf16", 0.5, 0.02, 10.0, 0.0,
+                                     (56,) * 22, (56,) * 22, 32, NORM_FP32, 32, NORM_FP32)
     return cfgs
 
 
