@@ -76,6 +76,8 @@ def parse_args():
     ap.add_argument("--e2e-chunk", type=int, default=8, help="(layer, K/V) blocks per e2e pipeline chunk")
     ap.add_argument("--tokens", type=int, default=0,
                     help="override tokens per (layer, K/V) block (smaller cases for profiling)")
+    ap.add_argument("--probe", choices=["rd"], default=None,
+                    help="rd: rate-distortion probe (relative MSE vs n on the workload distributions)")
     ap.add_argument("--cpu-rows", type=int, default=400_000,
                     help="rows in the bounded oracle sample (CPU baseline / reference arm)")
     return ap.parse_args()
@@ -396,8 +398,46 @@ def run_e2e(tac, ws, world, dev, steps, chunk_blocks, step_bytes, barrier):
     return out
 
 
+def probe_rd(args):
+    """Rate-distortion probe: relative reconstruction MSE (sum |x^ - x|^2 / sum |x|^2)
+    of GPU encode -> decode with fp32 norms (angle-only) for every supported n,
+    on blocks of the workload distributions, next to the uniform-angle law
+    2 - 2 sin(pi/n)/(pi/n).  Tests the power-of-two aliasing conjecture (n = 56
+    vs 64) and the effect of the non-uniform angle density of channel-scaled rows."""
+    import math
+    import torch
+    from paper_2603_27467_gb300 import build as tb
+    tb.build()
+    import paper_2603_27467_gb300 as tac
+    tac.load()
+    ns = [16, 32, 48, 56, 64, 128, 256]
+    out = {}
+    for name in ("mistral7b", "llama1b", "tinyllama_n56"):
+        w = workloads.CONFIGS[name]
+        layers = sorted({0, w.layers // 2, w.layers - 1})
+        res = {}
+        for n in ns:
+            err = tot = 0.0
+            for l in layers:
+                for kv in (workloads.K, workloads.V):
+                    x = workloads.block(w, l, kv, tokens=4096, device="cuda", dtype=torch.bfloat16)
+                    cfg = tac.layer_cfg(w.d, n, 32, tac.NORM_FP32, 0, l, kv)
+                    y = tac.decode(tac.encode(x, cfg), cfg, dtype=torch.float32)
+                    xd = x.double()
+                    err += float((y.double() - xd).pow(2).sum())
+                    tot += float(xd.pow(2).sum())
+            res[str(n)] = err / tot
+        out[name] = res
+    law = {str(n): 2 - 2 * math.sin(math.pi / n) / (math.pi / n) for n in ns}
+    print(json.dumps({"probe": "rate-distortion", "norms": "fp32", "tokens_per_block": 4096,
+                      "rel_mse": out, "uniform_angle_law": law}), flush=True)
+
+
 def main():
     args = parse_args()
+    if args.probe == "rd":
+        probe_rd(args)
+        return
     if args.impl == "reference":
         run_reference(args)
         return
