@@ -72,6 +72,8 @@ def _load():
         lib.orc_avg_angle_bits.argtypes = [c_int, vp, vp]
         lib.orc_total_bits.restype = c_dbl
         lib.orc_total_bits.argtypes = [c_dbl, c_dbl, c_int]
+        lib.orc_attend.restype = c_int
+        lib.orc_attend.argtypes = [vp, c_int, vp, vp, c_i64, c_int, c_dbl, vp]
         _lib = lib
         return lib
 
@@ -188,6 +190,18 @@ def avg_angle_bits(nK, nV) -> float:
 def total_bits(b_angle: float, b_norm: float, d: int) -> float:
     """Eq. 3: b_angle + b_norm / 2 + 64 / d."""
     return float(_load().orc_total_bits(b_angle, b_norm, d))
+
+
+def attend(q: np.ndarray, khat: np.ndarray, vhat: np.ndarray, scale: float) -> np.ndarray:
+    """Softmax attention of q (nq x d) over decoded rows khat, vhat (T x d), fp64."""
+    q = np.ascontiguousarray(q, dtype=np.float64)
+    khat = np.ascontiguousarray(khat, dtype=np.float64)
+    vhat = np.ascontiguousarray(vhat, dtype=np.float64)
+    nq, d = q.shape
+    out = np.empty((nq, d), dtype=np.float64)
+    if _load().orc_attend(_ptr(q), nq, _ptr(khat), _ptr(vhat), khat.shape[0], d, float(scale), _ptr(out)):
+        raise ValueError("orc_attend failed")
+    return out
 
 
 def encode_threads(x: np.ndarray, s: np.ndarray, n: int, b: int, mode: int,

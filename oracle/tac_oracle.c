@@ -325,3 +325,42 @@ double orc_avg_angle_bits(int L, const int* nK, const int* nV) {
 double orc_total_bits(double b_angle, double b_norm, int d) {
   return b_angle + b_norm / 2.0 + 64.0 / (double)d;
 }
+
+/*
+ * Attention of nq query vectors over T decoded cache vectors (the consumer of
+ * the Sec. 3.1 reconstruction; the paper evaluates its codes through a model's
+ * attention, it does not describe a kernel for it):
+ *   s_t = scale * (q . k^_t),  p_t = exp(s_t - max_t s_t) / sum_t exp(...),
+ *   out = sum_t p_t v^_t
+ * with k^_t, v^_t the decoded K and V rows (orc_decode).  Plain fp64.
+ *   q     nq x d, khat, vhat  T x d, out  nq x d.  T >= 1.
+ */
+int orc_attend(const double* q, int nq, const double* khat, const double* vhat, int64_t T, int d,
+               double scale, double* out) {
+  if (nq < 1 || T < 1 || d < 1) return 1;
+  double* s = (double*)malloc(sizeof(double) * (size_t)T);
+  if (!s) return 2;
+  for (int a = 0; a < nq; ++a) {
+    const double* qa = q + (size_t)a * d;
+    double mx = -INFINITY;
+    for (int64_t t = 0; t < T; ++t) {
+      double acc = 0.0;
+      for (int j = 0; j < d; ++j) acc += qa[j] * khat[(size_t)t * d + j];
+      s[t] = scale * acc;
+      if (s[t] > mx) mx = s[t];
+    }
+    double den = 0.0;
+    for (int64_t t = 0; t < T; ++t) {
+      s[t] = exp(s[t] - mx);
+      den += s[t];
+    }
+    double* o = out + (size_t)a * d;
+    for (int j = 0; j < d; ++j) o[j] = 0.0;
+    for (int64_t t = 0; t < T; ++t) {
+      const double p = s[t] / den;
+      for (int j = 0; j < d; ++j) o[j] += p * vhat[(size_t)t * d + j];
+    }
+  }
+  free(s);
+  return 0;
+}

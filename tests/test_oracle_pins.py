@@ -443,3 +443,40 @@ def test_payload_bits_formula(orc):
             nrm = orc.pack(codes, b).nbytes * 8
             assert (ang + nrm) / d == math.log2(n) / 2 + b / 2
             assert (ang + nrm + 64) / d == orc.total_bits(math.log2(n) / 2, b, d)
+
+
+# ---------------------------------------------------------------------------
+# Attention over decoded vectors (the consumer of the Sec. 3.1 reconstruction)
+# ---------------------------------------------------------------------------
+def test_attend_special_cases(orc):
+    rng = np.random.default_rng(40)
+    d = 64
+    k = rng.standard_normal((5, d))
+    v = rng.standard_normal((5, d))
+    q = rng.standard_normal((3, d))
+    # one token: every query returns it
+    assert np.allclose(orc.attend(q, k[:1], v[:1], 0.3), np.repeat(v[:1], 3, axis=0), atol=1e-14)
+    # q = 0: uniform weights, the mean of the values
+    assert np.allclose(orc.attend(np.zeros((1, d)), k, v, 1.0), v.mean(axis=0, keepdims=True), atol=1e-14)
+    # two tokens: weights sigmoid(delta), delta the score difference (closed form)
+    qq = np.zeros((1, d)); qq[0, 3] = 1.0
+    kk = np.zeros((2, d)); kk[0, 3], kk[1, 3] = 2.0, -0.5
+    w0 = 1.0 / (1.0 + math.exp(-(0.7 * 2.0 - 0.7 * -0.5)))
+    assert np.allclose(orc.attend(qq, kk, v[:2], 0.7), w0 * v[0] + (1 - w0) * v[1], atol=1e-14)
+    # hard limit: a large scale selects the value of the highest score
+    s = q @ k.T
+    got = orc.attend(q, k, v, 1e4)
+    assert np.allclose(got, v[np.argmax(s, axis=1)], atol=1e-9)
+
+
+def test_attend_rotated_domain_identity(orc):
+    """q . (D H y) = (H D q) . y for every y: scores can be taken against the
+    rotated query without transforming each decoded row back."""
+    d = 128
+    rng = np.random.default_rng(41)
+    s = orc.signs(5, 3, 0, d)
+    q = rng.standard_normal((4, d))
+    y = rng.standard_normal((50, d))
+    khat = orc.transform(y, np.ones(d, dtype=np.int8)) * s      # D H y (H symmetric)
+    qr = orc.transform(q, s)                                     # H D q
+    assert np.allclose(q @ khat.T, qr @ y.T, atol=1e-11)
