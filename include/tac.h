@@ -165,6 +165,46 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
 int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream);
 
 /*
+ * Attention straight from the records (a consumer of the Sec. 3.1
+ * reconstruction; the paper has no counterpart: it evaluates its codes through
+ * a model's attention without a kernel for it).  For each of the job's nq
+ * query rows q_a, over the record slots t = 0 .. tokens-1 of a K and a V cache:
+ *   s_t = scale * (q_a . k^_t),   out_a = sum_t softmax(s)_t v^_t,
+ * where k^_t, v^_t are the rows tac_decode would produce.  Because H and D are
+ * orthogonal, s_t = scale * ((H D_K q_a) . y^K_t) and out_a = D_V H (sum_t p_t y^V_t)
+ * with y^ = r^ (cos, sin)(2 pi k / n): no record is transformed back.
+ * Results agree with decode-then-attend up to fp32 rounding (not bit-exact).
+ */
+#define TAC_MAX_QUERIES 8      /* query rows per job (a GQA group) */
+#define TAC_ATTEND_SPLIT 256   /* tokens per partial result in the workspace */
+
+typedef struct {
+  tac_layer_cfg cfg_k;     /* K codebook and D; cfg_v.d must equal cfg_k.d (64 or 128) */
+  tac_layer_cfg cfg_v;     /* V codebook and D */
+  const void* k_codes;     /* K cache planes (device), capacity slots */
+  const void* k_norms;
+  const void* v_codes;     /* V cache planes (device), capacity slots */
+  const void* v_norms;
+  int64_t capacity;
+  int64_t tokens;          /* 1 <= tokens <= capacity: attend to slots 0..tokens-1 */
+  tac_rows q;              /* nq = q.rows query rows, 1 <= nq <= TAC_MAX_QUERIES (device) */
+  tac_rows out;            /* nq output rows, same dtype as q (device) */
+  float scale;             /* softmax scale, e.g. 1/sqrt(d) */
+} tac_attend_job;
+
+/* Device workspace bytes tac_attend_multi needs for these jobs:
+ * sum over jobs of ceil(tokens / TAC_ATTEND_SPLIT) * nq * (d + 2) floats, each
+ * job's part rounded up to 16 bytes.  Returns -1 for invalid jobs. */
+int64_t tac_attend_workspace_bytes(const tac_attend_job* jobs, int njobs);
+
+/* Attention for every job (jobs of one (d, dtype) share a launch pair).
+ * `workspace` (device, 16-byte aligned, >= tac_attend_workspace_bytes) is the
+ * caller's; its contents need no initialisation and are overwritten.  Calls
+ * that share a workspace must not overlap in time. */
+int tac_attend_multi(const tac_attend_job* jobs, int njobs, void* workspace, int64_t workspace_bytes,
+                     tac_stream_t stream);
+
+/*
  * Transform only, for checking the butterfly: y = H D x (Sec. 2), normalized,
  * written as fp32 rows of d elements (row stride d).  signs: host words as in
  * tac_layer_cfg.signs.  d: any power of two 2..128.

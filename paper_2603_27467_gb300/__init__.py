@@ -24,6 +24,7 @@ __all__ = [
     "make_signs", "layer_cfg", "angle_row_bytes", "norm_row_bytes", "header_offset",
     "codes_bytes", "norms_bytes", "avg_angle_bits", "total_bits", "encode", "decode",
     "encode_multi", "decode_multi", "fwht_debug", "last_error", "version", "Cache",
+    "AttendJob", "attend_multi", "attend_workspace_bytes",
 ]
 
 TAC_OK, TAC_E_INVAL, TAC_E_UNSUPPORTED, TAC_E_CUDA = 0, 1, 2, 3
@@ -64,6 +65,12 @@ class _DecJob(ctypes.Structure):
                 ("capacity", ctypes.c_int64), ("slot", ctypes.c_void_p), ("y", _Rows)]
 
 
+class _AttJob(ctypes.Structure):
+    _fields_ = [("cfg_k", _Cfg), ("cfg_v", _Cfg), ("k_codes", ctypes.c_void_p), ("k_norms", ctypes.c_void_p),
+                ("v_codes", ctypes.c_void_p), ("v_norms", ctypes.c_void_p), ("capacity", ctypes.c_int64),
+                ("tokens", ctypes.c_int64), ("q", _Rows), ("out", _Rows), ("scale", ctypes.c_float)]
+
+
 def library_path() -> str:
     return _LIB_PATH
 
@@ -100,6 +107,10 @@ def load():
         lib.tac_encode_multi.argtypes = [P(_EncJob), i32, vp]
         lib.tac_decode_multi.restype = i32
         lib.tac_decode_multi.argtypes = [P(_DecJob), i32, vp]
+        lib.tac_attend_workspace_bytes.restype = i64
+        lib.tac_attend_workspace_bytes.argtypes = [P(_AttJob), i32]
+        lib.tac_attend_multi.restype = i32
+        lib.tac_attend_multi.argtypes = [P(_AttJob), i32, vp, i64, vp]
         lib.tac_fwht_debug.restype = i32
         lib.tac_fwht_debug.argtypes = [P(_Rows), i32, P(ctypes.c_uint32), vp, vp]
         lib.tac_last_error.restype = ctypes.c_char_p
@@ -335,6 +346,55 @@ def decode_multi(jobs, stream=None) -> None:
         e.slot = j.slot.data_ptr() if j.slot is not None else None
         e.y = _rows(j.y, j.cfg.d)
     _check(load().tac_decode_multi(arr, len(jobs), _stream_ptr(stream)))
+
+
+@dataclass
+class AttendJob:
+    """Attention of q rows over record slots 0..tokens-1 of a K and a V cache."""
+    k_cfg: LayerCfg
+    k_cache: Cache
+    v_cfg: LayerCfg
+    v_cache: Cache
+    tokens: int
+    q: object            # [nq, d] bf16/fp32 device tensor, nq <= 8
+    out: object          # [nq, d] device tensor, dtype of q
+    scale: float
+
+
+def _att_array(jobs):
+    arr = (_AttJob * max(1, len(jobs)))()
+    for i, j in enumerate(jobs):
+        a = arr[i]
+        a.cfg_k, a.cfg_v = j.k_cfg.to_c(), j.v_cfg.to_c()
+        a.k_codes, a.k_norms = j.k_cache.codes.data_ptr(), j.k_cache.norms.data_ptr()
+        a.v_codes, a.v_norms = j.v_cache.codes.data_ptr(), j.v_cache.norms.data_ptr()
+        a.capacity = min(j.k_cache.capacity, j.v_cache.capacity)
+        a.tokens = j.tokens
+        a.q = _rows(j.q, j.k_cfg.d)
+        a.out = _rows(j.out, j.k_cfg.d)
+        a.scale = float(j.scale)
+    return arr
+
+
+def attend_workspace_bytes(jobs) -> int:
+    """tac_attend_workspace_bytes."""
+    n = load().tac_attend_workspace_bytes(_att_array(jobs), len(jobs))
+    if n < 0:
+        raise TacError(TAC_E_INVAL, last_error())
+    return int(n)
+
+
+def attend_multi(jobs, workspace=None, stream=None):
+    """tac_attend_multi; allocates the workspace (torch) when none is given."""
+    torch = _torch()
+    arr = _att_array(jobs)
+    need = attend_workspace_bytes(jobs) if jobs else 0
+    if workspace is None:
+        dev = jobs[0].q.device if jobs else "cuda"
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    _check(load().tac_attend_multi(arr, len(jobs), workspace.data_ptr() if jobs else None,
+                                   workspace.numel() * workspace.element_size(), _stream_ptr(stream)))
+    return workspace
 
 
 def launch_count(jobs) -> int:

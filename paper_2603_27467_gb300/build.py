@@ -26,7 +26,8 @@ CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler",
 
 
 def _units():
-    units = [("tac_api.cu", [], "tac_api"), ("tac_fwht_debug.cu", [], "tac_fwht_debug")]
+    units = [("tac_api.cu", [], "tac_api"), ("tac_fwht_debug.cu", [], "tac_fwht_debug"),
+             ("tac_attend.cu", [], "tac_attend")]
     for kind in ("encode", "decode"):
         for t in ("BF16", "F32"):
             for d in (128, 64, 32, 16):  # biggest first: they dominate the wall time

@@ -68,6 +68,8 @@ static cudaError_t launch_decode(int d, int dtype, int n, int b, int mode, const
   }
   return cudaErrorInvalidValue;
 }
+cudaError_t launch_attend(int d, int dtype, int nq_max, const AttParams& p, int nrows_total, float* ws,
+                          cudaStream_t st);
 cudaError_t launch_fwht_debug(int d, const void* x, int dtype, int64_t rows, int64_t stride,
                               const uint32_t* signs, float* y, cudaStream_t st);
 }  // namespace tac
@@ -416,6 +418,134 @@ int tac_decode(const void* codes, const void* norms, const tac_layer_cfg* cfg, t
   j.slot = nullptr;
   j.y = *y;
   return tac_decode_multi(&j, 1, stream);
+}
+
+// ---------------------------------------------------------------------------
+// Attention from records
+// ---------------------------------------------------------------------------
+namespace {
+
+int check_attend_job(const tac_attend_job& J, int j, const char* who) {
+  int rc = check_cfg(&J.cfg_k, who);
+  if (rc) return rc;
+  rc = check_cfg(&J.cfg_v, who);
+  if (rc) return rc;
+  const int d = J.cfg_k.d;
+  if (J.cfg_v.d != d) return fail(TAC_E_INVAL, "%s: job %d K and V d differ (%d, %d)", who, j, d, J.cfg_v.d);
+  if (d != 64 && d != 128) return fail(TAC_E_UNSUPPORTED, "%s: job %d d = %d (64, 128)", who, j, d);
+  rc = check_rows(&J.q, d, who, "q");
+  if (rc) return rc;
+  rc = check_rows(&J.out, d, who, "out");
+  if (rc) return rc;
+  if (J.q.rows < 1 || J.q.rows > TAC_MAX_QUERIES)
+    return fail(TAC_E_INVAL, "%s: job %d has %lld query rows (1..%d)", who, j, (long long)J.q.rows, TAC_MAX_QUERIES);
+  if (J.out.rows != J.q.rows || J.out.dtype != J.q.dtype)
+    return fail(TAC_E_INVAL, "%s: job %d out must match q in rows and dtype", who, j);
+  if (J.tokens < 1 || J.tokens > J.capacity)
+    return fail(TAC_E_INVAL, "%s: job %d tokens %lld outside 1..capacity %lld", who, j, (long long)J.tokens,
+                (long long)J.capacity);
+  if ((J.tokens + TAC_ATTEND_SPLIT - 1) / TAC_ATTEND_SPLIT > (1 << 26))
+    return fail(TAC_E_UNSUPPORTED, "%s: job %d tokens %lld too many", who, j, (long long)J.tokens);
+  if (!J.k_codes || !J.k_norms || !J.v_codes || !J.v_norms)
+    return fail(TAC_E_INVAL, "%s: job %d record plane is NULL", who, j);
+  if (!aligned16(J.k_codes) || !aligned16(J.k_norms) || !aligned16(J.v_codes) || !aligned16(J.v_norms))
+    return fail(TAC_E_INVAL, "%s: job %d record planes not 16-byte aligned", who, j);
+  if (!(J.scale == J.scale)) return fail(TAC_E_INVAL, "%s: job %d scale is NaN", who, j);
+  return TAC_OK;
+}
+
+int64_t attend_ws_floats(const tac_attend_job& J) {
+  const int64_t splits = (J.tokens + TAC_ATTEND_SPLIT - 1) / TAC_ATTEND_SPLIT;
+  const int64_t f = splits * J.q.rows * tac::att_rec_floats(J.cfg_k.d);
+  return (f + 3) & ~(int64_t)3;  // 16-byte multiple
+}
+
+}  // namespace
+
+int64_t tac_attend_workspace_bytes(const tac_attend_job* jobs, int njobs) {
+  static const char* who = "tac_attend_workspace_bytes";
+  if (njobs < 0 || (njobs > 0 && !jobs)) { fail(TAC_E_INVAL, "%s: bad job array", who); return -1; }
+  int64_t f = 0;
+  for (int j = 0; j < njobs; ++j) {
+    if (check_attend_job(jobs[j], j, who)) return -1;
+    f += attend_ws_floats(jobs[j]);
+  }
+  ok();
+  return 4 * f;
+}
+
+int tac_attend_multi(const tac_attend_job* jobs, int njobs, void* workspace, int64_t workspace_bytes,
+                     tac_stream_t stream) {
+  static const char* who = "tac_attend_multi";
+  if (njobs < 0) return fail(TAC_E_INVAL, "%s: njobs = %d", who, njobs);
+  if (njobs > 0 && !jobs) return fail(TAC_E_INVAL, "%s: jobs is NULL", who);
+  int64_t need = 0;
+  for (int j = 0; j < njobs; ++j) {
+    const int rc = check_attend_job(jobs[j], j, who);
+    if (rc) return rc;
+    need += 4 * attend_ws_floats(jobs[j]);
+  }
+  if (njobs == 0) return ok();
+  if (!workspace || !aligned16(workspace) || workspace_bytes < need)
+    return fail(TAC_E_INVAL, "%s: workspace NULL, misaligned or smaller than %lld bytes", who, (long long)need);
+  if (num_sms() <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
+  // Group by (d, dtype); each job's workspace part follows the previous job's.
+  std::vector<int> order(njobs);
+  for (int j = 0; j < njobs; ++j) order[j] = j;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) {
+    return jobs[a].cfg_k.d * 4 + jobs[a].q.dtype < jobs[b].cfg_k.d * 4 + jobs[b].q.dtype;
+  });
+  static thread_local tac::AttParams P;
+  float* ws = static_cast<float*>(workspace);
+  int64_t ws_off = 0;
+  size_t i = 0;
+  while (i < order.size()) {
+    const int d = jobs[order[i]].cfg_k.d, dt = jobs[order[i]].q.dtype;
+    std::memset(&P, 0, sizeof(P));
+    int64_t ctas = 0, splits = 0;
+    int nrows = 0, nq_max = 1;
+    while (i < order.size() && P.njobs < TAC_MAX_JOBS && jobs[order[i]].cfg_k.d == d &&
+           jobs[order[i]].q.dtype == dt) {
+      const tac_attend_job& J = jobs[order[i]];
+      const int64_t ns = (J.tokens + TAC_ATTEND_SPLIT - 1) / TAC_ATTEND_SPLIT;
+      const int64_t nc = (ns + 3) / 4;
+      if (ctas + nc > 0x7fffffff || splits + ns > 0x7fffffff) break;
+      tac::AttJob& A = P.job[P.njobs];
+      A.kc = static_cast<const uint8_t*>(J.k_codes);
+      A.kn = static_cast<const uint8_t*>(J.k_norms);
+      A.kh = A.kn + header_offset(&J.cfg_k, J.capacity);
+      A.vc = static_cast<const uint8_t*>(J.v_codes);
+      A.vn = static_cast<const uint8_t*>(J.v_norms);
+      A.vh = A.vn + header_offset(&J.cfg_v, J.capacity);
+      A.q = J.q.data;
+      A.out = J.out.data;
+      A.q_stride = J.q.row_stride;
+      A.out_stride = J.out.row_stride;
+      A.tokens = J.tokens;
+      A.scale = J.scale;
+      A.nq = (int32_t)J.q.rows;
+      A.nk = J.cfg_k.n_angle; A.wk = tac::code_bits(J.cfg_k.n_angle); A.bk = J.cfg_k.norm_bits; A.mk = J.cfg_k.norm_mode;
+      A.nv = J.cfg_v.n_angle; A.wv = tac::code_bits(J.cfg_v.n_angle); A.bv = J.cfg_v.norm_bits; A.mv = J.cfg_v.norm_mode;
+      copy_signs(A.sk, &J.cfg_k);
+      copy_signs(A.sv, &J.cfg_v);
+      A.split0 = (int32_t)splits;
+      A.cta0 = (int32_t)ctas;
+      A.ws = ws_off;
+      ws_off += attend_ws_floats(J);
+      splits += ns;
+      ctas += nc;
+      nrows += A.nq;
+      nq_max = std::max(nq_max, (int)A.nq);
+      ++P.njobs;
+      ++i;
+    }
+    if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many tokens", who);
+    P.nctas = (int32_t)ctas;
+    P.nsplits = (int32_t)splits;
+    cudaError_t e = tac::launch_attend(d, dt, nq_max, P, nrows, ws, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+  }
+  return ok();
 }
 
 int tac_fwht_debug(const tac_rows* x, int d, const uint32_t* signs, float* y, tac_stream_t stream) {

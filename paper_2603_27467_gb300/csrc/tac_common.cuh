@@ -131,6 +131,33 @@ struct DecParams {
   DecJob job[TAC_MAX_JOBS];
 };
 
+// Attention jobs (tac_attend_multi): record planes, runtime codebooks, queries.
+struct AttJob {
+  const uint8_t* kc; const uint8_t* kn; const uint8_t* kh;   // K planes (angle, norm, header)
+  const uint8_t* vc; const uint8_t* vn; const uint8_t* vh;   // V planes
+  const void* q; void* out;
+  int64_t q_stride, out_stride;      // elements
+  int64_t tokens;
+  float scale;
+  int32_t nq;
+  int32_t nk, wk, bk, mk;            // K: bins, code bits, norm bits, norm mode
+  int32_t nv, wv, bv, mv;            // V
+  uint32_t sk[4], sv[4];             // D of K and of V
+  int32_t split0;                    // first global split of this job
+  int32_t cta0;                      // first CTA of this job
+  int64_t ws;                        // first workspace float of this job
+};
+
+struct AttParams {
+  int32_t njobs;
+  int32_t nctas;
+  int32_t nsplits;
+  AttJob job[TAC_MAX_JOBS];
+};
+
+// Per-split workspace record: max (log2 units), sum, accumulator (d floats).
+__host__ __device__ constexpr int att_rec_floats(int d) { return d + 2; }
+
 // Job owning global tile t (jobs are sorted by tile0, job 0 starts at tile 0).
 template <typename Params>
 __device__ __forceinline__ int find_job(const Params& p, int t) {

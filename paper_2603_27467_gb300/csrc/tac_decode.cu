@@ -304,32 +304,59 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
 #pragma unroll
   for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
 
+  static_assert((kNS & (kNS - 1)) == 0, "stage ring size");
   int stage = 0;
+  // Iterations ahead that need no checks: the decoded tile is a full tile of
+  // the current job and the prefetched tile a full tile of the (contiguous)
+  // issue job inside the warp's range.  Set by the general iterations.
+  int fast = 0;
   for (; t < t_end; ++t) {
     cp_async_wait<kNS - 2>();   // this warp tile's records have landed
     __syncwarp();               // ... and every lane is done with the previous tile
-    {
-      int ns = stage + kNS - 1;
-      if (ns >= kNS) ns -= kNS;
-      issue(ns);
-    }
-    if (t >= c_end) {  // next job
-      const int cj = find_job(p, t);
-      const DecJob& J = p.job[cj];
-      c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
-      const int64_t row0 = (int64_t)(t - J.tile0) * C::RW;
-      c_left = J.rows - row0;
-      const int64_t sb = J.stride * C::ESZ;
-      c_step = C::RW * sb;
-      o_row = reinterpret_cast<uint8_t*>(J.y) + (row0 + r) * sb + 2 * C::ESZ * l;
+    const int ns = (stage + kNS - 1) & (kNS - 1);
+    const bool fast_tile = fast > 0;
+    if (fast_tile) {
+      --fast;
+      uint8_t* dst = wsm + C::W_REC + ns * C::REC_W;
 #pragma unroll
-      for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
+      for (int q = 0; q < C::ROUNDS; ++q) {
+        const int ch = q * 32 + lane;
+        if (ch < C::NCH) cp_async16(dst + 16 * ch, i_src[q], 16);
+        i_src[q] += i_step[q];
+      }
+      cp_async_commit();
+      i_row0 += C::RW;
+      i_left -= C::RW;
+      ++it;
+    } else {
+      issue(ns);
+      if (t >= c_end) {  // next job
+        const int cj = find_job(p, t);
+        const DecJob& J = p.job[cj];
+        c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
+        const int64_t row0 = (int64_t)(t - J.tile0) * C::RW;
+        c_left = J.rows - row0;
+        const int64_t sb = J.stride * C::ESZ;
+        c_step = C::RW * sb;
+        o_row = reinterpret_cast<uint8_t*>(J.y) + (row0 + r) * sb + 2 * C::ESZ * l;
+#pragma unroll
+        for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
+      }
     }
     const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;
-    decode_body<D, TOut, N, B, MODE>(rec, wsm, ttab + (lane % C::TABR), lane, msk, o_row, r < c_left);
+    decode_body<D, TOut, N, B, MODE>(rec, wsm, ttab + (lane % C::TABR), lane, msk, o_row,
+                                     fast_tile || r < c_left);
     o_row += c_step;
     c_left -= C::RW;
-    stage = (stage + 1 == kNS) ? 0 : stage + 1;
+    stage = (stage + 1) & (kNS - 1);
+    if (!fast_tile) {
+      // c_left now counts the rows of the compute job from tile t + 1, i_left
+      // those of the issue job from tile it (the next to prefetch).
+      const int64_t cf = c_left / C::RW;
+      const int64_t pf = p_dense ? min(min((int64_t)(p_end - it), i_left / C::RW), (int64_t)(t_end - it)) : 0;
+      const int64_t f = min(cf, pf);
+      fast = f > 0 ? (int)f : 0;
+    }
   }
   cp_async_wait<0>();
 }

@@ -575,46 +575,60 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
 #pragma unroll
   for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
 
+  static_assert((kNS & (kNS - 1)) == 0, "stage ring size");
   int stage = 0;
+  // Iterations ahead that need no checks: the computed tile is a full tile of
+  // the current (dense) job and the prefetched tile a full tile of the issue
+  // job inside the warp's range.  Set by the general iterations.
+  int fast = 0;
   for (; t < t_end; ++t) {
     cp_async_wait<kNS - 2>();   // this warp tile has landed
     __syncwarp();               // ... and every lane is done with the previous one
-    {
-      int ns = stage + kNS - 1;
-      if (ns >= kNS) ns -= kNS;
+    const int ns = (stage + kNS - 1) & (kNS - 1);
+    const bool fast_tile = fast > 0;
+    if (fast_tile) {
+      --fast;
+      uint8_t* dst = in_dst + ns * IT::BYTES;
+#pragma unroll
+      for (int q = 0; q < C::CHUNKS; ++q) cp_async16(dst + q * C::RPQ * IT::STRIDE, i_src + q * i_qstep, 16);
+      cp_async_commit();
+      i_src += i_step;
+      i_left -= C::RW;
+      ++it;
+    } else {
       issue(ns);
-    }
-    if (t >= c_end) {  // next job
-      const int cj = find_job(p, t);
-      const EncJob& J = p.job[cj];
-      c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
-      const int rel = t - J.tile0;
-      c_row0 = (int64_t)rel * C::RW;
-      c_left = J.rows - c_row0;
-      c_dense = J.slot == nullptr;
+      if (t >= c_end) {  // next job
+        const int cj = find_job(p, t);
+        const EncJob& J = p.job[cj];
+        c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
+        const int rel = t - J.tile0;
+        c_row0 = (int64_t)rel * C::RW;
+        c_left = J.rows - c_row0;
+        c_dense = J.slot == nullptr;
 #pragma unroll
-      for (int q = 0; q < C::ROUNDS; ++q) {
-        const int ch = q * 32 + lane;
-        if (ch < C::NA) { o_dst[q] = J.codes + 16 * ch; o_step[q] = C::RW * C::AB; }
-        else if (ch < C::NA + C::NN) { o_dst[q] = J.norms + 16 * (ch - C::NA); o_step[q] = C::RW * C::NB; }
-        else { o_dst[q] = J.hdr + 16 * (ch - C::NA - C::NN); o_step[q] = C::RW * C::HB; }
-        o_dst[q] += (int64_t)rel * o_step[q];
+        for (int q = 0; q < C::ROUNDS; ++q) {
+          const int ch = q * 32 + lane;
+          if (ch < C::NA) { o_dst[q] = J.codes + 16 * ch; o_step[q] = C::RW * C::AB; }
+          else if (ch < C::NA + C::NN) { o_dst[q] = J.norms + 16 * (ch - C::NA); o_step[q] = C::RW * C::NB; }
+          else { o_dst[q] = J.hdr + 16 * (ch - C::NA - C::NN); o_step[q] = C::RW * C::HB; }
+          o_dst[q] += (int64_t)rel * o_step[q];
+        }
+        if (lane == 0) {
+          wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot; wj->capacity = J.capacity;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) wj->signs[q] = J.signs[q];
+        }
+        const int l = lane % C::L;
+#pragma unroll
+        for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
+        __syncwarp();
       }
-      if (lane == 0) {
-        wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot; wj->capacity = J.capacity;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) wj->signs[q] = J.signs[q];
-      }
-      const int l = lane % C::L;
-#pragma unroll
-      for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
-      __syncwarp();
     }
-    const int nrows = c_left < C::RW ? (int)c_left : C::RW;
+    const int nrows = (fast_tile || c_left >= C::RW) ? C::RW : (int)c_left;
     const uint8_t* in = wsm + C::W_IN + stage * IT::BYTES;
     tile_body<D, TIn, N, B, MODE>(in, wsm, etab + (lane % C::TABR), nrows, lane, msk, wj->signs);
     __syncwarp();
-    if (c_dense && nrows == C::RW) {
+    if (fast_tile || (c_dense && nrows == C::RW)) {
 #pragma unroll
       for (int q = 0; q < C::ROUNDS; ++q) {
         const int ch = q * 32 + lane;
@@ -628,7 +642,15 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
     for (int q = 0; q < C::ROUNDS; ++q) o_dst[q] += o_step[q];
     c_row0 += C::RW;
     c_left -= C::RW;
-    stage = (stage + 1 == kNS) ? 0 : stage + 1;
+    stage = (stage + 1) & (kNS - 1);
+    if (!fast_tile) {
+      // c_left now counts the rows of the compute job from tile t + 1, i_left
+      // those of the issue job from tile it (the next to prefetch).
+      const int64_t cf = c_dense ? c_left / C::RW : 0;
+      const int64_t pf = min(min((int64_t)(p_end - it), i_left / C::RW), (int64_t)(t_end - it));
+      const int64_t f = min(cf, pf);
+      fast = f > 0 ? (int)f : 0;
+    }
   }
   cp_async_wait<0>();
 }

@@ -175,3 +175,40 @@ def test_empty_calls_succeed_without_device(tac_host):
     assert lib.tac_decode(None, None, ctypes.byref(c), ctypes.byref(rows), None) == tac_host.TAC_OK
     assert lib.tac_encode_multi(None, 0, None) == tac_host.TAC_OK
     assert lib.tac_decode_multi(None, 0, None) == tac_host.TAC_OK
+
+
+def test_attend_validation_and_workspace_size(tac_host):
+    """tac_attend_*: argument checks happen before any device work; the
+    workspace holds ceil(tokens/256) * nq * (d + 2) floats per job, each job's
+    part rounded up to 16 bytes."""
+    lib = tac_host.load()
+
+    def job(d=128, nq=4, tokens=1000, capacity=1000, kn=64, vn=56, vb=4, vmode=1, qdt=0, odt=0, orows=None):
+        j = tac_host._AttJob()
+        j.cfg_k = tac_host.LayerCfg(d, kn, 8, 0).to_c()
+        j.cfg_v = tac_host.LayerCfg(d, vn, vb, vmode).to_c()
+        j.k_codes = j.k_norms = j.v_codes = j.v_norms = 4096
+        j.capacity, j.tokens = capacity, tokens
+        j.q.data, j.q.dtype, j.q.rows, j.q.row_stride = 8192, qdt, nq, d
+        j.out.data, j.out.dtype, j.out.rows, j.out.row_stride = 16384, odt, nq if orows is None else orows, d
+        j.scale = 0.088
+        return j
+
+    arr = (tac_host._AttJob * 2)(job(), job(d=64, nq=1, tokens=257, capacity=300, vn=256, vb=32, vmode=2))
+    want = (math.ceil(1000 / 256) * 4 * 130 + 3) // 4 * 4 * 4 + (2 * 1 * 66 + 3) // 4 * 4 * 4
+    assert lib.tac_attend_workspace_bytes(arr, 2) == want
+    bad = [dict(nq=0), dict(nq=9), dict(tokens=0), dict(tokens=1001), dict(orows=3), dict(odt=1),
+           dict(d=32)]
+    for kw in bad:
+        a = (tac_host._AttJob * 1)(job(**kw))
+        rc = lib.tac_attend_multi(a, 1, 4096, 1 << 30, None)
+        assert rc in (tac_host.TAC_E_INVAL, tac_host.TAC_E_UNSUPPORTED), kw
+        assert lib.tac_attend_workspace_bytes(a, 1) == -1, kw
+    a = (tac_host._AttJob * 1)(job())
+    j0 = a[0]
+    j0.cfg_v.d = 64
+    assert lib.tac_attend_multi(a, 1, 4096, 1 << 30, None) == tac_host.TAC_E_INVAL   # K and V d differ
+    a = (tac_host._AttJob * 1)(job())
+    assert lib.tac_attend_multi(a, 1, 4096, 16, None) == tac_host.TAC_E_INVAL        # workspace too small
+    assert lib.tac_attend_multi(a, 1, 4100, 1 << 30, None) == tac_host.TAC_E_INVAL   # misaligned workspace
+    assert lib.tac_attend_multi(None, 0, None, 0, None) == tac_host.TAC_OK
