@@ -69,7 +69,7 @@ def parse_args():
     ap.add_argument("--impl", choices=["tac", "reference"], default="tac")
     ap.add_argument("--config", default="mistral7b",
                     choices=["mistral7b", "llama1b", "append", "longctx", "mistral7b_angle", "mistral7b_norm8",
-                             "tinyllama_n56"])
+                             "tinyllama_n56", "attend"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
@@ -286,6 +286,10 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
+    if args.config == "attend":
+        print(json.dumps({"impl": "reference", "unavailable": "the reference arm times the oracle's encode/decode "
+                          "workloads; attention from records has no oracle timing mode"}), flush=True)
+        return
     import oracle
     oracle.build()
     threads = os.cpu_count() or 1
@@ -398,6 +402,77 @@ def run_e2e(tac, ws, world, dev, steps, chunk_blocks, step_bytes, barrier):
     return out
 
 
+def run_attend(args):
+    """Attention straight from records (tac_attend_multi) on the Mistral-7B-shaped
+    cache: one job per (layer, KV head) over all its tokens, 4 query rows per KV
+    head (GQA 4:1), bf16 queries and outputs.  value = record bytes read per
+    step (K and V records of every token) / step time."""
+    import torch
+    from paper_2603_27467_gb300 import build as tb
+    tb.build()
+    import paper_2603_27467_gb300 as tac
+    tac.load()
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    w = workloads.CONFIGS["mistral7b"]
+    T = args.tokens or w.tokens
+    nq = 4
+    jobs, rec_bytes, keep = [], 0, []
+    for l in range(w.layers):
+        caches = {}
+        for kv in (workloads.K, workloads.V):
+            d, n, b, mode = w.codebook(l, kv)
+            cfg = tac.layer_cfg(d, n, b, mode, 0, l, kv)
+            x = workloads.block(w, l, kv, tokens=T, device=dev, dtype=torch.bfloat16)
+            per_head = []
+            for h in range(w.heads):
+                c = tac.Cache.empty(cfg, T, device=dev)
+                tac.encode(x[h * T:(h + 1) * T], cfg, cache=c)
+                per_head.append(c)
+            caches[kv] = (cfg, per_head, record_bytes(d, n, b, mode))
+            del x
+        kcfg, kc, kb = caches[workloads.K]
+        vcfg, vc, vb = caches[workloads.V]
+        for h in range(w.heads):
+            g = torch.Generator(device=dev)
+            g.manual_seed(l * 64 + h)
+            q = torch.randn((nq, w.d), generator=g, device=dev).to(torch.bfloat16)
+            out = torch.empty_like(q)
+            jobs.append(tac.AttendJob(kcfg, kc[h], vcfg, vc[h], T, q, out, 1.0 / w.d ** 0.5))
+            rec_bytes += T * (kb + vb)
+        keep.append(caches)
+    ws = torch.empty(tac.attend_workspace_bytes(jobs), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+    for _ in range(args.warmup):
+        tac.attend_multi(jobs, ws, stream=stream)
+    torch.cuda.synchronize()
+    clk = ClockSampler(None)
+    clk.start()
+    time.sleep(0.3)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        tac.attend_multi(jobs, ws, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = clk.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    hbm, peak_kind = peaks()
+    gbs = rec_bytes / (ms / 1e3) / 1e9
+    print(json.dumps({
+        "metric": "attention from records GB/s (K+V records read) on 1 GB300", "value": gbs, "unit": "GB/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": f"mistral7b-shaped cache, {w.layers} L x {w.heads} KV heads x {T} tokens, "
+                               f"{nq} query rows per KV head (GQA 4:1), bf16 q/out, one job per (layer, head)",
+                   "record_bytes_per_step": rec_bytes},
+        "token_heads_per_s": w.layers * w.heads * T / (ms / 1e3),
+        "roofline": {"bound": "hbm", "kernel": "attend_partial + attend_combine", "achieved": gbs, "peak": hbm,
+                     "unit": "GB/s", "frac": gbs / hbm, "peak_source": f"{peak_kind} hbm_gbs", "traffic": None},
+        "gpu_launches": 2 * args.steps * (1 + (len(jobs) - 1) // 96), "clocks": clocks}), flush=True)
+
+
 def probe_rd(args):
     """Rate-distortion probe: relative reconstruction MSE (sum |x^ - x|^2 / sum |x|^2)
     of GPU encode -> decode with fp32 norms (angle-only) for every supported n,
@@ -437,6 +512,9 @@ def main():
     args = parse_args()
     if args.probe == "rd":
         probe_rd(args)
+        return
+    if args.config == "attend" and args.impl != "reference":
+        run_attend(args)
         return
     if args.impl == "reference":
         run_reference(args)

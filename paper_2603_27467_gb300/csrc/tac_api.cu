@@ -526,6 +526,8 @@ int tac_attend_multi(const tac_attend_job* jobs, int njobs, void* workspace, int
       A.nq = (int32_t)J.q.rows;
       A.nk = J.cfg_k.n_angle; A.wk = tac::code_bits(J.cfg_k.n_angle); A.bk = J.cfg_k.norm_bits; A.mk = J.cfg_k.norm_mode;
       A.nv = J.cfg_v.n_angle; A.wv = tac::code_bits(J.cfg_v.n_angle); A.bv = J.cfg_v.norm_bits; A.mv = J.cfg_v.norm_mode;
+      A.inv_lk = A.mk == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bk) - 1);
+      A.inv_lv = A.mv == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bv) - 1);
       copy_signs(A.sk, &J.cfg_k);
       copy_signs(A.sv, &J.cfg_v);
       A.split0 = (int32_t)splits;

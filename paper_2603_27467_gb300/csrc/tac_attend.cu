@@ -70,25 +70,14 @@ __device__ __forceinline__ uint64_t load_u64_any(const uint8_t* p) {
   return v;
 }
 
-// `bits` bits at bit offset `bit` of a record row starting on a 4-byte boundary.
-__device__ __forceinline__ uint32_t load_bits(const uint8_t* row, int bit, int bits) {
-  const uint32_t* w = reinterpret_cast<const uint32_t*>(row) + (bit >> 5);
-  const int sh = bit & 31;
-  uint32_t v = w[0] >> sh;
-  if (sh + bits > 32) v |= w[1] << (32 - sh);
-  return v & ((1u << bits) - 1u);
-}
-
 // Dequantization constants of one record (the inverse of Eq. 2): r^ = base + c step
-// (linear) or 2^(base + c step) (log); fp32 norms need none.
-__device__ __forceinline__ float2 norm_consts(const uint8_t* hdr, int bits, int mode) {
-  if (mode == TAC_NORM_FP32) return make_float2(0.f, 0.f);
+// (linear) or 2^(base + c step) (log); inv_l = 1 / (2^b - 1).
+__device__ __forceinline__ float2 norm_consts(const uint8_t* hdr, float inv_l, int mode) {
   const float2 h = *reinterpret_cast<const float2*>(hdr);
-  const float Lq = (float)((1 << bits) - 1);
   const bool spread = h.y > h.x;
-  if (mode == TAC_NORM_LINEAR) return make_float2(h.x, spread ? (h.y - h.x) / Lq : 0.f);
+  if (mode == TAC_NORM_LINEAR) return make_float2(h.x, spread ? (h.y - h.x) * inv_l : 0.f);
   const float lmin = lg2_approx(h.x);
-  return make_float2(lmin, spread ? (lg2_approx(h.y) - lmin) / Lq : 0.f);
+  return make_float2(lmin, spread ? (lg2_approx(h.y) - lmin) * inv_l : 0.f);
 }
 
 __device__ __forceinline__ float dequant(uint32_t c, float2 bs, int mode) {
@@ -199,6 +188,16 @@ __global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_const
   for (int s = 0; s < kAttNS - 1; ++s) issue(s);
 
   const int r = lane / L, l = lane % L;     // K layout: token r of the step, pairs 8l..8l+7
+  // V layout: lane owns pairs lane + 32 j; their code positions are fixed per job
+  int va_w[PV], va_s[PV], vn_w[PV], vn_s[PV];
+#pragma unroll
+  for (int j = 0; j < PV; ++j) {
+    const int i = lane + 32 * j, ba = i * J.wv, bn = i * J.bv;
+    va_w[j] = ba >> 5; va_s[j] = ba & 31;
+    vn_w[j] = bn >> 5; vn_s[j] = bn & 31;
+  }
+  const uint32_t vmask = (1u << J.wv) - 1u;
+  const uint32_t nvmask = J.bv >= 32 ? 0xffffffffu : (1u << J.bv) - 1u;
   float m_run[NQ], l_run[NQ];
   float acc[NQ][PV][2];
 #pragma unroll
@@ -215,6 +214,9 @@ __global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_const
     issue(s + kAttNS - 1);
     const uint8_t* st = wsm + (s % kAttNS) * C::STAGE;
     const int64_t row0 = t_begin + (int64_t)s * RW;
+    const int valid = (int)min((int64_t)RW, t_stop - row0);   // tokens of this step
+    // dequantization constants of the V record of token r (broadcast in the V phase)
+    const float2 vbs = hv ? norm_consts(st + C::S_VH + r * 8, J.inv_lv, J.mv) : make_float2(0.f, 0.f);
 
     // ---- K: partial scores of token r over pairs 8l..8l+7 ----
     float sc[NQ];
@@ -223,7 +225,7 @@ __global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_const
     {
       const uint64_t ka = load_u64_any(st + C::S_KA + r * ak + l * J.wk);
       const uint32_t kmask = (1u << J.wk) - 1u;
-      const float2 bs = hk ? norm_consts(st + C::S_KH + r * 8, J.bk, J.mk) : make_float2(0.f, 0.f);
+      const float2 bs = hk ? norm_consts(st + C::S_KH + r * 8, J.inv_lk, J.mk) : make_float2(0.f, 0.f);
       const uint8_t* nrow = st + C::S_KN + r * nbk;
       uint64_t kn = 0;
       if (J.mk != TAC_NORM_FP32)
@@ -264,7 +266,7 @@ __global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_const
 #pragma unroll
         for (int rr = 0; rr < RW; ++rr) {
           float v = __shfl_sync(0xffffffffu, sc[a], rr * L);
-          if (row0 + rr >= t_stop) v = -INFINITY;
+          if (rr >= valid) v = -INFINITY;
           pw[a][rr] = v;
           mx = fmaxf(mx, v);
         }
@@ -285,19 +287,19 @@ __global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_const
     // ---- V: accumulate p_t y^V_t, lane l owning pairs l + 32 j ----
 #pragma unroll
     for (int rr = 0; rr < RW; ++rr) {
-      if (row0 + rr >= t_stop) break;
-      const uint8_t* arow = st + C::S_VA + rr * av;
-      const uint8_t* nrow = st + C::S_VN + rr * nbv;
-      const float2 bs = hv ? norm_consts(st + C::S_VH + rr * 8, J.bv, J.mv) : make_float2(0.f, 0.f);
+      if (rr >= valid) break;
+      const uint32_t* arow = reinterpret_cast<const uint32_t*>(st + C::S_VA + rr * av);
+      const uint32_t* nrow = reinterpret_cast<const uint32_t*>(st + C::S_VN + rr * nbv);
+      const float2 bs = make_float2(__shfl_sync(0xffffffffu, vbs.x, rr * L), __shfl_sync(0xffffffffu, vbs.y, rr * L));
 #pragma unroll
       for (int j = 0; j < PV; ++j) {
         const int i = lane + 32 * j;
         if (i < P) {
-          uint32_t k = load_bits(arow, i * J.wv, J.wv);
+          uint32_t k = __funnelshift_r(arow[va_w[j]], arow[va_w[j] + 1], va_s[j]) & vmask;
           k = min(k, (uint32_t)(J.nv - 1));
           float rh;
-          if (J.mv == TAC_NORM_FP32) rh = reinterpret_cast<const float*>(nrow)[i];
-          else rh = dequant(load_bits(nrow, i * J.bv, J.bv), bs, J.mv);
+          if (J.mv == TAC_NORM_FP32) rh = __uint_as_float(nrow[i]);
+          else rh = dequant((nrow[vn_w[j]] >> vn_s[j]) & nvmask, bs, J.mv);
           const float2 cs = tv[k];
           const float yc = rh * cs.x, ys = rh * cs.y;
 #pragma unroll

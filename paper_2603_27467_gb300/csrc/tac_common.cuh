@@ -142,6 +142,7 @@ struct AttJob {
   int32_t nq;
   int32_t nk, wk, bk, mk;            // K: bins, code bits, norm bits, norm mode
   int32_t nv, wv, bv, mv;            // V
+  float inv_lk, inv_lv;              // 1 / (2^b - 1) of K and V norms (0 for fp32 norms)
   uint32_t sk[4], sv[4];             // D of K and of V
   int32_t split0;                    // first global split of this job
   int32_t cta0;                      // first CTA of this job
