@@ -205,6 +205,34 @@ int tac_attend_multi(const tac_attend_job* jobs, int njobs, void* workspace, int
                      tac_stream_t stream);
 
 /*
+ * tac_attend_multi without a caller workspace, for callers that cannot
+ * allocate device memory (the paper has no counterpart: this is an interface
+ * convenience of this library).  The partial results live in one static
+ * device array of TAC_ATTEND_STATIC_WS_BYTES per device, built into the
+ * library; nothing is allocated, on the device or the host heap.
+ *
+ *   - Same jobs, results and errors as tac_attend_multi with a workspace.
+ *   - Jobs whose tac_attend_workspace_bytes exceeds TAC_ATTEND_STATIC_WS_BYTES
+ *     are rejected with TAC_E_UNSUPPORTED (nothing launched); split them over
+ *     several calls, or pass a workspace to tac_attend_multi.
+ *   - Nothing in the array needs to start at zero: every partial record is
+ *     written by the first kernel before the second reads it.
+ *   - First call on each device: resolves the array's address with
+ *     cudaGetSymbolAddress, which may load the library's attention module.
+ *     Make that first call outside stream capture; a call with njobs = 0 does
+ *     only this setup and returns TAC_E_CUDA if it fails.  The first launch
+ *     of each kernel shape (d, q dtype, query count) on a device also sets its
+ *     shared-memory limit, as in tac_attend_multi.  After both, a call makes
+ *     no CUDA runtime call but cudaGetDevice, the launches and
+ *     cudaGetLastError, and can be captured into a CUDA graph.
+ *   - All calls on one device share the array: two calls that overlap in time
+ *     (different streams, or host threads without ordering) race on it and
+ *     give undefined results.  Calls in one stream are ordered and safe.
+ */
+#define TAC_ATTEND_STATIC_WS_BYTES (8 << 20)
+int tac_attend_multi_static(const tac_attend_job* jobs, int njobs, tac_stream_t stream);
+
+/*
  * Transform only, for checking the butterfly: y = H D x (Sec. 2), normalized,
  * written as fp32 rows of d elements (row stride d).  signs: host words as in
  * tac_layer_cfg.signs.  d: any power of two 2..128.

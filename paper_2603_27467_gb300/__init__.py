@@ -32,6 +32,7 @@ NORM_LINEAR, NORM_LOG, NORM_FP32 = 0, 1, 2
 BF16, FP32 = 0, 1
 MAX_D = 128
 MAX_JOBS = 96  # TAC_MAX_JOBS: jobs per kernel launch
+ATTEND_STATIC_WS_BYTES = 8 << 20  # TAC_ATTEND_STATIC_WS_BYTES: static attention workspace per device
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "_build", "libtac.so")
@@ -111,6 +112,8 @@ def load():
         lib.tac_attend_workspace_bytes.argtypes = [P(_AttJob), i32]
         lib.tac_attend_multi.restype = i32
         lib.tac_attend_multi.argtypes = [P(_AttJob), i32, vp, i64, vp]
+        lib.tac_attend_multi_static.restype = i32
+        lib.tac_attend_multi_static.argtypes = [P(_AttJob), i32, vp]
         lib.tac_fwht_debug.restype = i32
         lib.tac_fwht_debug.argtypes = [P(_Rows), i32, P(ctypes.c_uint32), vp, vp]
         lib.tac_last_error.restype = ctypes.c_char_p
@@ -395,6 +398,13 @@ def attend_multi(jobs, workspace=None, stream=None):
     _check(load().tac_attend_multi(arr, len(jobs), workspace.data_ptr() if jobs else None,
                                    workspace.numel() * workspace.element_size(), _stream_ptr(stream)))
     return workspace
+
+
+def attend_multi_static(jobs, stream=None):
+    """tac_attend_multi_static: the library's static device workspace
+    (ATTEND_STATIC_WS_BYTES per device), nothing allocated.  An empty job
+    list only resolves the workspace address on the current device."""
+    _check(load().tac_attend_multi_static(_att_array(jobs), len(jobs), _stream_ptr(stream)))
 
 
 def launch_count(jobs) -> int:

@@ -70,6 +70,7 @@ static cudaError_t launch_decode(int d, int dtype, int n, int b, int mode, const
 }
 cudaError_t launch_attend(int d, int dtype, int nq_max, const AttParams& p, int nrows_total, float* ws,
                           cudaStream_t st);
+cudaError_t attend_static_workspace(float** ws);
 cudaError_t launch_fwht_debug(int d, const void* x, int dtype, int64_t rows, int64_t stride,
                               const uint32_t* signs, float* y, cudaStream_t st);
 }  // namespace tac
@@ -474,80 +475,119 @@ int64_t tac_attend_workspace_bytes(const tac_attend_job* jobs, int njobs) {
   return 4 * f;
 }
 
-int tac_attend_multi(const tac_attend_job* jobs, int njobs, void* workspace, int64_t workspace_bytes,
-                     tac_stream_t stream) {
-  static const char* who = "tac_attend_multi";
+namespace {
+
+// Validates the jobs; *need = the workspace bytes they take.
+int check_attend_jobs(const tac_attend_job* jobs, int njobs, int64_t* need, const char* who) {
   if (njobs < 0) return fail(TAC_E_INVAL, "%s: njobs = %d", who, njobs);
   if (njobs > 0 && !jobs) return fail(TAC_E_INVAL, "%s: jobs is NULL", who);
-  int64_t need = 0;
+  *need = 0;
   for (int j = 0; j < njobs; ++j) {
     const int rc = check_attend_job(jobs[j], j, who);
     if (rc) return rc;
-    need += 4 * attend_ws_floats(jobs[j]);
+    *need += 4 * attend_ws_floats(jobs[j]);
   }
+  return TAC_OK;
+}
+
+// Launches checked jobs, grouped by (d, dtype) in job order, up to
+// TAC_MAX_JOBS per launch pair; each job's workspace part follows the
+// previous one's.  Allocates nothing.
+int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st, const char* who) {
+  static thread_local tac::AttParams P;
+  static const int kD[2] = {64, 128};
+  static const int kDt[2] = {TAC_BF16, TAC_FP32};
+  int64_t ws_off = 0;
+  for (int d : kD) {
+    for (int dt : kDt) {
+      int i = 0;
+      auto next = [&](int from) {
+        while (from < njobs && !(jobs[from].cfg_k.d == d && jobs[from].q.dtype == dt)) ++from;
+        return from;
+      };
+      i = next(0);
+      while (i < njobs) {
+        std::memset(&P, 0, sizeof(P));
+        int64_t ctas = 0, splits = 0;
+        int nrows = 0, nq_max = 1;
+        while (i < njobs && P.njobs < TAC_MAX_JOBS) {
+          const tac_attend_job& J = jobs[i];
+          const int64_t ns = (J.tokens + TAC_ATTEND_SPLIT - 1) / TAC_ATTEND_SPLIT;
+          const int64_t nc = (ns + 3) / 4;
+          if (ctas + nc > 0x7fffffff || splits + ns > 0x7fffffff) break;
+          tac::AttJob& A = P.job[P.njobs];
+          A.kc = static_cast<const uint8_t*>(J.k_codes);
+          A.kn = static_cast<const uint8_t*>(J.k_norms);
+          A.kh = A.kn + header_offset(&J.cfg_k, J.capacity);
+          A.vc = static_cast<const uint8_t*>(J.v_codes);
+          A.vn = static_cast<const uint8_t*>(J.v_norms);
+          A.vh = A.vn + header_offset(&J.cfg_v, J.capacity);
+          A.q = J.q.data;
+          A.out = J.out.data;
+          A.q_stride = J.q.row_stride;
+          A.out_stride = J.out.row_stride;
+          A.tokens = J.tokens;
+          A.scale = J.scale;
+          A.nq = (int32_t)J.q.rows;
+          A.nk = J.cfg_k.n_angle; A.wk = tac::code_bits(J.cfg_k.n_angle); A.bk = J.cfg_k.norm_bits; A.mk = J.cfg_k.norm_mode;
+          A.nv = J.cfg_v.n_angle; A.wv = tac::code_bits(J.cfg_v.n_angle); A.bv = J.cfg_v.norm_bits; A.mv = J.cfg_v.norm_mode;
+          A.inv_lk = A.mk == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bk) - 1);
+          A.inv_lv = A.mv == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bv) - 1);
+          copy_signs(A.sk, &J.cfg_k);
+          copy_signs(A.sv, &J.cfg_v);
+          A.split0 = (int32_t)splits;
+          A.cta0 = (int32_t)ctas;
+          A.ws = ws_off;
+          ws_off += attend_ws_floats(J);
+          splits += ns;
+          ctas += nc;
+          nrows += A.nq;
+          nq_max = std::max(nq_max, (int)A.nq);
+          ++P.njobs;
+          i = next(i + 1);
+        }
+        if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many tokens", who);
+        P.nctas = (int32_t)ctas;
+        P.nsplits = (int32_t)splits;
+        cudaError_t e = tac::launch_attend(d, dt, nq_max, P, nrows, ws, st);
+        if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+      }
+    }
+  }
+  return ok();
+}
+
+}  // namespace
+
+int tac_attend_multi(const tac_attend_job* jobs, int njobs, void* workspace, int64_t workspace_bytes,
+                     tac_stream_t stream) {
+  static const char* who = "tac_attend_multi";
+  int64_t need = 0;
+  const int rc = check_attend_jobs(jobs, njobs, &need, who);
+  if (rc) return rc;
   if (njobs == 0) return ok();
   if (!workspace || !aligned16(workspace) || workspace_bytes < need)
     return fail(TAC_E_INVAL, "%s: workspace NULL, misaligned or smaller than %lld bytes", who, (long long)need);
   if (num_sms() <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
-  // Group by (d, dtype); each job's workspace part follows the previous job's.
-  std::vector<int> order(njobs);
-  for (int j = 0; j < njobs; ++j) order[j] = j;
-  std::stable_sort(order.begin(), order.end(), [&](int a, int b) {
-    return jobs[a].cfg_k.d * 4 + jobs[a].q.dtype < jobs[b].cfg_k.d * 4 + jobs[b].q.dtype;
-  });
-  static thread_local tac::AttParams P;
-  float* ws = static_cast<float*>(workspace);
-  int64_t ws_off = 0;
-  size_t i = 0;
-  while (i < order.size()) {
-    const int d = jobs[order[i]].cfg_k.d, dt = jobs[order[i]].q.dtype;
-    std::memset(&P, 0, sizeof(P));
-    int64_t ctas = 0, splits = 0;
-    int nrows = 0, nq_max = 1;
-    while (i < order.size() && P.njobs < TAC_MAX_JOBS && jobs[order[i]].cfg_k.d == d &&
-           jobs[order[i]].q.dtype == dt) {
-      const tac_attend_job& J = jobs[order[i]];
-      const int64_t ns = (J.tokens + TAC_ATTEND_SPLIT - 1) / TAC_ATTEND_SPLIT;
-      const int64_t nc = (ns + 3) / 4;
-      if (ctas + nc > 0x7fffffff || splits + ns > 0x7fffffff) break;
-      tac::AttJob& A = P.job[P.njobs];
-      A.kc = static_cast<const uint8_t*>(J.k_codes);
-      A.kn = static_cast<const uint8_t*>(J.k_norms);
-      A.kh = A.kn + header_offset(&J.cfg_k, J.capacity);
-      A.vc = static_cast<const uint8_t*>(J.v_codes);
-      A.vn = static_cast<const uint8_t*>(J.v_norms);
-      A.vh = A.vn + header_offset(&J.cfg_v, J.capacity);
-      A.q = J.q.data;
-      A.out = J.out.data;
-      A.q_stride = J.q.row_stride;
-      A.out_stride = J.out.row_stride;
-      A.tokens = J.tokens;
-      A.scale = J.scale;
-      A.nq = (int32_t)J.q.rows;
-      A.nk = J.cfg_k.n_angle; A.wk = tac::code_bits(J.cfg_k.n_angle); A.bk = J.cfg_k.norm_bits; A.mk = J.cfg_k.norm_mode;
-      A.nv = J.cfg_v.n_angle; A.wv = tac::code_bits(J.cfg_v.n_angle); A.bv = J.cfg_v.norm_bits; A.mv = J.cfg_v.norm_mode;
-      A.inv_lk = A.mk == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bk) - 1);
-      A.inv_lv = A.mv == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bv) - 1);
-      copy_signs(A.sk, &J.cfg_k);
-      copy_signs(A.sv, &J.cfg_v);
-      A.split0 = (int32_t)splits;
-      A.cta0 = (int32_t)ctas;
-      A.ws = ws_off;
-      ws_off += attend_ws_floats(J);
-      splits += ns;
-      ctas += nc;
-      nrows += A.nq;
-      nq_max = std::max(nq_max, (int)A.nq);
-      ++P.njobs;
-      ++i;
-    }
-    if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many tokens", who);
-    P.nctas = (int32_t)ctas;
-    P.nsplits = (int32_t)splits;
-    cudaError_t e = tac::launch_attend(d, dt, nq_max, P, nrows, ws, reinterpret_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
-  }
-  return ok();
+  return run_attend(jobs, njobs, static_cast<float*>(workspace), reinterpret_cast<cudaStream_t>(stream), who);
+}
+
+int tac_attend_multi_static(const tac_attend_job* jobs, int njobs, tac_stream_t stream) {
+  static const char* who = "tac_attend_multi_static";
+  int64_t need = 0;
+  const int rc = check_attend_jobs(jobs, njobs, &need, who);
+  if (rc) return rc;
+  if (need > TAC_ATTEND_STATIC_WS_BYTES)
+    return fail(TAC_E_UNSUPPORTED,
+                "%s: these jobs need %lld bytes of workspace, the static workspace holds %lld; "
+                "split them over several calls or use tac_attend_multi",
+                who, (long long)need, (long long)TAC_ATTEND_STATIC_WS_BYTES);
+  float* ws = nullptr;
+  const cudaError_t e = tac::attend_static_workspace(&ws);
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: static workspace: %s", who, cudaGetErrorString(e));
+  if (njobs == 0) return ok();
+  if (num_sms() <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
+  return run_attend(jobs, njobs, ws, reinterpret_cast<cudaStream_t>(stream), who);
 }
 
 int tac_fwht_debug(const tac_rows* x, int d, const uint32_t* signs, float* y, tac_stream_t stream) {

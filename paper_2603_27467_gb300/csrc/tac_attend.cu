@@ -24,6 +24,8 @@
 //                   applies D H (fp32 butterfly) and stores the row.
 // Codebooks (n, norm bits, norm mode) are runtime parameters: K and V may
 // differ, and any codebook the encoder supports is accepted.
+#include <atomic>
+
 #include "tac_common.cuh"
 
 namespace tac {
@@ -397,6 +399,29 @@ static cudaError_t launch_attend_t(const AttParams& p, int nrows_total, float* w
   const int blocks = (nrows_total + 3) / 4;
   if (blocks > 0) attend_combine<D, TQ><<<blocks, 128, 0, st>>>(p, ws, nrows_total);
   return cudaGetLastError();
+}
+
+// The workspace of tac_attend_multi_static: one array per device, in the
+// module image (no allocation at call time).
+static __device__ __align__(256) float g_attend_ws[TAC_ATTEND_STATIC_WS_BYTES / 4];
+
+// Address of g_attend_ws on the current device, resolved once per device.
+cudaError_t attend_static_workspace(float** ws) {
+  constexpr int kMaxDevices = 64;
+  static std::atomic<void*> cache[kMaxDevices];
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  void* a = cache[dev].load(std::memory_order_acquire);
+  if (!a) {
+    e = cudaGetSymbolAddress(&a, g_attend_ws);
+    if (e != cudaSuccess) return e;
+    if (!a || (reinterpret_cast<uintptr_t>(a) & 255)) return cudaErrorInvalidSymbol;
+    cache[dev].store(a, std::memory_order_release);   // racing first calls store the same address
+  }
+  *ws = static_cast<float*>(a);
+  return cudaSuccess;
 }
 
 // nq_max: the largest query count of the jobs (the kernel is built for 1, 2, 4, 8).
