@@ -361,6 +361,8 @@ def run_e2e(tac, ws, world, dev, steps, chunk_blocks, step_bytes, barrier):
     ev_cmp = [torch.cuda.Event() for _ in chunks]   # chunk c encoded and decoded
     ev_out = [torch.cuda.Event() for _ in chunks]   # decoded rows of chunk c are on the host
     state = {"first": True}
+    enc_calls = [tac.encode_multi_prepared(ws.enc_jobs[lo:hi]) for lo, hi in chunks]
+    dec_calls = [tac.decode_multi_prepared(ws.dec_jobs[lo:hi]) for lo, hi in chunks]
 
     def one_step():
         first = state["first"]
@@ -374,8 +376,8 @@ def run_e2e(tac, ws, world, dev, steps, chunk_blocks, step_bytes, barrier):
                 s_cmp.wait_event(ev_in[c])
                 if not first:
                     s_cmp.wait_event(ev_out[c])       # last step's copy-out has read these rows
-                tac.encode_multi(ws.enc_jobs[lo:hi], stream=s_cmp)
-                tac.decode_multi(ws.dec_jobs[lo:hi], stream=s_cmp)
+                enc_calls[c](s_cmp)
+                dec_calls[c](s_cmp)
                 ev_cmp[c].record(s_cmp)
             with torch.cuda.stream(s_out):
                 s_out.wait_event(ev_cmp[c])
@@ -443,8 +445,9 @@ def run_attend(args):
         keep.append(caches)
     ws = torch.empty(tac.attend_workspace_bytes(jobs), dtype=torch.uint8, device=dev)
     stream = torch.cuda.Stream(device=dev)
+    call = tac.attend_multi_prepared(jobs, ws)
     for _ in range(args.warmup):
-        tac.attend_multi(jobs, ws, stream=stream)
+        call(stream)
     torch.cuda.synchronize()
     clk = ClockSampler(None)
     clk.start()
@@ -453,7 +456,7 @@ def run_attend(args):
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        tac.attend_multi(jobs, ws, stream=stream)
+        call(stream)
     e1.record(stream)
     torch.cuda.synchronize()
     clocks = clk.stop()
@@ -545,10 +548,13 @@ def main():
     stream = torch.cuda.Stream(device=dev)
     enc_only = args.config == "append"
 
+    enc_call = tac.encode_multi_prepared(ws.enc_jobs)
+    dec_call = tac.decode_multi_prepared(ws.dec_jobs)
+
     def step():
-        tac.encode_multi(ws.enc_jobs, stream=stream)
+        enc_call(stream)
         if not enc_only:
-            tac.decode_multi(ws.dec_jobs, stream=stream)
+            dec_call(stream)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -571,10 +577,10 @@ def main():
     t_start.record(stream)
     for i in range(K):
         ev[i][0].record(stream)
-        tac.encode_multi(ws.enc_jobs, stream=stream)
+        enc_call(stream)
         ev[i][1].record(stream)
         if not enc_only:
-            tac.decode_multi(ws.dec_jobs, stream=stream)
+            dec_call(stream)
         ev[i][2].record(stream)
     t_end.record(stream)
     barrier()

@@ -323,8 +323,19 @@ def decode(cache: Cache, cfg: LayerCfg, rows: int | None = None, dtype=None, y=N
     return y
 
 
-def encode_multi(jobs, stream=None) -> None:
-    """tac_encode_multi: one launch per kernel group (see launch_count)."""
+class Prepared:
+    """A batched call with its job array marshalled once: calling it makes only
+    the C call.  The jobs' tensors must stay allocated (their addresses are in
+    the array) and the jobs unchanged while it is used."""
+
+    def __init__(self, fn, arr, n, extra, keep):
+        self._fn, self._arr, self._n, self._extra, self._keep = fn, arr, n, extra, keep
+
+    def __call__(self, stream=None) -> None:
+        _check(self._fn(self._arr, self._n, *self._extra, _stream_ptr(stream)))
+
+
+def _enc_array(jobs):
     arr = (_EncJob * max(1, len(jobs)))()
     for i, j in enumerate(jobs):
         e = arr[i]
@@ -334,11 +345,20 @@ def encode_multi(jobs, stream=None) -> None:
         e.norms = j.cache.norms.data_ptr()
         e.capacity = j.cache.capacity
         e.slot = j.slot.data_ptr() if j.slot is not None else None
-    _check(load().tac_encode_multi(arr, len(jobs), _stream_ptr(stream)))
+    return arr
 
 
-def decode_multi(jobs, stream=None) -> None:
-    """tac_decode_multi: one launch per kernel group (see launch_count)."""
+def encode_multi(jobs, stream=None) -> None:
+    """tac_encode_multi: one launch per kernel group (see launch_count)."""
+    _check(load().tac_encode_multi(_enc_array(jobs), len(jobs), _stream_ptr(stream)))
+
+
+def encode_multi_prepared(jobs) -> Prepared:
+    """tac_encode_multi over `jobs`, marshalled once (see Prepared)."""
+    return Prepared(load().tac_encode_multi, _enc_array(jobs), len(jobs), (), list(jobs))
+
+
+def _dec_array(jobs):
     arr = (_DecJob * max(1, len(jobs)))()
     for i, j in enumerate(jobs):
         e = arr[i]
@@ -348,7 +368,17 @@ def decode_multi(jobs, stream=None) -> None:
         e.capacity = j.cache.capacity
         e.slot = j.slot.data_ptr() if j.slot is not None else None
         e.y = _rows(j.y, j.cfg.d)
-    _check(load().tac_decode_multi(arr, len(jobs), _stream_ptr(stream)))
+    return arr
+
+
+def decode_multi(jobs, stream=None) -> None:
+    """tac_decode_multi: one launch per kernel group (see launch_count)."""
+    _check(load().tac_decode_multi(_dec_array(jobs), len(jobs), _stream_ptr(stream)))
+
+
+def decode_multi_prepared(jobs) -> Prepared:
+    """tac_decode_multi over `jobs`, marshalled once (see Prepared)."""
+    return Prepared(load().tac_decode_multi, _dec_array(jobs), len(jobs), (), list(jobs))
 
 
 @dataclass
@@ -398,6 +428,22 @@ def attend_multi(jobs, workspace=None, stream=None):
     _check(load().tac_attend_multi(arr, len(jobs), workspace.data_ptr() if jobs else None,
                                    workspace.numel() * workspace.element_size(), _stream_ptr(stream)))
     return workspace
+
+
+def attend_multi_prepared(jobs, workspace=None, static=False) -> Prepared:
+    """tac_attend_multi (or tac_attend_multi_static) over `jobs`, marshalled
+    once (see Prepared); allocates the workspace (torch) when none is given."""
+    lib = load()
+    arr = _att_array(jobs)
+    if static:
+        return Prepared(lib.tac_attend_multi_static, arr, len(jobs), (), list(jobs))
+    torch = _torch()
+    need = attend_workspace_bytes(jobs) if jobs else 0
+    if workspace is None:
+        dev = jobs[0].q.device if jobs else "cuda"
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    extra = (workspace.data_ptr() if jobs else None, workspace.numel() * workspace.element_size())
+    return Prepared(lib.tac_attend_multi, arr, len(jobs), extra, (list(jobs), workspace))
 
 
 def attend_multi_static(jobs, stream=None):

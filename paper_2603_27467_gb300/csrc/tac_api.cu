@@ -533,6 +533,10 @@ int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st
           A.nv = J.cfg_v.n_angle; A.wv = tac::code_bits(J.cfg_v.n_angle); A.bv = J.cfg_v.norm_bits; A.mv = J.cfg_v.norm_mode;
           A.inv_lk = A.mk == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bk) - 1);
           A.inv_lv = A.mv == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bv) - 1);
+          A.lgrk = tac::att_table_lgr(A.nk);
+          A.lgrv = tac::att_table_lgr(A.nv);
+          A.ck = tac::att_norm_case(A.bk, A.mk);
+          A.cv = tac::att_norm_case(A.bv, A.mv);
           copy_signs(A.sk, &J.cfg_k);
           copy_signs(A.sv, &J.cfg_v);
           A.split0 = (int32_t)splits;
@@ -549,6 +553,7 @@ int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st
         if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many tokens", who);
         P.nctas = (int32_t)ctas;
         P.nsplits = (int32_t)splits;
+        P.q_bf16 = dt == TAC_BF16;
         cudaError_t e = tac::launch_attend(d, dt, nq_max, P, nrows, ws, st);
         if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
       }

@@ -24,67 +24,87 @@
 //                   applies D H (fp32 butterfly) and stores the row.
 // Codebooks (n, norm bits, norm mode) are runtime parameters: K and V may
 // differ, and any codebook the encoder supports is accepted.
+#include <algorithm>
 #include <atomic>
 
 #include "tac_common.cuh"
 
 namespace tac {
 
+template <int V>
+struct IC { static constexpr int value = V; };
+
 constexpr int kAttWarps = 4;                  // warps (splits) per CTA
 constexpr int kAttThreads = 32 * kAttWarps;
-constexpr int kAttSplit = TAC_ATTEND_SPLIT;   // tokens per split
-constexpr int kAttNS = 3;                     // record stages per warp
+constexpr int kAttSplit = TAC_ATTEND_SPLIT;   // tokens per split (one warp)
+constexpr int kAttNS = 2;                     // staged batches per warp
 constexpr float kLog2e = 1.4426950408889634f;
+static_assert(kAttSplit % kAttBatch == 0, "a split is whole batches");
 
-template <int D>
+template <int D, int NQ>
 struct Att {
   using G = Geo<D>;
-  static constexpr int P = G::P, L = G::L, RW = G::RW;
-  static constexpr int PV = P / 32 > 0 ? P / 32 : 1;         // V pairs per lane (d = 64: 1, 128: 2)
-  // record stage: K angle | K norm | K header | V angle | V norm | V header, each
-  // at most RW * (P, 4P, 8) bytes (angle codes <= 8 bits, fp32 norms)
-  static constexpr int SEG_A = RW * P, SEG_N = RW * 4 * P, SEG_H = RW * 8;
-  static constexpr int S_KA = 0, S_KN = S_KA + SEG_A, S_KH = S_KN + SEG_N;
-  static constexpr int S_VA = S_KH + SEG_H, S_VN = S_VA + SEG_A, S_VH = S_VN + SEG_N;
-  static constexpr int STAGE = S_VH + SEG_H + 16;            // + slack for funnel reads
-  static constexpr int QROW = P + P / 8;                      // skewed rotated-query row (float2 units)
-  // CTA shared memory
-  static constexpr int OFF_Q = 0;                                             // float2 [TAC_MAX_QUERIES][QROW]
-  static constexpr int OFF_TK = OFF_Q + TAC_MAX_QUERIES * QROW * 8;           // float2 [256] K (cos, sin)
-  static constexpr int OFF_TV = OFF_TK + 256 * 8;                             // float2 [256] V (cos, sin)
-  static constexpr int OFF_W = OFF_TV + 256 * 8;                              // per-warp stages
-  static constexpr int SMEM = OFF_W + kAttWarps * kAttNS * STAGE;
-  static_assert(STAGE % 16 == 0 && OFF_W % 16 == 0, "alignment");
+  static constexpr int P = G::P, L = G::L, RW = G::RW;   // K: L lanes per token, RW tokens per pass
+  static constexpr int PV = P / 32;                      // V: pairs per lane
+  static constexpr int QROW = P + P / 4;                 // skewed rotated-query row (float2 units)
+  static constexpr int PBROW = 16 + 16 * ((NQ + 1) / 2); // per token: V constants, then (p, p) per query
+  static constexpr int PB = kAttBatch * PBROW;
+  // CTA shared memory: rotated queries | K table | V table | per warp (PB, kAttNS stages)
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_TK = OFF_Q + NQ * QROW * 8;
+  static constexpr int OFF_TV = OFF_TK + kAttTabBytes;
+  static constexpr int OFF_W = OFF_TV + kAttTabBytes;
+  static constexpr int smem(int stage) { return OFF_W + kAttWarps * (PB + kAttNS * stage); }
+  static_assert(OFF_TK % 16 == 0 && PB % 16 == 0 && P % 32 == 0, "layout");
 };
 
-// The skewed position of pair i in a rotated-query row: pairs 8l..8l+7 of the
-// L lanes of a row then fall on distinct bank pairs.
-__device__ __forceinline__ int qpos(int i) { return i + (i >> 3); }
+// The skewed position of pair i in a rotated-query row: the 16-byte granules
+// (pairs 8l + 2m, 8l + 2m + 1) of the L lanes of a token fall on distinct banks.
+__device__ __forceinline__ int qpos(int i) { return i + 2 * (i >> 3); }
 
-// Up to 8 bytes from a shared byte address with any alignment.
-__device__ __forceinline__ uint64_t load_u64_any(const uint8_t* p) {
-  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
-  const uint32_t* w = reinterpret_cast<const uint32_t*>(a & ~(uintptr_t)3);
-  const int sh = (int)(a & 3) * 8;
-  const uint64_t lo = (uint64_t)w[0] | ((uint64_t)w[1] << 32);
-  uint64_t v = lo >> sh;
-  if (sh) v |= (uint64_t)w[2] << (64 - sh);
+__device__ __forceinline__ uint32_t rotr(uint32_t x, int s) { return __funnelshift_r(x, x, s); }
+
+// A shared-memory float4 load the compiler may not hoist or merge: keeps a
+// loop-invariant operand in shared memory instead of in registers.
+__device__ __forceinline__ float4 lds_f4_reload(const void* ptr) {
+  float4 v;
+  const uint32_t a = (uint32_t)__cvta_generic_to_shared(ptr);
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];\n" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a));
   return v;
 }
 
-// Dequantization constants of one record (the inverse of Eq. 2): r^ = base + c step
-// (linear) or 2^(base + c step) (log); inv_l = 1 / (2^b - 1).
-__device__ __forceinline__ float2 norm_consts(const uint8_t* hdr, float inv_l, int mode) {
-  const float2 h = *reinterpret_cast<const float2*>(hdr);
-  const bool spread = h.y > h.x;
-  if (mode == TAC_NORM_LINEAR) return make_float2(h.x, spread ? (h.y - h.x) * inv_l : 0.f);
-  const float lmin = lg2_approx(h.x);
-  return make_float2(lmin, spread ? (lg2_approx(h.y) - lmin) * inv_l : 0.f);
+// Reduce-scatter over the L lanes of a token, as a tree over the passes: the
+// lane's value for the pass set {I + k S} is its half, selected by lane bit S,
+// of the two sets {I + 2kS} and {I + S + 2kS}, plus the partner's.  At the
+// top (I = 0, S = 1) lane l holds the sum over the L lanes of pass l.
+template <int L, int I, int S, int NQ, typename PF>
+__device__ __forceinline__ void att_tree(PF& pass, int l, float (&v)[NQ]) {
+  float va[NQ], vb[NQ];
+  if constexpr (2 * S == L) {
+    pass(IC<I>{}, va);
+    pass(IC<I + S>{}, vb);
+  } else {
+    att_tree<L, I, 2 * S, NQ>(pass, l, va);
+    att_tree<L, I + S, 2 * S, NQ>(pass, l, vb);
+  }
+  const bool up = (l & S) != 0;
+#pragma unroll
+  for (int a = 0; a < NQ; ++a) {
+    const float kept = up ? vb[a] : va[a];
+    const float send = up ? va[a] : vb[a];
+    v[a] = kept + __shfl_xor_sync(0xffffffffu, send, S);
+  }
 }
 
-__device__ __forceinline__ float dequant(uint32_t c, float2 bs, int mode) {
-  const float v = __fmaf_rn((float)c, bs.y, bs.x);
-  return mode == TAC_NORM_LOG ? ex2_approx(v) : v;
+// (A, B) of one record's norms: r^ = A f + B for the code c entered as
+// f = 1 + c 2^-b (its bits in the mantissa of 1.0); log mode gives log2 r^.
+// This is the inverse of Eq. 2: base + c step = f 2^b step + (base - 2^b step).
+__device__ __forceinline__ float2 norm_ab(float2 h, float inv_l, float two_b, bool lg) {
+  const float lo = lg ? lg2_approx(h.x) : h.x;
+  const float hi = lg ? lg2_approx(h.y) : h.y;
+  const float step = h.y > h.x ? (hi - lo) * inv_l : 0.f;
+  const float A = step * two_b;
+  return make_float2(A, lo - A);
 }
 
 // In-place normalized Walsh-Hadamard transform of `rows` rows of d floats in
@@ -105,12 +125,10 @@ __device__ __forceinline__ void smem_fwht(float* buf, int rows, int tid, int nth
   if (block_sync) __syncthreads(); else __syncwarp();
 }
 
-template <int D, typename TQ, int NQ>
-__global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_constant__ AttParams p, float* ws) {
-  using C = Att<D>;
-  using G = Geo<D>;
+template <int D, int NQ>
+__global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(const __grid_constant__ AttParams p, float* ws) {
+  using C = Att<D, NQ>;
   constexpr int P = C::P, L = C::L, RW = C::RW, PV = C::PV;
-  constexpr int ESZ = (int)sizeof(TQ);
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
@@ -127,28 +145,39 @@ __global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_const
   const AttJob& J = p.job[jb];
   const int nq = J.nq;
 
+  // ---- batch geometry of this job's records ----
+  const int ak = P * J.wk / 8, nbk = P * J.bk / 8, av = P * J.wv / 8, nbv = P * J.bv / 8;
+  const int hkb = J.mk != TAC_NORM_FP32 ? 8 : 0, hvb = J.mv != TAC_NORM_FP32 ? 8 : 0;
+  const int S_KN = kAttBatch * ak, S_KH = S_KN + kAttBatch * nbk, S_VA = S_KH + kAttBatch * hkb;
+  const int S_VN = S_VA + kAttBatch * av, S_VH = S_VN + kAttBatch * nbv;
+  const int stage = S_VH + kAttBatch * hvb + 16;   // == att_stage_bytes(...)
+
   // ---- rotated queries q' = H D_K q * scale * log2(e), skewed float2 rows ----
-  float* qbuf = reinterpret_cast<float*>(smem + C::OFF_W);   // staging, reused by the record ring below
+  float* qbuf = reinterpret_cast<float*>(smem + C::OFF_W);   // staging, reused by the batches below
   for (int e = tid; e < nq * D; e += kAttThreads) {
     const int a = e / D, j = e % D;
-    const uint8_t* qr = reinterpret_cast<const uint8_t*>(J.q) + (int64_t)a * J.q_stride * ESZ;
     float x;
-    if constexpr (ESZ == 2) x = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(qr)[j]);
-    else x = reinterpret_cast<const float*>(qr)[j];
+    if (p.q_bf16) {
+      x = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(J.q)[(int64_t)a * J.q_stride + j]);
+    } else {
+      x = reinterpret_cast<const float*>(J.q)[(int64_t)a * J.q_stride + j];
+    }
     qbuf[e] = ((J.sk[j >> 5] >> (j & 31)) & 1u) ? -x : x;
   }
   smem_fwht<D>(qbuf, nq, tid, kAttThreads, true);
   float2* qrot = reinterpret_cast<float2*>(smem + C::OFF_Q);
   const float qs = J.scale * kLog2e * rsqrtf((float)D);
-  for (int e = tid; e < nq * P; e += kAttThreads) {
+  for (int e = tid; e < NQ * P; e += kAttThreads) {
     const int a = e / P, i = e % P;
-    qrot[a * C::QROW + qpos(i)] = make_float2(qbuf[a * D + 2 * i] * qs, qbuf[a * D + 2 * i + 1] * qs);
+    qrot[a * C::QROW + qpos(i)] =
+        a < nq ? make_float2(qbuf[a * D + 2 * i] * qs, qbuf[a * D + 2 * i + 1] * qs) : make_float2(0.f, 0.f);
   }
-  // ---- bin-centre tables (cos, sin)(2 pi k / n) ----
+  // ---- bin-centre tables (cos, sin)(2 pi k / n), 2^lgr copies: entry k copy c at k 2^lgr + c ----
+  const int lgrk = J.lgrk, lgrv = J.lgrv;
   float2* tk = reinterpret_cast<float2*>(smem + C::OFF_TK);
   float2* tv = reinterpret_cast<float2*>(smem + C::OFF_TV);
-  for (int k = tid; k < J.nk; k += kAttThreads) tk[k] = cos_sin_q8(8 * k, J.nk);
-  for (int k = tid; k < J.nv; k += kAttThreads) tv[k] = cos_sin_q8(8 * k, J.nv);
+  for (int e = tid; e < (J.nk << lgrk); e += kAttThreads) tk[e] = cos_sin_q8(8 * (e >> lgrk), J.nk);
+  for (int e = tid; e < (J.nv << lgrv); e += kAttThreads) tv[e] = cos_sin_q8(8 * (e >> lgrv), J.nv);
   __syncthreads();
 
   // ---- this warp's split ----
@@ -156,27 +185,24 @@ __global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_const
   const int64_t t_begin = (int64_t)(split - J.split0) * kAttSplit;
   if (t_begin >= J.tokens) return;
   const int64_t t_stop = min(J.tokens, t_begin + kAttSplit);
-  const int nsteps = (int)((t_stop - t_begin + RW - 1) / RW);
-  uint8_t* wsm = smem + C::OFF_W + warp * kAttNS * C::STAGE;
+  const int nb = (int)((t_stop - t_begin + kAttBatch - 1) / kAttBatch);
+  uint8_t* pb = smem + C::OFF_W + warp * (C::PB + kAttNS * stage);
+  uint8_t* stg = pb + C::PB;
 
-  const int ak = P * J.wk / 8, nbk = P * J.bk / 8;     // K record bytes per row (angle, norm)
-  const int av = P * J.wv / 8, nbv = P * J.bv / 8;
-  const bool hk = J.mk != TAC_NORM_FP32, hv = J.mv != TAC_NORM_FP32;
-
-  // Stage the records of step s (tokens t_begin + s*RW ...): six segments,
-  // 16-byte chunks, bytes past the last token zero-filled.
+  // Stage batch s (tokens t_begin + 32 s ...): six segments in 16-byte
+  // chunks, bytes past the last token zero-filled.
   auto issue = [&](int s) {
-    if (s < nsteps) {
-      const int64_t row0 = t_begin + (int64_t)s * RW;
-      const int rows = (int)min((int64_t)RW, J.tokens - row0);
-      uint8_t* st = wsm + (s % kAttNS) * C::STAGE;
+    if (s < nb) {
+      const int64_t row0 = t_begin + (int64_t)s * kAttBatch;
+      const int rows = (int)min((int64_t)kAttBatch, J.tokens - row0);
+      uint8_t* st = stg + (s % kAttNS) * stage;
       const uint8_t* src[6] = {J.kc + row0 * ak, J.kn + row0 * nbk, J.kh + row0 * 8,
                                J.vc + row0 * av, J.vn + row0 * nbv, J.vh + row0 * 8};
-      const int rb[6] = {ak, nbk, hk ? 8 : 0, av, nbv, hv ? 8 : 0};
-      const int off[6] = {C::S_KA, C::S_KN, C::S_KH, C::S_VA, C::S_VN, C::S_VH};
+      const int rb[6] = {ak, nbk, hkb, av, nbv, hvb};
+      const int off[6] = {0, S_KN, S_KH, S_VA, S_VN, S_VH};
 #pragma unroll
       for (int g = 0; g < 6; ++g) {
-        const int full = RW * rb[g], valid = rows * rb[g];
+        const int full = kAttBatch * rb[g], valid = rows * rb[g];
         for (int c = lane * 16; c < full; c += 32 * 16) {
           const int rem = valid - c;
           const int n = rem >= 16 ? 16 : (rem > 0 ? rem : 0);
@@ -186,149 +212,233 @@ __global__ void __launch_bounds__(kAttThreads) attend_partial(const __grid_const
     }
     cp_async_commit();
   };
-#pragma unroll
-  for (int s = 0; s < kAttNS - 1; ++s) issue(s);
 
-  const int r = lane / L, l = lane % L;     // K layout: token r of the step, pairs 8l..8l+7
-  // V layout: lane owns pairs lane + 32 j; their code positions are fixed per job
-  int va_w[PV], va_s[PV], vn_w[PV], vn_s[PV];
+  // ---- lane constants ----
+  // K: lane (r, l) takes pairs 8l..8l+7 of token r of each pass of RW tokens;
+  // its 8 codes start at bit 8 W l of the row.  A code becomes the byte offset
+  // of its table entry (copy lane % 2^lgr) by one rotate and one mask.
+  const int r = lane / L, l = lane % L;
+  const int wk = J.wk, Tk = 3 + lgrk;
+  const int kbit = 8 * wk * l, kwa = kbit >> 5, ksa = kbit & 31;
+  const bool kup = ksa + 4 * wk >= 32;                    // codes 4..7 start in the next word
+  const int ksb = (ksa + 4 * wk) & 31;
+  const uint32_t kC = (uint32_t)(lane & ((1 << lgrk) - 1)) << 3;
+  const uint32_t kM = ((1u << wk) - 1u) << Tk;
+  const uint32_t kMax = ((uint32_t)(J.nk - 1) << Tk) | kC;   // clamps codes >= n (n not a power of two)
+  int kra[4];
 #pragma unroll
-  for (int j = 0; j < PV; ++j) {
-    const int i = lane + 32 * j, ba = i * J.wv, bn = i * J.bv;
-    va_w[j] = ba >> 5; va_s[j] = ba & 31;
-    vn_w[j] = bn >> 5; vn_s[j] = bn & 31;
-  }
-  const uint32_t vmask = (1u << J.wv) - 1u;
-  const uint32_t nvmask = J.bv >= 32 ? 0xffffffffu : (1u << J.bv) - 1u;
+  for (int j = 0; j < 4; ++j) kra[j] = (wk * j - Tk) & 31;
+  // V: lane owns pairs PV lane .. PV lane + PV - 1; its codes start at bit PV W lane.
+  const int wv = J.wv, Tv = 3 + lgrv;
+  const int vbit = PV * wv * lane, vwa = vbit >> 5, vsa = vbit & 31;
+  const uint32_t vC = (uint32_t)(lane & ((1 << lgrv) - 1)) << 3;
+  const uint32_t vM = ((1u << wv) - 1u) << Tv;
+  const uint32_t vMax = ((uint32_t)(J.nv - 1) << Tv) | vC;
+  int vra[PV];
+#pragma unroll
+  for (int j = 0; j < PV; ++j) vra[j] = (wv * j - Tv) & 31;
+  const float kinv = J.inv_lk, vinv = J.inv_lv;
+  const bool vlog = J.mv == TAC_NORM_LOG;
+  const float v2b = J.mv == TAC_NORM_FP32 ? 0.f : (float)(1 << J.bv);
+
   float m_run[NQ], l_run[NQ];
-  float acc[NQ][PV][2];
+  float2 acc[NQ][PV];
 #pragma unroll
   for (int a = 0; a < NQ; ++a) {
     m_run[a] = -INFINITY;
     l_run[a] = 0.f;
 #pragma unroll
-    for (int j = 0; j < PV; ++j) acc[a][j][0] = acc[a][j][1] = 0.f;
+    for (int j = 0; j < PV; ++j) acc[a][j] = make_float2(0.f, 0.f);
   }
 
-  for (int s = 0; s < nsteps; ++s) {
-    cp_async_wait<kAttNS - 2>();
-    __syncwarp();
-    issue(s + kAttNS - 1);
-    const uint8_t* st = wsm + (s % kAttNS) * C::STAGE;
-    const int64_t row0 = t_begin + (int64_t)s * RW;
-    const int valid = (int)min((int64_t)RW, t_stop - row0);   // tokens of this step
-    // dequantization constants of the V record of token r (broadcast in the V phase)
-    const float2 vbs = hv ? norm_consts(st + C::S_VH + r * 8, J.inv_lv, J.mv) : make_float2(0.f, 0.f);
-
-    // ---- K: partial scores of token r over pairs 8l..8l+7 ----
-    float sc[NQ];
+  // Scores of the batch in `st`: after the passes and the reduction, lane
+  // (r, l) holds, for each query, the score of token RW l + r.
+  auto scores = [&](const uint8_t* st, float (&keep)[NQ], auto kc_) {
+    constexpr int KC = decltype(kc_)::value;
+    constexpr bool F32 = KC == 4, LOG = KC == 1 || KC == 3;
+    constexpr int KB = KC <= 1 ? 4 : 8;
+    auto pass = [&](auto k_, float (&part)[NQ]) {
+      const int row = decltype(k_)::value * RW + r;
+      const uint32_t* arow = reinterpret_cast<const uint32_t*>(st + row * ak);
+      const uint32_t w0 = arow[kwa], w1 = arow[kwa + 1], w2 = arow[kwa + 2];
+      const uint32_t x0 = __funnelshift_r(w0, w1, ksa);
+      const uint32_t x1 = kup ? __funnelshift_r(w1, w2, ksb) : __funnelshift_r(w0, w1, ksb);
+      float rh[8];
+      if constexpr (F32) {
+        const float4* nr = reinterpret_cast<const float4*>(st + S_KN + row * nbk + 32 * l);
+        const float4 n0 = nr[0], n1 = nr[1];
+        rh[0] = n0.x; rh[1] = n0.y; rh[2] = n0.z; rh[3] = n0.w;
+        rh[4] = n1.x; rh[5] = n1.y; rh[6] = n1.z; rh[7] = n1.w;
+      } else {
+        const float2 ab = norm_ab(*reinterpret_cast<const float2*>(st + S_KH + row * 8), kinv, (float)(1 << KB), LOG);
+        uint32_t nw[2];
+        if constexpr (KB == 8) {
+          const uint2 v = *reinterpret_cast<const uint2*>(st + S_KN + row * nbk + 8 * l);
+          nw[0] = v.x; nw[1] = v.y;
+        } else {
+          nw[0] = nw[1] = *reinterpret_cast<const uint32_t*>(st + S_KN + row * nbk + 4 * l);
+        }
 #pragma unroll
-    for (int a = 0; a < NQ; ++a) sc[a] = 0.f;
-    {
-      const uint64_t ka = load_u64_any(st + C::S_KA + r * ak + l * J.wk);
-      const uint32_t kmask = (1u << J.wk) - 1u;
-      const float2 bs = hk ? norm_consts(st + C::S_KH + r * 8, J.inv_lk, J.mk) : make_float2(0.f, 0.f);
-      const uint8_t* nrow = st + C::S_KN + r * nbk;
-      uint64_t kn = 0;
-      if (J.mk != TAC_NORM_FP32)
-        kn = J.bk == 8 ? load_u64_any(nrow + l * 8) : (uint64_t)reinterpret_cast<const uint32_t*>(nrow)[l];
+        for (int j = 0; j < 8; ++j) {
+          constexpr uint32_t NM = ((1u << KB) - 1u) << (23 - KB);
+          const int bit = KB * j;
+          const uint32_t fb = (rotr(nw[bit >> 5], ((bit & 31) - (23 - KB)) & 31) & NM) | 0x3F800000u;
+          float v = __fmaf_rn(__uint_as_float(fb), ab.x, ab.y);
+          if constexpr (LOG) v = ex2_approx(v);
+          rh[j] = v;
+        }
+      }
+      float2 sc[NQ];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        uint32_t k = (uint32_t)(ka >> (j * J.wk)) & kmask;
-        k = min(k, (uint32_t)(J.nk - 1));
-        float rh;
-        if (J.mk == TAC_NORM_FP32) rh = reinterpret_cast<const float*>(nrow)[8 * l + j];
-        else rh = dequant((uint32_t)(kn >> (j * J.bk)) & ((1u << J.bk) - 1u), bs, J.mk);
-        const float2 cs = tk[k];
-        const float rc = rh * cs.x, rs = rh * cs.y;
-        const int qi = qpos(8 * l + j);
+      for (int a = 0; a < NQ; ++a) sc[a] = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        const uint32_t xa = m < 2 ? x0 : x1;
+        const uint32_t o0 = min((rotr(xa, kra[(2 * m) & 3]) & kM) | kC, kMax);
+        const uint32_t o1 = min((rotr(xa, kra[(2 * m + 1) & 3]) & kM) | kC, kMax);
+        const float2 c0 = *reinterpret_cast<const float2*>(reinterpret_cast<const uint8_t*>(tk) + o0);
+        const float2 c1 = *reinterpret_cast<const float2*>(reinterpret_cast<const uint8_t*>(tk) + o1);
+        const float2 y0 = mul2(make_float2(rh[2 * m], rh[2 * m]), c0);
+        const float2 y1 = mul2(make_float2(rh[2 * m + 1], rh[2 * m + 1]), c1);
 #pragma unroll
         for (int a = 0; a < NQ; ++a) {
-          if (a < nq) {
-            const float2 qq = qrot[a * C::QROW + qi];
-            sc[a] = __fmaf_rn(qq.x, rc, __fmaf_rn(qq.y, rs, sc[a]));
-          }
+          const float2* qa = qrot + a * C::QROW + 10 * l + 2 * m;
+          const float4 q = NQ >= 4 ? lds_f4_reload(qa) : *reinterpret_cast<const float4*>(qa);
+          sc[a] = __ffma2_rn(make_float2(q.x, q.y), y0, sc[a]);
+          sc[a] = __ffma2_rn(make_float2(q.z, q.w), y1, sc[a]);
         }
       }
-    }
 #pragma unroll
-    for (int a = 0; a < NQ; ++a) {
-      if (a < nq) {
-#pragma unroll
-        for (int off = 1; off < L; off <<= 1) sc[a] += __shfl_xor_sync(0xffffffffu, sc[a], off);
-      }
-    }
+      for (int a = 0; a < NQ; ++a) part[a] = sc[a].x + sc[a].y;
+    };
+    att_tree<L, 0, 1, NQ>(pass, l, keep);
+  };
 
-    // ---- online softmax over the step's tokens (base 2) ----
-    float pw[NQ][RW];
+  // V accumulation over the batch's valid tokens: acc += p_t y^V_t.
+  auto values = [&](const uint8_t* st, int valid, auto vc_) {
+    constexpr int VC = decltype(vc_)::value;
+    constexpr bool F32 = VC == 4, LOG = VC == 1 || VC == 3;
+    constexpr int VB = VC <= 1 ? 4 : 8;
+    constexpr uint32_t NM = ((1u << VB) - 1u) << (23 - VB);
+    const int nbit = PV * VB * lane, nwa = nbit >> 5;
+    int nra[PV];
 #pragma unroll
-    for (int a = 0; a < NQ; ++a) {
-      if (a < nq) {
-        float mx = m_run[a];
-#pragma unroll
-        for (int rr = 0; rr < RW; ++rr) {
-          float v = __shfl_sync(0xffffffffu, sc[a], rr * L);
-          if (rr >= valid) v = -INFINITY;
-          pw[a][rr] = v;
-          mx = fmaxf(mx, v);
+    for (int j = 0; j < PV; ++j) nra[j] = ((nbit & 31) + VB * j - (23 - VB)) & 31;
+#pragma unroll 4
+    for (int t = 0; t < valid; ++t) {
+      const uint32_t* arow = reinterpret_cast<const uint32_t*>(st + S_VA + t * av);
+      const uint32_t x = __funnelshift_r(arow[vwa], arow[vwa + 1], vsa);
+      const uint8_t* prow = pb + t * C::PBROW;
+      float rh[PV];
+      if constexpr (F32) {
+        const float* nr = reinterpret_cast<const float*>(st + S_VN + t * nbv) + PV * lane;
+        if constexpr (PV == 2) {
+          const float2 v = *reinterpret_cast<const float2*>(nr);
+          rh[0] = v.x; rh[1] = v.y;
+        } else {
+          rh[0] = nr[0];
         }
-        const float f = ex2_approx(m_run[a] - mx);   // m_run = -inf at first: f = 0
-        float sum = 0.f;
+      } else {
+        const float2 ab = *reinterpret_cast<const float2*>(prow);
+        const uint32_t w = reinterpret_cast<const uint32_t*>(st + S_VN + t * nbv)[nwa];
 #pragma unroll
-        for (int rr = 0; rr < RW; ++rr) {
-          pw[a][rr] = ex2_approx(pw[a][rr] - mx);
-          sum += pw[a][rr];
+        for (int j = 0; j < PV; ++j) {
+          const uint32_t fb = (rotr(w, nra[j]) & NM) | 0x3F800000u;
+          float v = __fmaf_rn(__uint_as_float(fb), ab.x, ab.y);
+          if constexpr (LOG) v = ex2_approx(v);
+          rh[j] = v;
         }
-        l_run[a] = __fmaf_rn(l_run[a], f, sum);
-        m_run[a] = mx;
-#pragma unroll
-        for (int j = 0; j < PV; ++j) { acc[a][j][0] *= f; acc[a][j][1] *= f; }
       }
-    }
-
-    // ---- V: accumulate p_t y^V_t, lane l owning pairs l + 32 j ----
+      float2 pp[NQ];
 #pragma unroll
-    for (int rr = 0; rr < RW; ++rr) {
-      if (rr >= valid) break;
-      const uint32_t* arow = reinterpret_cast<const uint32_t*>(st + C::S_VA + rr * av);
-      const uint32_t* nrow = reinterpret_cast<const uint32_t*>(st + C::S_VN + rr * nbv);
-      const float2 bs = make_float2(__shfl_sync(0xffffffffu, vbs.x, rr * L), __shfl_sync(0xffffffffu, vbs.y, rr * L));
+      for (int a = 0; a < NQ; a += 2) {
+        if (a + 1 < NQ) {
+          const float4 q = *reinterpret_cast<const float4*>(prow + 16 + 8 * a);
+          pp[a] = make_float2(q.x, q.y);
+          pp[a + 1] = make_float2(q.z, q.w);
+        } else {
+          pp[a] = *reinterpret_cast<const float2*>(prow + 16 + 8 * a);
+        }
+      }
 #pragma unroll
       for (int j = 0; j < PV; ++j) {
-        const int i = lane + 32 * j;
-        if (i < P) {
-          uint32_t k = __funnelshift_r(arow[va_w[j]], arow[va_w[j] + 1], va_s[j]) & vmask;
-          k = min(k, (uint32_t)(J.nv - 1));
-          float rh;
-          if (J.mv == TAC_NORM_FP32) rh = __uint_as_float(nrow[i]);
-          else rh = dequant((nrow[vn_w[j]] >> vn_s[j]) & nvmask, bs, J.mv);
-          const float2 cs = tv[k];
-          const float yc = rh * cs.x, ys = rh * cs.y;
+        const uint32_t o = min((rotr(x, vra[j]) & vM) | vC, vMax);
+        const float2 cs = *reinterpret_cast<const float2*>(reinterpret_cast<const uint8_t*>(tv) + o);
+        const float2 y = mul2(make_float2(rh[j], rh[j]), cs);
 #pragma unroll
-          for (int a = 0; a < NQ; ++a) {
-            if (a < nq) {
-              acc[a][j][0] = __fmaf_rn(pw[a][rr], yc, acc[a][j][0]);
-              acc[a][j][1] = __fmaf_rn(pw[a][rr], ys, acc[a][j][1]);
-            }
-          }
-        }
+        for (int a = 0; a < NQ; ++a) acc[a][j] = __ffma2_rn(pp[a], y, acc[a][j]);
       }
     }
+  };
+
+  issue(0);
+  for (int s = 0; s < nb; ++s) {
+    issue(s + 1);
+    cp_async_wait<1>();
+    __syncwarp();
+    const uint8_t* st = stg + (s % kAttNS) * stage;
+    const int valid = (int)min((int64_t)kAttBatch, t_stop - (t_begin + (int64_t)s * kAttBatch));
+
+    float keep[NQ];
+    switch (J.ck) {
+      case 0: scores(st, keep, IC<0>{}); break;
+      case 1: scores(st, keep, IC<1>{}); break;
+      case 2: scores(st, keep, IC<2>{}); break;
+      case 3: scores(st, keep, IC<3>{}); break;
+      default: scores(st, keep, IC<4>{}); break;
+    }
+
+    // ---- online softmax (base 2); lane (r, l) owns token t = RW l + r ----
+    const int t = RW * l + r;
+    const bool live = t < valid;
+    uint8_t* prow = pb + t * C::PBROW;
+    float pw[NQ];
+#pragma unroll
+    for (int a = 0; a < NQ; ++a) {
+      const float sa = live ? keep[a] : -INFINITY;
+      float mx = sa;
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      const float mn = fmaxf(m_run[a], mx);
+      const float f = ex2_approx(m_run[a] - mn);   // m_run = -inf at first: f = 0
+      pw[a] = ex2_approx(sa - mn);
+      l_run[a] = __fmaf_rn(l_run[a], f, pw[a]);
+      m_run[a] = mn;
+#pragma unroll
+      for (int j = 0; j < PV; ++j) acc[a][j] = mul2(acc[a][j], make_float2(f, f));
+    }
+    if (live && J.mv != TAC_NORM_FP32)
+      *reinterpret_cast<float2*>(prow) = norm_ab(*reinterpret_cast<const float2*>(st + S_VH + t * 8), vinv, v2b, vlog);
+#pragma unroll
+    for (int a = 0; a < NQ; a += 2) {
+      if (a + 1 < NQ) *reinterpret_cast<float4*>(prow + 16 + 8 * a) = make_float4(pw[a], pw[a], pw[a + 1], pw[a + 1]);
+      else *reinterpret_cast<float2*>(prow + 16 + 8 * a) = make_float2(pw[a], pw[a]);
+    }
+    __syncwarp();
+
+    switch (J.cv) {
+      case 0: values(st, valid, IC<0>{}); break;
+      case 1: values(st, valid, IC<1>{}); break;
+      case 2: values(st, valid, IC<2>{}); break;
+      case 3: values(st, valid, IC<3>{}); break;
+      default: values(st, valid, IC<4>{}); break;
+    }
+    __syncwarp();
   }
   cp_async_wait<0>();
 
-  // ---- write the split's partial results ----
+  // ---- the split's partial results: (max, sum, accumulator) per query ----
   float* rec = ws + J.ws + (int64_t)(split - J.split0) * nq * att_rec_floats(D);
 #pragma unroll
   for (int a = 0; a < NQ; ++a) {
+    float ls = l_run[a];
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) ls += __shfl_xor_sync(0xffffffffu, ls, o);
     if (a < nq) {
       float* ra = rec + a * att_rec_floats(D);
-      if (lane == 0) { ra[0] = m_run[a]; ra[1] = l_run[a]; }
+      if (lane == 0) { ra[0] = m_run[a]; ra[1] = ls; }
 #pragma unroll
-      for (int j = 0; j < PV; ++j) {
-        const int i = lane + 32 * j;
-        if (i < P) *reinterpret_cast<float2*>(ra + 2 + 2 * i) = make_float2(acc[a][j][0], acc[a][j][1]);
-      }
+      for (int j = 0; j < PV; ++j) *reinterpret_cast<float2*>(ra + 2 + 2 * (PV * lane + j)) = acc[a][j];
     }
   }
 }
@@ -383,17 +493,24 @@ __global__ void __launch_bounds__(128) attend_combine(const __grid_constant__ At
 
 template <int D, typename TQ, int NQ>
 static cudaError_t launch_attend_t(const AttParams& p, int nrows_total, float* ws, cudaStream_t st) {
-  using C = Att<D>;
-  auto kp = attend_partial<D, TQ, NQ>;
+  using C = Att<D, NQ>;
+  auto kp = attend_partial<D, NQ>;
   static int configured[64] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    // the largest batch stage: 8-bit codes and fp32 norms for K and V
+    const int smax = C::smem(att_stage_bytes(D, 8, 32, TAC_NORM_FP32, 8, 32, TAC_NORM_FP32));
+    cudaError_t e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize, smax);
     if (e != cudaSuccess) return e;
     configured[dev] = 1;
   }
-  if (p.nctas > 0) kp<<<p.nctas, kAttThreads, C::SMEM, st>>>(p, ws);
+  int stage = 0;
+  for (int j = 0; j < p.njobs; ++j) {
+    const AttJob& J = p.job[j];
+    stage = std::max(stage, att_stage_bytes(D, J.wk, J.bk, J.mk, J.wv, J.bv, J.mv));
+  }
+  if (p.nctas > 0) kp<<<p.nctas, kAttThreads, C::smem(stage), st>>>(p, ws);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int blocks = (nrows_total + 3) / 4;

@@ -100,3 +100,30 @@ def test_attend_codebook_mix_and_many_jobs(tac_gpu, orc):
         dict(d=64, T=5, nq=1, k=(2, 8, 0), v=(4, 4, 0), seed=5),
     ]
     _check(orc, tac_gpu, spec)
+
+
+def test_attend_prepared_call_matches_direct(tac_gpu):
+    """attend_multi_prepared (job array marshalled once, called twice) gives the
+    bits of attend_multi."""
+    import torch
+    tac = tac_gpu
+    w = workloads.CONFIGS["mistral7b"]
+    jobs = []
+    for seed, T in ((7, 777), (8, 33)):
+        xk = workloads.block(w, 1, 0, tokens=T, seed=seed, device="cuda")[:T].contiguous()
+        xv = workloads.block(w, 1, 1, tokens=T, seed=seed, device="cuda")[:T].contiguous()
+        kcfg, kcache = _cache(tac, xk, 128, 128, 8, 0, 1, 0)
+        vcfg, vcache = _cache(tac, xv, 128, 64, 4, 1, 1, 1)
+        q = torch.randn((4, 128), device="cuda").to(torch.bfloat16)
+        jobs.append(tac.AttendJob(kcfg, kcache, vcfg, vcache, T, q, torch.empty_like(q), 0.088))
+    tac.attend_multi(jobs)
+    torch.cuda.synchronize()
+    want = [j.out.clone() for j in jobs]
+    call = tac.attend_multi_prepared(jobs)
+    for _ in range(2):
+        for j in jobs:
+            j.out.zero_()
+        call()
+        torch.cuda.synchronize()
+        for j, ref in zip(jobs, want):
+            assert torch.equal(j.out, ref)
