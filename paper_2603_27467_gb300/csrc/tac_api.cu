@@ -508,13 +508,12 @@ int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st
       i = next(0);
       while (i < njobs) {
         std::memset(&P, 0, sizeof(P));
-        int64_t ctas = 0, splits = 0;
+        int64_t splits = 0;
         int nrows = 0, nq_max = 1;
         while (i < njobs && P.njobs < TAC_MAX_JOBS) {
           const tac_attend_job& J = jobs[i];
           const int64_t ns = (J.tokens + TAC_ATTEND_SPLIT - 1) / TAC_ATTEND_SPLIT;
-          const int64_t nc = (ns + 3) / 4;
-          if (ctas + nc > 0x7fffffff || splits + ns > 0x7fffffff) break;
+          if (splits + ns > 0x7fffffff) break;   // CTAs (<= splits) are assigned at launch
           tac::AttJob& A = P.job[P.njobs];
           A.kc = static_cast<const uint8_t*>(J.k_codes);
           A.kn = static_cast<const uint8_t*>(J.k_norms);
@@ -533,25 +532,22 @@ int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st
           A.nv = J.cfg_v.n_angle; A.wv = tac::code_bits(J.cfg_v.n_angle); A.bv = J.cfg_v.norm_bits; A.mv = J.cfg_v.norm_mode;
           A.inv_lk = A.mk == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bk) - 1);
           A.inv_lv = A.mv == TAC_NORM_FP32 ? 0.f : 1.f / (float)((1 << A.bv) - 1);
-          A.lgrk = tac::att_table_lgr(A.nk);
-          A.lgrv = tac::att_table_lgr(A.nv);
+          A.lgrk = tac::att_table_lgr(1 << A.wk);
+          A.lgrv = tac::att_table_lgr(1 << A.wv);
           A.ck = tac::att_norm_case(A.bk, A.mk);
           A.cv = tac::att_norm_case(A.bv, A.mv);
           copy_signs(A.sk, &J.cfg_k);
           copy_signs(A.sv, &J.cfg_v);
           A.split0 = (int32_t)splits;
-          A.cta0 = (int32_t)ctas;
           A.ws = ws_off;
           ws_off += attend_ws_floats(J);
           splits += ns;
-          ctas += nc;
           nrows += A.nq;
           nq_max = std::max(nq_max, (int)A.nq);
           ++P.njobs;
           i = next(i + 1);
         }
         if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many tokens", who);
-        P.nctas = (int32_t)ctas;
         P.nsplits = (int32_t)splits;
         P.q_bf16 = dt == TAC_BF16;
         cudaError_t e = tac::launch_attend(d, dt, nq_max, P, nrows, ws, st);

@@ -34,8 +34,7 @@ namespace tac {
 template <int V>
 struct IC { static constexpr int value = V; };
 
-constexpr int kAttWarps = 4;                  // warps (splits) per CTA
-constexpr int kAttThreads = 32 * kAttWarps;
+constexpr int kAttMaxWarps = 6;               // warps (splits) per CTA: 1..6, chosen per launch
 constexpr int kAttSplit = TAC_ATTEND_SPLIT;   // tokens per split (one warp)
 constexpr int kAttNS = 2;                     // staged batches per warp
 constexpr float kLog2e = 1.4426950408889634f;
@@ -54,7 +53,7 @@ struct Att {
   static constexpr int OFF_TK = OFF_Q + NQ * QROW * 8;
   static constexpr int OFF_TV = OFF_TK + kAttTabBytes;
   static constexpr int OFF_W = OFF_TV + kAttTabBytes;
-  static constexpr int smem(int stage) { return OFF_W + kAttWarps * (PB + kAttNS * stage); }
+  static constexpr int smem(int stage, int warps) { return OFF_W + warps * (PB + kAttNS * stage); }
   static_assert(OFF_TK % 16 == 0 && PB % 16 == 0 && P % 32 == 0, "layout");
 };
 
@@ -76,13 +75,13 @@ __device__ __forceinline__ float4 lds_f4_reload(const void* ptr) {
 // Reduce-scatter over the L lanes of a token, as a tree over the passes: the
 // lane's value for the pass set {I + k S} is its half, selected by lane bit S,
 // of the two sets {I + 2kS} and {I + S + 2kS}, plus the partner's.  At the
-// top (I = 0, S = 1) lane l holds the sum over the L lanes of pass l.
+// top (I = 0, S = 1) lane l holds the sum over the L lanes of pass l.  The
+// two passes of a base set {I, I + L/2} are computed together (one call).
 template <int L, int I, int S, int NQ, typename PF>
 __device__ __forceinline__ void att_tree(PF& pass, int l, float (&v)[NQ]) {
   float va[NQ], vb[NQ];
   if constexpr (2 * S == L) {
-    pass(IC<I>{}, va);
-    pass(IC<I + S>{}, vb);
+    pass(IC<I>{}, IC<I + S>{}, va, vb);
   } else {
     att_tree<L, I, 2 * S, NQ>(pass, l, va);
     att_tree<L, I + S, 2 * S, NQ>(pass, l, vb);
@@ -126,11 +125,12 @@ __device__ __forceinline__ void smem_fwht(float* buf, int rows, int tid, int nth
 }
 
 template <int D, int NQ>
-__global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(const __grid_constant__ AttParams p, float* ws) {
+__global__ void __launch_bounds__(32 * kAttMaxWarps, NQ <= 4 ? 2 : 1) attend_partial(const __grid_constant__ AttParams p, float* ws) {
   using C = Att<D, NQ>;
   constexpr int P = C::P, L = C::L, RW = C::RW, PV = C::PV;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nthr = blockDim.x, wpc = nthr >> 5;
 
   // ---- the CTA's job ----
   int jb = 0;
@@ -154,7 +154,7 @@ __global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(c
 
   // ---- rotated queries q' = H D_K q * scale * log2(e), skewed float2 rows ----
   float* qbuf = reinterpret_cast<float*>(smem + C::OFF_W);   // staging, reused by the batches below
-  for (int e = tid; e < nq * D; e += kAttThreads) {
+  for (int e = tid; e < nq * D; e += nthr) {
     const int a = e / D, j = e % D;
     float x;
     if (p.q_bf16) {
@@ -164,24 +164,25 @@ __global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(c
     }
     qbuf[e] = ((J.sk[j >> 5] >> (j & 31)) & 1u) ? -x : x;
   }
-  smem_fwht<D>(qbuf, nq, tid, kAttThreads, true);
+  smem_fwht<D>(qbuf, nq, tid, nthr, true);
   float2* qrot = reinterpret_cast<float2*>(smem + C::OFF_Q);
   const float qs = J.scale * kLog2e * rsqrtf((float)D);
-  for (int e = tid; e < NQ * P; e += kAttThreads) {
+  for (int e = tid; e < NQ * P; e += nthr) {
     const int a = e / P, i = e % P;
     qrot[a * C::QROW + qpos(i)] =
         a < nq ? make_float2(qbuf[a * D + 2 * i] * qs, qbuf[a * D + 2 * i + 1] * qs) : make_float2(0.f, 0.f);
   }
-  // ---- bin-centre tables (cos, sin)(2 pi k / n), 2^lgr copies: entry k copy c at k 2^lgr + c ----
+  // ---- bin-centre tables (cos, sin)(2 pi k / n), 2^lgr copies: entry k copy c
+  // at k 2^lgr + c; entries n..2^W-1 repeat entry n-1 (codes >= n clamp) ----
   const int lgrk = J.lgrk, lgrv = J.lgrv;
   float2* tk = reinterpret_cast<float2*>(smem + C::OFF_TK);
   float2* tv = reinterpret_cast<float2*>(smem + C::OFF_TV);
-  for (int e = tid; e < (J.nk << lgrk); e += kAttThreads) tk[e] = cos_sin_q8(8 * (e >> lgrk), J.nk);
-  for (int e = tid; e < (J.nv << lgrv); e += kAttThreads) tv[e] = cos_sin_q8(8 * (e >> lgrv), J.nv);
+  for (int e = tid; e < (1 << (J.wk + lgrk)); e += nthr) tk[e] = cos_sin_q8(8 * min(e >> lgrk, J.nk - 1), J.nk);
+  for (int e = tid; e < (1 << (J.wv + lgrv)); e += nthr) tv[e] = cos_sin_q8(8 * min(e >> lgrv, J.nv - 1), J.nv);
   __syncthreads();
 
   // ---- this warp's split ----
-  const int split = J.split0 + ((int)blockIdx.x - J.cta0) * kAttWarps + warp;
+  const int split = J.split0 + ((int)blockIdx.x - J.cta0) * wpc + warp;
   const int64_t t_begin = (int64_t)(split - J.split0) * kAttSplit;
   if (t_begin >= J.tokens) return;
   const int64_t t_stop = min(J.tokens, t_begin + kAttSplit);
@@ -224,7 +225,6 @@ __global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(c
   const int ksb = (ksa + 4 * wk) & 31;
   const uint32_t kC = (uint32_t)(lane & ((1 << lgrk) - 1)) << 3;
   const uint32_t kM = ((1u << wk) - 1u) << Tk;
-  const uint32_t kMax = ((uint32_t)(J.nk - 1) << Tk) | kC;   // clamps codes >= n (n not a power of two)
   int kra[4];
 #pragma unroll
   for (int j = 0; j < 4; ++j) kra[j] = (wk * j - Tk) & 31;
@@ -233,7 +233,6 @@ __global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(c
   const int vbit = PV * wv * lane, vwa = vbit >> 5, vsa = vbit & 31;
   const uint32_t vC = (uint32_t)(lane & ((1 << lgrv) - 1)) << 3;
   const uint32_t vM = ((1u << wv) - 1u) << Tv;
-  const uint32_t vMax = ((uint32_t)(J.nv - 1) << Tv) | vC;
   int vra[PV];
 #pragma unroll
   for (int j = 0; j < PV; ++j) vra[j] = (wv * j - Tv) & 31;
@@ -257,13 +256,12 @@ __global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(c
     constexpr int KC = decltype(kc_)::value;
     constexpr bool F32 = KC == 4, LOG = KC == 1 || KC == 3;
     constexpr int KB = KC <= 1 ? 4 : 8;
-    auto pass = [&](auto k_, float (&part)[NQ]) {
-      const int row = decltype(k_)::value * RW + r;
+    // Decoded norms r^ and packed angle codes of this lane's 8 pairs of one token.
+    auto load_row = [&](int row, uint32_t& x0, uint32_t& x1, float (&rh)[8]) {
       const uint32_t* arow = reinterpret_cast<const uint32_t*>(st + row * ak);
       const uint32_t w0 = arow[kwa], w1 = arow[kwa + 1], w2 = arow[kwa + 2];
-      const uint32_t x0 = __funnelshift_r(w0, w1, ksa);
-      const uint32_t x1 = kup ? __funnelshift_r(w1, w2, ksb) : __funnelshift_r(w0, w1, ksb);
-      float rh[8];
+      x0 = __funnelshift_r(w0, w1, ksa);
+      x1 = kup ? __funnelshift_r(w1, w2, ksb) : __funnelshift_r(w0, w1, ksb);
       if constexpr (F32) {
         const float4* nr = reinterpret_cast<const float4*>(st + S_KN + row * nbk + 32 * l);
         const float4 n0 = nr[0], n1 = nr[1];
@@ -288,28 +286,43 @@ __global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(c
           rh[j] = v;
         }
       }
-      float2 sc[NQ];
+    };
+    auto ydec = [&](uint32_t x, int j, float rh) {
+      const uint32_t o = (rotr(x, kra[j & 3]) & kM) | kC;
+      const float2 c = *reinterpret_cast<const float2*>(reinterpret_cast<const uint8_t*>(tk) + o);
+      return mul2(make_float2(rh, rh), c);
+    };
+    // Partial scores of tokens kA RW + r and kB RW + r over this lane's pairs;
+    // each rotated-query granule is loaded once for both.
+    auto pass = [&](auto ka_, auto kb_, float (&pa)[NQ], float (&pb)[NQ]) {
+      uint32_t xa0, xa1, xb0, xb1;
+      float ra[8], rb[8];
+      load_row(decltype(ka_)::value * RW + r, xa0, xa1, ra);
+      load_row(decltype(kb_)::value * RW + r, xb0, xb1, rb);
+      float2 sa[NQ], sb[NQ];
 #pragma unroll
-      for (int a = 0; a < NQ; ++a) sc[a] = make_float2(0.f, 0.f);
+      for (int a = 0; a < NQ; ++a) sa[a] = sb[a] = make_float2(0.f, 0.f);
 #pragma unroll
       for (int m = 0; m < 4; ++m) {
-        const uint32_t xa = m < 2 ? x0 : x1;
-        const uint32_t o0 = min((rotr(xa, kra[(2 * m) & 3]) & kM) | kC, kMax);
-        const uint32_t o1 = min((rotr(xa, kra[(2 * m + 1) & 3]) & kM) | kC, kMax);
-        const float2 c0 = *reinterpret_cast<const float2*>(reinterpret_cast<const uint8_t*>(tk) + o0);
-        const float2 c1 = *reinterpret_cast<const float2*>(reinterpret_cast<const uint8_t*>(tk) + o1);
-        const float2 y0 = mul2(make_float2(rh[2 * m], rh[2 * m]), c0);
-        const float2 y1 = mul2(make_float2(rh[2 * m + 1], rh[2 * m + 1]), c1);
+        const float2 ya0 = ydec(m < 2 ? xa0 : xa1, 2 * m, ra[2 * m]);
+        const float2 ya1 = ydec(m < 2 ? xa0 : xa1, 2 * m + 1, ra[2 * m + 1]);
+        const float2 yb0 = ydec(m < 2 ? xb0 : xb1, 2 * m, rb[2 * m]);
+        const float2 yb1 = ydec(m < 2 ? xb0 : xb1, 2 * m + 1, rb[2 * m + 1]);
 #pragma unroll
         for (int a = 0; a < NQ; ++a) {
           const float2* qa = qrot + a * C::QROW + 10 * l + 2 * m;
           const float4 q = NQ >= 4 ? lds_f4_reload(qa) : *reinterpret_cast<const float4*>(qa);
-          sc[a] = __ffma2_rn(make_float2(q.x, q.y), y0, sc[a]);
-          sc[a] = __ffma2_rn(make_float2(q.z, q.w), y1, sc[a]);
+          sa[a] = __ffma2_rn(make_float2(q.x, q.y), ya0, sa[a]);
+          sa[a] = __ffma2_rn(make_float2(q.z, q.w), ya1, sa[a]);
+          sb[a] = __ffma2_rn(make_float2(q.x, q.y), yb0, sb[a]);
+          sb[a] = __ffma2_rn(make_float2(q.z, q.w), yb1, sb[a]);
         }
       }
 #pragma unroll
-      for (int a = 0; a < NQ; ++a) part[a] = sc[a].x + sc[a].y;
+      for (int a = 0; a < NQ; ++a) {
+        pa[a] = sa[a].x + sa[a].y;
+        pb[a] = sb[a].x + sb[a].y;
+      }
     };
     att_tree<L, 0, 1, NQ>(pass, l, keep);
   };
@@ -362,7 +375,7 @@ __global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(c
       }
 #pragma unroll
       for (int j = 0; j < PV; ++j) {
-        const uint32_t o = min((rotr(x, vra[j]) & vM) | vC, vMax);
+        const uint32_t o = (rotr(x, vra[j]) & vM) | vC;
         const float2 cs = *reinterpret_cast<const float2*>(reinterpret_cast<const uint8_t*>(tv) + o);
         const float2 y = mul2(make_float2(rh[j], rh[j]), cs);
 #pragma unroll
@@ -443,14 +456,18 @@ __global__ void __launch_bounds__(kAttThreads, NQ <= 4 ? 3 : 2) attend_partial(c
   }
 }
 
-// One warp per (job, query): merge the splits, normalize, out = D_V H y.
+// One CTA of 4 warps per (job, query): warp w merges splits w, w + 4, ...
+// against the row's overall max, the warps' sums are added in shared memory,
+// and warp 0 normalizes, applies D H (fp32 butterfly) and stores the row.
 template <int D, typename TO>
 __global__ void __launch_bounds__(128) attend_combine(const __grid_constant__ AttParams p, const float* ws,
                                                       int nrows_total) {
   constexpr int ESZ = (int)sizeof(TO);
-  __shared__ float buf[4][D];
+  constexpr int E = D / 32;
+  __shared__ float part[4][D];
+  __shared__ float red[4][2];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int g = blockIdx.x * 4 + warp;           // global (job, query) index
+  const int g = blockIdx.x;                      // global (job, query) index
   if (g >= nrows_total) return;
   int jb = 0, base = 0;
   for (; jb < p.njobs; ++jb) {
@@ -460,29 +477,44 @@ __global__ void __launch_bounds__(128) attend_combine(const __grid_constant__ At
   const AttJob& J = p.job[jb];
   const int a = g - base;
   const int nsp = (int)((J.tokens + kAttSplit - 1) / kAttSplit);
-  const float* recs = ws + J.ws;
+  const float* recs = ws + J.ws + (int64_t)a * att_rec_floats(D);
+  const int64_t stride = (int64_t)J.nq * att_rec_floats(D);   // between splits
   float M = -INFINITY;
-  for (int s = 0; s < nsp; ++s) M = fmaxf(M, recs[((int64_t)s * J.nq + a) * att_rec_floats(D)]);
-  float Lsum = 0.f;
-  float y[D / 32];
+  for (int s = threadIdx.x; s < nsp; s += 128) M = fmaxf(M, recs[s * stride]);
 #pragma unroll
-  for (int e = 0; e < D / 32; ++e) y[e] = 0.f;
-  for (int s = 0; s < nsp; ++s) {
-    const float* ra = recs + ((int64_t)s * J.nq + a) * att_rec_floats(D);
+  for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  if (lane == 0) red[warp][0] = M;
+  __syncthreads();
+  M = fmaxf(fmaxf(red[0][0], red[1][0]), fmaxf(red[2][0], red[3][0]));
+  float Ls = 0.f;
+  float y[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) y[e] = 0.f;
+#pragma unroll 4
+  for (int s = warp; s < nsp; s += 4) {
+    const float* ra = recs + s * stride;
     const float f = ex2_approx(ra[0] - M);
-    Lsum = __fmaf_rn(ra[1], f, Lsum);
+    Ls = __fmaf_rn(ra[1], f, Ls);
 #pragma unroll
-    for (int e = 0; e < D / 32; ++e) y[e] = __fmaf_rn(ra[2 + lane + 32 * e], f, y[e]);
+    for (int e = 0; e < E; ++e) y[e] = __fmaf_rn(ra[2 + lane + 32 * e], f, y[e]);
   }
-  const float inv = 1.f / Lsum;
-  float* row = buf[warp];
 #pragma unroll
-  for (int e = 0; e < D / 32; ++e) row[lane + 32 * e] = y[e] * inv;
+  for (int e = 0; e < E; ++e) part[warp][lane + 32 * e] = y[e];
+  if (lane == 0) red[warp][1] = Ls;
+  __syncthreads();
+  if (warp != 0) return;
+  const float inv = 1.f / (red[0][1] + red[1][1] + red[2][1] + red[3][1]);
+  float* row = part[0];
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int j = lane + 32 * e;
+    row[j] = (part[0][j] + part[1][j] + part[2][j] + part[3][j]) * inv;
+  }
   smem_fwht<D>(row, 1, lane, 32, false);
   const float sc = rsqrtf((float)D);
   uint8_t* orow = reinterpret_cast<uint8_t*>(J.out) + (int64_t)a * J.out_stride * ESZ;
 #pragma unroll
-  for (int e = 0; e < D / 32; ++e) {
+  for (int e = 0; e < E; ++e) {
     const int j = lane + 32 * e;
     float v = row[j] * sc;
     if ((J.sv[j >> 5] >> (j & 31)) & 1u) v = -v;
@@ -491,30 +523,64 @@ __global__ void __launch_bounds__(128) attend_combine(const __grid_constant__ At
   }
 }
 
+// Warps per CTA for a launch: the count (1..kAttMaxWarps) that keeps the most
+// warps resident per SM, given the CTA's shared memory (which grows with the
+// warps) and the kernel's registers; ties go to more warps per CTA.
+static int att_warps_per_cta(int smem_fixed, int smem_per_warp, int regs) {
+  constexpr int kSmemSM = 228 * 1024, kSmemCTA = 227 * 1024, kReserved = 1024;
+  const int regs_warp = ((regs * 32 + 255) / 256) * 256;
+  int best = 1, best_res = -1;
+  for (int w = 1; w <= kAttMaxWarps; ++w) {
+    const int sm = smem_fixed + w * smem_per_warp;
+    if (sm > kSmemCTA) break;
+    const int by_smem = kSmemSM / (sm + kReserved);
+    const int by_regs = 65536 / (regs_warp * w);
+    const int by_warps = 64 / w;
+    const int res = std::min(by_smem, std::min(by_regs, by_warps)) * w;
+    if (res >= best_res) { best_res = res; best = w; }
+  }
+  return best;
+}
+
+// Launches the partial and combine kernels for one group of jobs.  The CTA
+// assignment (cta0 per job, nctas) is made here, after the warps per CTA.
 template <int D, typename TQ, int NQ>
-static cudaError_t launch_attend_t(const AttParams& p, int nrows_total, float* ws, cudaStream_t st) {
+static cudaError_t launch_attend_t(const AttParams& p_in, int nrows_total, float* ws, cudaStream_t st) {
   using C = Att<D, NQ>;
   auto kp = attend_partial<D, NQ>;
   static int configured[64] = {0};
+  static int regs[64] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
-  if (dev >= 0 && dev < 64 && !configured[dev]) {
-    // the largest batch stage: 8-bit codes and fp32 norms for K and V
-    const int smax = C::smem(att_stage_bytes(D, 8, 32, TAC_NORM_FP32, 8, 32, TAC_NORM_FP32));
-    cudaError_t e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize, smax);
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     if (e != cudaSuccess) return e;
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, kp);
+    if (e != cudaSuccess) return e;
+    regs[dev] = fa.numRegs;
     configured[dev] = 1;
   }
+  AttParams p = p_in;
   int stage = 0;
   for (int j = 0; j < p.njobs; ++j) {
     const AttJob& J = p.job[j];
     stage = std::max(stage, att_stage_bytes(D, J.wk, J.bk, J.mk, J.wv, J.bv, J.mv));
   }
-  if (p.nctas > 0) kp<<<p.nctas, kAttThreads, C::smem(stage), st>>>(p, ws);
+  const int wpc = att_warps_per_cta(C::smem(stage, 0), C::smem(stage, 1) - C::smem(stage, 0), regs[dev]);
+  int64_t ctas = 0;
+  for (int j = 0; j < p.njobs; ++j) {
+    AttJob& J = p.job[j];
+    const int64_t ns = (J.tokens + kAttSplit - 1) / kAttSplit;
+    J.cta0 = (int32_t)ctas;
+    ctas += (ns + wpc - 1) / wpc;
+  }
+  p.nctas = (int32_t)ctas;
+  if (p.nctas > 0) kp<<<p.nctas, 32 * wpc, C::smem(stage, wpc), st>>>(p, ws);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const int blocks = (nrows_total + 3) / 4;
-  if (blocks > 0) attend_combine<D, TQ><<<blocks, 128, 0, st>>>(p, ws, nrows_total);
+  if (nrows_total > 0) attend_combine<D, TQ><<<nrows_total, 128, 0, st>>>(p, ws, nrows_total);
   return cudaGetLastError();
 }
 
