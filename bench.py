@@ -39,10 +39,12 @@ FALLBACK_HBM_GBS = 6800.0
 # so its traffic is this figure times its rows).  Each figure holds only for the
 # kernel sources it was measured on; after any change to them it reads null.
 MEASURED_TRAFFIC = {
-    "encode": {"sources": ("tac_common.cuh", "tac_encode.cu"), "sha256_16": "73575d5810d8d294",
-               "bytes_per_row": 349.596},
-    "decode": {"sources": ("tac_common.cuh", "tac_decode.cu"), "sha256_16": "94a05f1c3d5736cb",
-               "bytes_per_row": 334.232},
+    "encode": {"sources": ("tac_common.cuh", "tac_encode.cu"), "sha256_16": "3069af8194be1e5e",
+               "bytes_per_row": 318.974},
+    "decode": {"sources": ("tac_common.cuh", "tac_decode.cu"), "sha256_16": "3708cb9c8bda0ef3",
+               "bytes_per_row": 275.051},
+    "attend": {"sources": ("tac_common.cuh", "tac_attend.cuh", "tac_attend.cu"), "sha256_16": "b9b7bb097c305745",
+               "bytes_per_row": 228.550},
 }
 
 
@@ -472,7 +474,10 @@ def run_attend(args):
                    "record_bytes_per_step": rec_bytes},
         "token_heads_per_s": w.layers * w.heads * T / (ms / 1e3),
         "roofline": {"bound": "hbm", "kernel": "attend_partial + attend_combine", "achieved": gbs, "peak": hbm,
-                     "unit": "GB/s", "frac": gbs / hbm, "peak_source": f"{peak_kind} hbm_gbs", "traffic": None},
+                     "unit": "GB/s", "frac": gbs / hbm, "peak_source": f"{peak_kind} hbm_gbs",
+                     "traffic": measured_traffic("attend", w.layers * w.heads * T),
+                     "traffic_note": "attend_partial DRAM bytes per token-head from ncu at 4096 tokens, "
+                                     "scaled by token-heads; null once the kernel source changes"},
         "gpu_launches": 2 * args.steps * (1 + (len(jobs) - 1) // 96), "clocks": clocks}), flush=True)
 
 

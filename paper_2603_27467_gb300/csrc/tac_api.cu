@@ -9,7 +9,7 @@
 #include <string>
 #include <vector>
 
-#include "tac_common.cuh"
+#include "tac_attend.cuh"
 
 namespace tac {
 cudaError_t launch_encode_16_bf16(const EncParams& p, int n, int b, int mode, int sms,

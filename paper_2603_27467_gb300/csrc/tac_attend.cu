@@ -27,7 +27,7 @@
 #include <algorithm>
 #include <atomic>
 
-#include "tac_common.cuh"
+#include "tac_attend.cuh"
 
 namespace tac {
 
