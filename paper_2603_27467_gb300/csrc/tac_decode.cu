@@ -24,6 +24,22 @@ namespace tac {
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles of records in flight
 
+// Copies of an n-entry table of esz-byte entries within `budget` bytes (at most maxr).
+__host__ __device__ constexpr int tab_copies_e(int n, int budget, int esz, int maxr) {
+  int r = maxr;
+  while (r > 1 && n * r * esz > budget) r >>= 1;
+  return r;
+}
+
+// Centre-table entries: fp32 pairs for fp32 output; for bf16 output, fp16
+// pairs (relative error 2^-11 per entry, an output error below 2^-11 |x^|,
+// within the bf16 output tolerance) so a warp's lookups take one shared
+// wavefront with one table copy per lane.
+template <int ESZ> struct CentreT { using T = float2; };
+template <> struct CentreT<2> { using T = __half2; };
+__device__ __forceinline__ float2 centre(float2 t) { return t; }
+__device__ __forceinline__ float2 centre(__half2 t) { return __half22float2(t); }
+
 // Shape of one kernel: n bins (W = ceil(log2 n) bits per code), B norm bits
 // (4, 8, or 32 for fp32 norms), MODE; HB header bytes per row (none for fp32).
 template <int D, typename TOut, int N, int B, int MODE>
@@ -48,9 +64,11 @@ struct Dec {
   static constexpr int W_REC = 0;                           // kNS record stages
   static constexpr int W_TP = W_REC + kNS * REC_W;          // transpose rows
   static constexpr int WARP_B = W_TP + G::TP_W;
-  static constexpr int TABR = tab_copies(n, 16384);          // centre table copies
+  using TabT = typename CentreT<ESZ>::T;
+  static constexpr int TAB_E = (int)sizeof(TabT);
+  static constexpr int TABR = tab_copies_e(n, 16384, TAB_E, ESZ == 2 ? 32 : 16);   // centre table copies
   static constexpr int OFF_TAB = kWarps * WARP_B;           // centre table of this n (TABR copies)
-  static constexpr int SMEM = OFF_TAB + n * TABR * 8;
+  static constexpr int SMEM = OFF_TAB + n * TABR * TAB_E;
   static_assert(REC_W % 16 == 0 && W_TP % 16 == 0 && WARP_B % 16 == 0, "alignment");
 };
 
@@ -128,7 +146,8 @@ __device__ __forceinline__ uint64_t load_bytes(const uint8_t* p) {
 // lane's copy of the replicated centre table; orow: the lane's first output
 // pair, element 2l of its row; live: the row exists).
 template <int D, typename TOut, int N, int B, int MODE>
-__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab, int lane,
+__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm,
+                                            const typename Dec<D, TOut, N, B, MODE>::TabT* ttab, int lane,
                                             const uint2 (&msk)[8], uint8_t* orow, bool live) {
   using C = Dec<D, TOut, N, B, MODE>;
   using G = Geo<D>;
@@ -151,7 +170,7 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
     const float4 a = rp[0], b = rp[1];
     const float rr[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
 #pragma unroll
-    for (int j = 0; j < 8; ++j) v[j] = mul2(make_float2(rr[j], rr[j]), ttab[code(j) * C::TABR]);
+    for (int j = 0; j < 8; ++j) v[j] = mul2(make_float2(rr[j], rr[j]), centre(ttab[code(j) * C::TABR]));
   } else {
   constexpr int Lq = (1 << B) - 1;
   const uint64_t acc_n = load_bytes<B>(rec + C::R_NRM + r * NB + l * B);
@@ -180,7 +199,7 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
     const float f = __uint_as_float(0x3F800000u | (cb << (23 - B)));
     float rh = __fmaf_rn(f, S, base2);
     if constexpr (MODE != TAC_NORM_LINEAR) rh = ex2_ftz(rh);
-    v[j] = mul2(make_float2(rh, rh), ttab[code(j) * C::TABR]);
+    v[j] = mul2(make_float2(rh, rh), centre(ttab[code(j) * C::TABR]));
   }
   }
   // Butterfly stages on pair-index bits 0..2 (this lane holds pairs 8l..8l+7).
@@ -223,12 +242,16 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
   const int warp = tid >> 5, lane = tid & 31;
 
   // Centre table of this n: (cos + sin, cos - sin)(2 pi k / n) / sqrt(d).
-  float2* ttab = reinterpret_cast<float2*>(smem + C::OFF_TAB);
+  using TabT = typename C::TabT;
+  TabT* ttab = reinterpret_cast<TabT*>(smem + C::OFF_TAB);
   const float sc = sqrtf(2.f / (float)D);  // sqrt2 / sqrt(d)
   for (int k = tid; k < C::n; k += kThreads) {
     const float2 cs = cos_sin_q8(centre_q8(k, C::n), C::n);  // (cos psi, sin psi), psi = phi + pi/4
+    TabT e;
+    if constexpr (C::ESZ == 2) e = __floats2half2_rn(sc * cs.y, sc * cs.x);
+    else e = make_float2(sc * cs.y, sc * cs.x);
 #pragma unroll
-    for (int c = 0; c < C::TABR; ++c) ttab[k * C::TABR + c] = make_float2(sc * cs.y, sc * cs.x);
+    for (int c = 0; c < C::TABR; ++c) ttab[k * C::TABR + c] = e;
   }
   __syncthreads();
 
