@@ -143,3 +143,53 @@ def test_longctx_decode_sweep_sampled(tac_gpu, orc):
             ref = orc.encode(x64, s, n, b, mode)
             parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=f"longctx enc n={n}")
             del x, y, cache
+
+
+def test_full_cache_attention_sampled(tac_gpu, orc):
+    """Attention from the records at the bench's size and launch configuration
+    (`bench.py --config attend`: 32 layers x 8 KV heads x 32768 tokens, one job
+    per (layer, head), 4 query rows, one tac_attend_multi call): every output
+    finite, sampled jobs equal to fp64 softmax attention over the oracle's
+    decode of their records within the bound of tests/test_gpu_attend.py."""
+    torch = _torch()
+    tac = tac_gpu
+    w = workloads.CONFIGS["mistral7b"]
+    T, nq = w.tokens, 4
+    caches, jobs = {}, []
+    for l in range(w.layers):
+        for kv in (workloads.K, workloads.V):
+            d, n, b, mode = w.codebook(l, kv)
+            cfg = tac.layer_cfg(d, n, b, mode, 0, l, kv)
+            x = workloads.block(w, l, kv, device="cuda", dtype=torch.bfloat16)
+            for h in range(w.heads):
+                caches[(l, kv, h)] = (cfg, tac.encode(x[h * T:(h + 1) * T], cfg))
+            del x
+        for h in range(w.heads):
+            g = torch.Generator(device="cuda")
+            g.manual_seed(l * 64 + h)
+            q = torch.randn((nq, w.d), generator=g, device="cuda").to(torch.bfloat16)
+            (kc, kk), (vc, vk) = caches[(l, workloads.K, h)], caches[(l, workloads.V, h)]
+            jobs.append(((l, h), tac.AttendJob(kc, kk, vc, vk, T, q, torch.empty_like(q), 1.0 / math.sqrt(w.d))))
+    tac.attend_multi([j for _, j in jobs])
+    torch.cuda.synchronize()
+    for _, j in jobs:
+        assert torch.isfinite(j.out.float()).all()
+    picks = {(0, 0), (17, 3), (31, 7)}
+    for (l, h), j in jobs:
+        if (l, h) not in picks:
+            continue
+        dec = []
+        for kv in (workloads.K, workloads.V):
+            cfg, cache = caches[(l, kv, h)]
+            k, c, hdr = parity.gpu_codes(orc, cache, T)
+            if hdr is None:
+                hdr = np.zeros((T, 2), dtype=np.float32)
+            dec.append(orc.decode(k, c, hdr, parity.signs_pm1(cfg.signs, cfg.d), cfg.n_angle, cfg.norm_bits,
+                                  cfg.norm_mode))
+        kh, vh = dec
+        q64 = parity.to_f64(j.q)
+        want = orc.attend(q64, kh, vh, j.scale)
+        tol = (2.0**-11 * j.scale * np.linalg.norm(q64, axis=1, keepdims=True) * np.linalg.norm(kh, axis=1).max()
+               + 2.0**-16) * np.abs(vh).max() + parity.bf16_half_ulp(want)
+        err = np.abs(parity.to_f64(j.out) - want)
+        assert np.all(err <= tol), ((l, h), float((err / tol).max()))
