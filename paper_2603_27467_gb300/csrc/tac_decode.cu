@@ -9,7 +9,8 @@
 //      lane for contiguous slots, per-row copies for gathered slots;
 //   2. lane l unpacks its 8 consecutive codes (pairs 8l..8l+7) and rebuilds each
 //      pair from its bin-centre angle by table lookup: the table holds
-//      (cos phi_k + sin phi_k, cos phi_k - sin phi_k) / sqrt(d), i.e. the
+//      (cos phi_k + sin phi_k, cos phi_k - sin phi_k) / sqrt(d) (fp16 pairs
+//      for bf16 output, fp32 pairs for fp32 output), i.e. the
 //      element-pair butterfly stage and the 1/sqrt(d) normalization are folded
 //      into the lookup, so the remaining butterfly stages run straight from
 //      (E_i, O_i) = r^_i * T[k_i] on packed fp32 pairs (FADD2/FFMA2): the low
