@@ -68,6 +68,12 @@ def _load():
         lib.orc_pack.argtypes = [vp, c_i64, c_int, c_int, vp]
         lib.orc_unpack.restype = c_int
         lib.orc_unpack.argtypes = [vp, c_i64, c_int, c_int, vp]
+        lib.orc_slot_pair.restype = c_int
+        lib.orc_slot_pair.argtypes = [c_int, c_int]
+        lib.orc_pack_record.restype = c_int
+        lib.orc_pack_record.argtypes = [vp, c_i64, c_int, c_int, vp]
+        lib.orc_unpack_record.restype = c_int
+        lib.orc_unpack_record.argtypes = [vp, c_i64, c_int, c_int, vp]
         lib.orc_avg_angle_bits.restype = c_dbl
         lib.orc_avg_angle_bits.argtypes = [c_int, vp, vp]
         lib.orc_total_bits.restype = c_dbl
@@ -177,6 +183,33 @@ def unpack(buf: np.ndarray, count: int, bits: int) -> np.ndarray:
     out = np.empty((rows, count), dtype=np.int32)
     if _load().orc_unpack(_ptr(buf), rows, count, bits, _ptr(out)):
         raise ValueError("orc_unpack failed")
+    return out
+
+
+def slot_order(d: int) -> np.ndarray:
+    """Record order (reading R9): element v = the pair whose code sits in slot v."""
+    lib = _load()
+    return np.array([lib.orc_slot_pair(d, v) for v in range(d // 2)], dtype=np.int64)
+
+
+def pack_record(codes: np.ndarray, d: int, bits: int) -> np.ndarray:
+    """Records of rows of d/2 codes given in pair order (slot order, then packed)."""
+    codes = np.ascontiguousarray(codes, dtype=np.int32)
+    rows = codes.shape[0]
+    stride = ((d // 2) * bits + 7) // 8
+    out = np.zeros((rows, stride), dtype=np.uint8)
+    if _load().orc_pack_record(_ptr(codes), rows, d, bits, _ptr(out)):
+        raise ValueError("orc_pack_record failed")
+    return out
+
+
+def unpack_record(buf: np.ndarray, d: int, bits: int) -> np.ndarray:
+    """Codes in pair order from records (inverse of pack_record)."""
+    buf = np.ascontiguousarray(buf, dtype=np.uint8)
+    rows = buf.shape[0]
+    out = np.zeros((rows, d // 2), dtype=np.int32)
+    if _load().orc_unpack_record(_ptr(buf), rows, d, bits, _ptr(out)):
+        raise ValueError("orc_unpack_record failed")
     return out
 
 

@@ -38,8 +38,10 @@
  *   R8 Signs D: s_j = -1 iff bit 63 of SplitMix64 output #j of the stream seeded with
  *      key = SplitMix64 output #q of the stream seeded with `seed`, q = 2*layer + kv
  *      (q = 0 for every (layer, kv) in "shared" mode, the paper's single D).
- *   R9 Bit packing: each vector's codes form one LSB-first bitstream (code i at bit
- *      i*w); a vector's stream starts on a byte boundary.
+ *   R9 Bit packing: each vector's codes form one LSB-first bitstream (code in slot
+ *      v at bit v*w); a vector's stream starts on a byte boundary.  Slot v holds
+ *      the code of pair phi_d(v) (orc_slot_pair: the natural order for d <= 32, a
+ *      fixed relabeling of the pair-index bits for d = 64, 128).
  *   R16 fp32 norm storage (mode 2, the angle-only configuration whose rates count
  *      angle bits only, Sec. 3.1 and Tables 1-4): each pair norm r_i is stored as
  *      the fp32 value nearest to it (its 32 bits are the "norm code", b = 32) and
@@ -312,6 +314,45 @@ int orc_unpack(const uint8_t* in, int64_t rows, int count, int bits, int32_t* co
     }
   }
   return 0;
+}
+
+/* Reading R9, record order: slot v of a vector's record (angle and norm codes
+ * alike) holds the code of pair phi_d(v).  For d = 64 and 128, with L = d/16:
+ *   phi(v) = 4 (v mod L) + ((v / L) mod 4) + 4 L floor(v / 4L),
+ * a relabeling of the pair-index bits under which the pairs held by one lane
+ * of a kernel that splits a vector over L lanes of 8 pairs (slots l + L m,
+ * m = 0..7) are two runs of 4 consecutive pairs.  For d <= 32 the order is
+ * the natural one. */
+int orc_slot_pair(int d, int v) {
+  if (d != 64 && d != 128) return v;
+  const int L = d / 16;
+  return 4 * (v % L) + (v / L) % 4 + 4 * L * (v / (4 * L));
+}
+
+/* Records of `rows` vectors of d/2 codes given in pair order: codes placed in
+ * slot order, then packed as orc_pack does. */
+int orc_pack_record(const int32_t* codes, int64_t rows, int d, int bits, uint8_t* out) {
+  const int P = d / 2;
+  int32_t* tmp = (int32_t*)malloc(sizeof(int32_t) * (size_t)P * (size_t)(rows > 0 ? rows : 1));
+  if (!tmp) return 2;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int v = 0; v < P; ++v) tmp[r * P + v] = codes[r * P + orc_slot_pair(d, v)];
+  const int rc = orc_pack(tmp, rows, P, bits, out);
+  free(tmp);
+  return rc;
+}
+
+/* The inverse: unpack a record and return its codes in pair order. */
+int orc_unpack_record(const uint8_t* in, int64_t rows, int d, int bits, int32_t* codes) {
+  const int P = d / 2;
+  int32_t* tmp = (int32_t*)malloc(sizeof(int32_t) * (size_t)P * (size_t)(rows > 0 ? rows : 1));
+  if (!tmp) return 2;
+  int rc = orc_unpack(in, rows, P, bits, tmp);
+  if (!rc)
+    for (int64_t r = 0; r < rows; ++r)
+      for (int v = 0; v < P; ++v) codes[r * P + orc_slot_pair(d, v)] = tmp[r * P + v];
+  free(tmp);
+  return rc;
 }
 
 /* Eq. 1: average angle bits over L layers with per-layer (n_K, n_V). */

@@ -167,10 +167,10 @@ __global__ void __launch_bounds__(32 * kAttMaxWarps, NQ <= 4 ? 2 : 1) attend_par
   smem_fwht<D>(qbuf, nq, tid, nthr, true);
   float2* qrot = reinterpret_cast<float2*>(smem + C::OFF_Q);
   const float qs = J.scale * kLog2e * rsqrtf((float)D);
-  for (int e = tid; e < NQ * P; e += nthr) {
-    const int a = e / P, i = e % P;
+  for (int e = tid; e < NQ * P; e += nthr) {   // in record (slot) order: slot i holds pair slot_pair(i)
+    const int a = e / P, i = e % P, ip = slot_pair<D>(i);
     qrot[a * C::QROW + qpos(i)] =
-        a < nq ? make_float2(qbuf[a * D + 2 * i] * qs, qbuf[a * D + 2 * i + 1] * qs) : make_float2(0.f, 0.f);
+        a < nq ? make_float2(qbuf[a * D + 2 * ip] * qs, qbuf[a * D + 2 * ip + 1] * qs) : make_float2(0.f, 0.f);
   }
   // ---- bin-centre tables (cos, sin)(2 pi k / n), 2^lgr copies: entry k copy c
   // at k 2^lgr + c; entries n..2^W-1 repeat entry n-1 (codes >= n clamp) ----
@@ -451,7 +451,8 @@ __global__ void __launch_bounds__(32 * kAttMaxWarps, NQ <= 4 ? 2 : 1) attend_par
       float* ra = rec + a * att_rec_floats(D);
       if (lane == 0) { ra[0] = m_run[a]; ra[1] = ls; }
 #pragma unroll
-      for (int j = 0; j < PV; ++j) *reinterpret_cast<float2*>(ra + 2 + 2 * (PV * lane + j)) = acc[a][j];
+      for (int j = 0; j < PV; ++j)   // accumulators are per slot; the record holds pairs in order
+        *reinterpret_cast<float2*>(ra + 2 + 2 * slot_pair<D>(PV * lane + j)) = acc[a][j];
     }
   }
 }

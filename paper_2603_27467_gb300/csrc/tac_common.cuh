@@ -79,10 +79,30 @@ struct RowTile {
   static constexpr int ROWB = D * ESZ;
   static constexpr int CPR = ROWB / 16;
   static constexpr int SPAN = 2 * ESZ * Geo<D>::L;
-  static constexpr int STRIDE = ROWB + (SPAN > 16 ? SPAN : 16);
+  // padded row pitch: the 16-byte run loads of two bf16 rows of d = 64 (one
+  // quarter-warp) fall on disjoint banks when the pitch is 64 mod 128
+  static constexpr int STRIDE = ROWB + ((D == 64 && ESZ == 2) ? 64 : (SPAN > 16 ? SPAN : 16));
   static constexpr int BYTES = Geo<D>::RW * STRIDE;            // one warp tile
   static constexpr int CHUNKS = Geo<D>::RW * CPR / 32;         // 16-byte chunks per lane
 };
+
+// Record order (reading R9): slot v of a record holds the code of pair
+// phi_d(v).  For d = 64 and 128 (L = d/16), phi(v) = 4 (v mod L) + ((v / L)
+// mod 4) + 4 L floor(v / 4L): the kernels work in slot order throughout, and
+// the slots l + L m (m = 0..7) a lane loads (encode) or stores (decode) are the
+// pairs 4 l + (m mod 4) + 4 L (m / 4), two runs of 4 consecutive pairs.  For
+// d <= 32 the order is natural.
+template <int D>
+__host__ __device__ constexpr bool run_layout() { return D == 64 || D == 128; }
+template <int D>
+__host__ __device__ constexpr int slot_pair(int v) {
+  if constexpr (run_layout<D>()) {
+    constexpr int L = D / 16;
+    return 4 * (v % L) + (v / L) % 4 + 4 * L * (v / (4 * L));
+  } else {
+    return v;
+  }
+}
 
 // ---------------------------------------------------------------------------
 // Device job descriptors (kernel parameters, copied by value at launch).

@@ -218,9 +218,37 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm,
     // Stages on pair-index bits 3..log2(P)-1 (this lane now holds pairs l + L*m).
     butterfly8<8, 8 / L>(v);
   }
-  // D, convert, store: pair i = l + L*m is element pair (2i, 2i+1).  The L
-  // lanes of a row store L consecutive pairs (a whole 32-byte sector for bf16),
-  // so every store instruction writes full sectors.
+  // D, convert, store.  Record order: slot l + L*m is pair 4l + (m & 3) +
+  // 4L (m >> 2), so a lane stores two runs of 4 pairs and the L lanes of a row
+  // fill two whole lines (d = 128, bf16) per pair of store instructions.
+  if constexpr (run_layout<D>()) {
+    if (live) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        uint8_t* run = orow + h * 8 * C::ESZ * L;
+        if constexpr (C::ESZ == 2) {
+          uint32_t w[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const __nv_bfloat162 bb = __floats2bfloat162_rn(v[4 * h + j].x, v[4 * h + j].y);
+            w[j] = (*reinterpret_cast<const uint32_t*>(&bb)) ^ msk[4 * h + j].x;
+          }
+          *reinterpret_cast<uint4*>(run) = make_uint4(w[0], w[1], w[2], w[3]);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 2; ++k) {
+            const int m0 = 4 * h + 2 * k;
+            *reinterpret_cast<uint4*>(run + 16 * k) =
+                make_uint4(__float_as_uint(v[m0].x) ^ msk[m0].x, __float_as_uint(v[m0].y) ^ msk[m0].y,
+                           __float_as_uint(v[m0 + 1].x) ^ msk[m0 + 1].x, __float_as_uint(v[m0 + 1].y) ^ msk[m0 + 1].y);
+          }
+        }
+      }
+    }
+    return;
+  }
+  // Natural order (d <= 32): pair i = l + L*m; the L lanes of a row store L
+  // consecutive pairs per instruction.
   if (live) {
 #pragma unroll
     for (int m = 0; m < 8; ++m) {
@@ -362,9 +390,9 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         c_left = J.rows - row0;
         const int64_t sb = J.stride * C::ESZ;
         c_step = C::RW * sb;
-        o_row = reinterpret_cast<uint8_t*>(J.y) + (row0 + r) * sb + 2 * C::ESZ * l;
+        o_row = reinterpret_cast<uint8_t*>(J.y) + (row0 + r) * sb + (run_layout<D>() ? 8 : 2) * C::ESZ * l;
 #pragma unroll
-        for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
+        for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, slot_pair<D>(l + C::L * m));
       }
     }
     const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;

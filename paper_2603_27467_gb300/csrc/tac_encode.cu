@@ -193,6 +193,7 @@ __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uin
   constexpr int ESZ = (int)sizeof(TIn);
   constexpr int P = G::P;
   float eh = 0.f, el = 0.f, oh = 0.f, ol = 0.f;
+  const int ip = slot_pair<D>(i);   // the pair held in slot i
   const uint8_t* row = in + rr * IT::STRIDE;
 #pragma unroll
   for (int j0 = 0; j0 < P; j0 += 32) {
@@ -207,7 +208,7 @@ __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uin
         const float2 u = *reinterpret_cast<const float2*>(row + 8 * jj);
         x0 = u.x; x1 = u.y;
       }
-      const bool neg = __popc((unsigned)(i & jj)) & 1;
+      const bool neg = __popc((unsigned)(ip & jj)) & 1;
       if (((signs[e0 >> 5] >> (e0 & 31)) & 1u) != (uint32_t)neg) x0 = -x0;
       if (((signs[e1 >> 5] >> (e1 & 31)) & 1u) != (uint32_t)neg) x1 = -x1;
       float t;
@@ -278,7 +279,33 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
 
   // ---- load 8 pairs (i = l + L*m), apply D, widen ----
   float2 v[8];
-  {
+  if constexpr (run_layout<D>()) {
+    // slots l + L m: pairs 4l + (m & 3) + 4L (m >> 2), two 16-byte (bf16) or
+    // 32-byte (fp32) runs of 4 pairs
+    const uint8_t* row = in + r * IT::STRIDE + 8 * C::ESZ * l;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const uint8_t* run = row + h * 8 * C::ESZ * L;
+      if constexpr (C::ESZ == 2) {
+        const uint4 q = *reinterpret_cast<const uint4*>(run);
+        const uint32_t u[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t w = u[j] ^ msk[4 * h + j].x;
+          v[4 * h + j] = make_float2(bf16lo(w), bf16hi(w));
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          const uint4 q = *reinterpret_cast<const uint4*>(run + 16 * k);
+          v[4 * h + 2 * k] = make_float2(__uint_as_float(q.x ^ msk[4 * h + 2 * k].x),
+                                         __uint_as_float(q.y ^ msk[4 * h + 2 * k].y));
+          v[4 * h + 2 * k + 1] = make_float2(__uint_as_float(q.z ^ msk[4 * h + 2 * k + 1].x),
+                                             __uint_as_float(q.w ^ msk[4 * h + 2 * k + 1].y));
+        }
+      }
+    }
+  } else {
     const uint8_t* row = in + r * IT::STRIDE + 2 * C::ESZ * l;
 #pragma unroll
     for (int m = 0; m < 8; ++m) {
@@ -620,7 +647,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
         }
         const int l = lane % C::L;
 #pragma unroll
-        for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, l + C::L * m);
+        for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, slot_pair<D>(l + C::L * m));
         __syncwarp();
       }
     }

@@ -55,9 +55,8 @@ def gpu_codes(orc, cache, rows: int | None = None, slots: np.ndarray | None = No
     codes, norms = codes[sel], norms[sel]
     if hdr is not None:
         hdr = np.array(hdr[sel], dtype=np.float32)
-    P = cfg.d // 2
-    k = orc.unpack(codes, P, code_bits(cfg.n_angle))
-    c = orc.unpack(norms, P, cfg.norm_bits)
+    k = orc.unpack_record(codes, cfg.d, code_bits(cfg.n_angle))
+    c = orc.unpack_record(norms, cfg.d, cfg.norm_bits)
     return k, c, hdr
 
 

@@ -21,8 +21,8 @@ def _oracle_cache(tac, orc, cfg, ref):
     rows = ref["k"].shape[0]
     w = parity.code_bits(cfg.n_angle)
     cache = tac.Cache.empty(cfg, rows)
-    ang = orc.pack(ref["k"], w).reshape(-1)
-    nrm = orc.pack(ref["c"], cfg.norm_bits).reshape(-1)
+    ang = orc.pack_record(ref["k"], cfg.d, w).reshape(-1)
+    nrm = orc.pack_record(ref["c"], cfg.d, cfg.norm_bits).reshape(-1)
     off = tac.header_offset(cfg, rows)
     nb = np.zeros(tac.norms_bytes(cfg, rows), dtype=np.uint8)
     nb[: nrm.size] = nrm

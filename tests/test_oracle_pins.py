@@ -480,3 +480,38 @@ def test_attend_rotated_domain_identity(orc):
     khat = orc.transform(y, np.ones(d, dtype=np.int8)) * s      # D H y (H symmetric)
     qr = orc.transform(q, s)                                     # H D q
     assert np.allclose(q @ khat.T, qr @ y.T, atol=1e-11)
+
+
+def test_record_slot_order(orc):
+    """Reading R9's record order: slot v holds pair phi_d(v).  A bijection of the
+    d/2 pairs; the natural order for d <= 32; for d = 64, 128 (L = d/16) the
+    slots l + L m (m = 0..3 and 4..7) hold the runs of 4 consecutive pairs
+    starting at 4 l and 4 L + 4 l; values written out by hand for d = 128."""
+    for d in (2, 4, 8, 16, 32, 64, 128):
+        phi = orc.slot_order(d)
+        assert sorted(phi.tolist()) == list(range(d // 2)), d
+        if d <= 32:
+            assert phi.tolist() == list(range(d // 2))
+    phi = orc.slot_order(128)
+    assert phi[:10].tolist() == [0, 4, 8, 12, 16, 20, 24, 28, 1, 5]
+    assert phi[31] == 31 and phi[32] == 32 and phi[33] == 36 and phi[63] == 63
+    assert orc.slot_order(64)[:6].tolist() == [0, 4, 8, 12, 1, 5]
+    for d in (64, 128):
+        L = d // 16
+        phi = orc.slot_order(d)
+        for l in range(L):
+            for h in (0, 1):
+                run = sorted(phi[l + L * m] for m in range(4 * h, 4 * h + 4))
+                assert run == [4 * L * h + 4 * l + j for j in range(4)], (d, l, h)
+
+
+def test_record_pack_is_pack_in_slot_order(orc):
+    """pack_record = pack of the codes taken in slot order; unpack_record inverts it."""
+    rng = np.random.default_rng(5)
+    for d in (16, 64, 128):
+        for bits in (3, 6, 8, 32):
+            codes = rng.integers(0, 2**min(bits, 31), size=(5, d // 2))
+            phi = orc.slot_order(d)
+            rec = orc.pack_record(codes, d, bits)
+            assert np.array_equal(rec, orc.pack(codes[:, phi], bits))
+            assert np.array_equal(orc.unpack_record(rec, d, bits), codes)
