@@ -19,9 +19,15 @@
  *
  * Record layout ("three planes", caller-owned device memory, one record slot per row):
  *   angle plane   slot s at  codes + s * tac_angle_row_bytes(cfg):  d/2 codes of w = ceil(log2 n)
- *                 bits, one LSB-first bitstream per row (code i occupies bits [i*w, i*w + w)).
- *   norm plane    slot s at  norms + s * tac_norm_row_bytes(cfg):   d/2 codes of b bits, same order
- *                 (TAC_NORM_FP32: d/2 little-endian floats r_i).
+ *                 bits, one LSB-first bitstream per row (the code in position v occupies bits
+ *                 [v*w, v*w + w)).  Position v holds the code of pair i = phi(v):
+ *                   d = 64, 128 (L = d/16):  phi(v) = 4 (v mod L) + ((v / L) mod 4) + 4 L floor(v / 4L)
+ *                   d = 16, 32:              phi(v) = v
+ *                 (pair i = elements 2i, 2i+1 of the transformed row).  The order lets a kernel
+ *                 that splits a row over L lanes of 8 positions move two runs of 4 consecutive
+ *                 pairs per lane; the paper fixes no layout.
+ *   norm plane    slot s at  norms + s * tac_norm_row_bytes(cfg):   d/2 codes of b bits, same
+ *                 positions (TAC_NORM_FP32: d/2 little-endian floats, position v = r_phi(v)).
  *   header plane  slot s at  norms + tac_header_offset(cfg, capacity) + 8*s:
  *                 float r_min, float r_max (little endian); absent with TAC_NORM_FP32.
  *
