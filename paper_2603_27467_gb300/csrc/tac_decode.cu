@@ -25,6 +25,8 @@ namespace tac {
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles of records in flight
 
+__host__ __device__ constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v >> 1); }
+
 // Copies of an n-entry table of esz-byte entries within `budget` bytes (at most maxr).
 __host__ __device__ constexpr int tab_copies_e(int n, int budget, int esz, int maxr) {
   int r = maxr;
@@ -158,12 +160,20 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm,
   const int r = lane / L, l = lane % L;
 
   const uint64_t acc_a = load_bytes<W>(rec + C::R_ANG + r * AB + l * W);
-  // A code of a non-power-of-two n is < n in every record this library
-  // writes; clamping keeps any other record's table reads in bounds.
-  auto code = [&](int j) -> uint32_t {
-    const uint32_t k = (uint32_t)(acc_a >> (j * W)) & (uint32_t)((1 << W) - 1);
-    if constexpr (is_pow2(N)) return k;
-    else return min(k, (uint32_t)(n - 1));
+  // Code j's table entry: the W-bit field shifted straight to bit TSH (one
+  // entry = TABR copies of TAB_E bytes), masked and OR'd with this lane's copy
+  // offset: the byte offset of the entry in one shift and one logic op.  A
+  // code of a non-power-of-two n is < n in every record this library writes;
+  // clamping keeps any other record's table reads in bounds.
+  constexpr int TSH = ilog2(C::TABR * C::TAB_E);
+  const uint32_t lane_off = (uint32_t)((lane % C::TABR) * C::TAB_E);
+  const uint8_t* tb = reinterpret_cast<const uint8_t*>(ttab);
+  auto entry = [&](int j) -> float2 {
+    const int pos = j * W;
+    const uint32_t x = pos >= TSH ? (uint32_t)(acc_a >> (pos - TSH)) : (uint32_t)acc_a << (TSH - pos);
+    uint32_t o = (x & ((uint32_t)((1 << W) - 1) << TSH)) | lane_off;
+    if constexpr (!is_pow2(N)) o = min(o, ((uint32_t)(n - 1) << TSH) | lane_off);
+    return centre(*reinterpret_cast<const typename C::TabT*>(tb + o));
   };
   float2 v[8];
   if constexpr (MODE == TAC_NORM_FP32) {  // r^ = the stored fp32 norm (Sec. 3.1)
@@ -171,7 +181,7 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm,
     const float4 a = rp[0], b = rp[1];
     const float rr[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
 #pragma unroll
-    for (int j = 0; j < 8; ++j) v[j] = mul2(make_float2(rr[j], rr[j]), centre(ttab[code(j) * C::TABR]));
+    for (int j = 0; j < 8; ++j) v[j] = mul2(make_float2(rr[j], rr[j]), entry(j));
   } else {
   constexpr int Lq = (1 << B) - 1;
   const uint64_t acc_n = load_bytes<B>(rec + C::R_NRM + r * NB + l * B);
@@ -196,11 +206,14 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm,
 
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    const uint32_t cb = (uint32_t)(acc_n >> (j * B)) & (uint32_t)Lq;
-    const float f = __uint_as_float(0x3F800000u | (cb << (23 - B)));
+    // norm code j shifted straight into the mantissa position 23 - B
+    constexpr int NSH = 23 - B;
+    const int pos = j * B;
+    const uint32_t x = pos >= NSH ? (uint32_t)(acc_n >> (pos - NSH)) : (uint32_t)acc_n << (NSH - pos);
+    const float f = __uint_as_float(0x3F800000u | (x & ((uint32_t)Lq << NSH)));
     float rh = __fmaf_rn(f, S, base2);
     if constexpr (MODE != TAC_NORM_LINEAR) rh = ex2_ftz(rh);
-    v[j] = mul2(make_float2(rh, rh), centre(ttab[code(j) * C::TABR]));
+    v[j] = mul2(make_float2(rh, rh), entry(j));
   }
   }
   // Butterfly stages on pair-index bits 0..2 (this lane holds pairs 8l..8l+7).
@@ -396,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
       }
     }
     const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;
-    decode_body<D, TOut, N, B, MODE>(rec, wsm, ttab + (lane % C::TABR), lane, msk, o_row,
+    decode_body<D, TOut, N, B, MODE>(rec, wsm, ttab, lane, msk, o_row,
                                      fast_tile || r < c_left);
     o_row += c_step;
     c_left -= C::RW;
