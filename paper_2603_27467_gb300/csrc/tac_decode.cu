@@ -9,8 +9,7 @@
 //      lane for contiguous slots, per-row copies for gathered slots;
 //   2. lane l unpacks its 8 consecutive codes (pairs 8l..8l+7) and rebuilds each
 //      pair from its bin-centre angle by table lookup: the table holds
-//      (cos phi_k + sin phi_k, cos phi_k - sin phi_k) / sqrt(d) (fp16 pairs
-//      for bf16 output, fp32 pairs for fp32 output), i.e. the
+//      (cos phi_k + sin phi_k, cos phi_k - sin phi_k) / sqrt(d), i.e. the
 //      element-pair butterfly stage and the 1/sqrt(d) normalization are folded
 //      into the lookup, so the remaining butterfly stages run straight from
 //      (E_i, O_i) = r^_i * T[k_i] on packed fp32 pairs (FADD2/FFMA2): the low
@@ -27,21 +26,6 @@ constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles of recor
 
 __host__ __device__ constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v >> 1); }
 
-// Copies of an n-entry table of esz-byte entries within `budget` bytes (at most maxr).
-__host__ __device__ constexpr int tab_copies_e(int n, int budget, int esz, int maxr) {
-  int r = maxr;
-  while (r > 1 && n * r * esz > budget) r >>= 1;
-  return r;
-}
-
-// Centre-table entries: fp32 pairs for fp32 output; for bf16 output, fp16
-// pairs (relative error 2^-11 per entry, an output error below 2^-11 |x^|,
-// within the bf16 output tolerance) so a warp's lookups take one shared
-// wavefront with one table copy per lane.
-template <int ESZ> struct CentreT { using T = float2; };
-template <> struct CentreT<2> { using T = __half2; };
-__device__ __forceinline__ float2 centre(float2 t) { return t; }
-__device__ __forceinline__ float2 centre(__half2 t) { return __half22float2(t); }
 
 // Shape of one kernel: n bins (W = ceil(log2 n) bits per code), B norm bits
 // (4, 8, or 32 for fp32 norms), MODE; HB header bytes per row (none for fp32).
@@ -67,9 +51,8 @@ struct Dec {
   static constexpr int W_REC = 0;                           // kNS record stages
   static constexpr int W_TP = W_REC + kNS * REC_W;          // transpose rows
   static constexpr int WARP_B = W_TP + G::TP_W;
-  using TabT = typename CentreT<ESZ>::T;
-  static constexpr int TAB_E = (int)sizeof(TabT);
-  static constexpr int TABR = tab_copies_e(n, 16384, TAB_E, ESZ == 2 ? 32 : 16);   // centre table copies
+  static constexpr int TAB_E = 8;                           // one (float2) centre-table entry
+  static constexpr int TABR = tab_copies(n, 16384);          // centre table copies
   static constexpr int OFF_TAB = kWarps * WARP_B;           // centre table of this n (TABR copies)
   static constexpr int SMEM = OFF_TAB + n * TABR * TAB_E;
   static_assert(REC_W % 16 == 0 && W_TP % 16 == 0 && WARP_B % 16 == 0, "alignment");
@@ -149,8 +132,7 @@ __device__ __forceinline__ uint64_t load_bytes(const uint8_t* p) {
 // lane's copy of the replicated centre table; orow: the lane's first output
 // pair, element 2l of its row; live: the row exists).
 template <int D, typename TOut, int N, int B, int MODE>
-__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm,
-                                            const typename Dec<D, TOut, N, B, MODE>::TabT* ttab, int lane,
+__device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, const float2* ttab, int lane,
                                             const uint2 (&msk)[8], uint8_t* orow, bool live) {
   using C = Dec<D, TOut, N, B, MODE>;
   using G = Geo<D>;
@@ -173,7 +155,7 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm,
     const uint32_t x = pos >= TSH ? (uint32_t)(acc_a >> (pos - TSH)) : (uint32_t)acc_a << (TSH - pos);
     uint32_t o = (x & ((uint32_t)((1 << W) - 1) << TSH)) | lane_off;
     if constexpr (!is_pow2(N)) o = min(o, ((uint32_t)(n - 1) << TSH) | lane_off);
-    return centre(*reinterpret_cast<const typename C::TabT*>(tb + o));
+    return *reinterpret_cast<const float2*>(tb + o);
   };
   float2 v[8];
   if constexpr (MODE == TAC_NORM_FP32) {  // r^ = the stored fp32 norm (Sec. 3.1)
@@ -284,14 +266,11 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
   const int warp = tid >> 5, lane = tid & 31;
 
   // Centre table of this n: (cos + sin, cos - sin)(2 pi k / n) / sqrt(d).
-  using TabT = typename C::TabT;
-  TabT* ttab = reinterpret_cast<TabT*>(smem + C::OFF_TAB);
+  float2* ttab = reinterpret_cast<float2*>(smem + C::OFF_TAB);
   const float sc = sqrtf(2.f / (float)D);  // sqrt2 / sqrt(d)
   for (int k = tid; k < C::n; k += kThreads) {
     const float2 cs = cos_sin_q8(centre_q8(k, C::n), C::n);  // (cos psi, sin psi), psi = phi + pi/4
-    TabT e;
-    if constexpr (C::ESZ == 2) e = __floats2half2_rn(sc * cs.y, sc * cs.x);
-    else e = make_float2(sc * cs.y, sc * cs.x);
+    const float2 e = make_float2(sc * cs.y, sc * cs.x);
 #pragma unroll
     for (int c = 0; c < C::TABR; ++c) ttab[k * C::TABR + c] = e;
   }
