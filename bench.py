@@ -40,11 +40,11 @@ FALLBACK_HBM_GBS = 6800.0
 # kernel sources it was measured on; after any change to them it reads null.
 MEASURED_TRAFFIC = {
     "encode": {"sources": ("tac_common.cuh", "tac_encode.cu"), "sha256_16": "df393bd8eb0f7ce4",
-               "bytes_per_row": 318.914},
-    "decode": {"sources": ("tac_common.cuh", "tac_decode.cu"), "sha256_16": "3708cb9c8bda0ef3",
-               "bytes_per_row": 275.051},
-    "attend": {"sources": ("tac_common.cuh", "tac_attend.cuh", "tac_attend.cu"), "sha256_16": "b9b7bb097c305745",
-               "bytes_per_row": 228.550},
+               "bytes_per_row": 319.086},
+    "decode": {"sources": ("tac_common.cuh", "tac_decode.cu"), "sha256_16": "878c3bece0e051e9",
+               "bytes_per_row": 272.643},
+    "attend": {"sources": ("tac_common.cuh", "tac_attend.cuh", "tac_attend.cu"), "sha256_16": "2cc127dfe6dba2aa",
+               "bytes_per_row": 215.310},
 }
 
 
@@ -486,8 +486,8 @@ def run_attend(args):
         "roofline": {"bound": "hbm", "kernel": "attend_partial + attend_combine", "achieved": gbs, "peak": hbm,
                      "unit": "GB/s", "frac": gbs / hbm, "peak_source": f"{peak_kind} hbm_gbs",
                      "traffic": measured_traffic("attend", w.layers * w.heads * T),
-                     "traffic_note": "attend_partial DRAM bytes per token-head from ncu at 4096 tokens, "
-                                     "scaled by token-heads; null once the kernel source changes"},
+                     "traffic_note": "attend_partial DRAM bytes per token-head (all launches of a step) from ncu "
+                                     "at 4096 tokens, scaled by token-heads; null once the kernel source changes"},
         "gpu_launches": 2 * args.steps * (1 + (len(jobs) - 1) // 96), "clocks": clocks}), flush=True)
 
 
