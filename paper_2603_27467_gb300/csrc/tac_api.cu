@@ -3,6 +3,7 @@
 // tac_decode.cu and tac_fwht_debug.cu.
 #include <algorithm>
 #include <cmath>
+#include <mutex>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -246,6 +247,88 @@ double tac_total_bits(double b_angle, double b_norm, int d) {
   return b_angle + b_norm / 2.0 + 64.0 / (double)d;
 }
 
+namespace {
+
+// The kernel groups of one multi call are independent.  The first runs on the
+// caller's stream, the others on library-owned streams (kSide per device,
+// created on the first call that has several groups) that wait for the
+// caller's stream at the call; the caller's stream waits for them before the
+// call returns.  Small groups then fill the tail of the large one instead of
+// queueing behind it, and the call stays ordered on the caller's stream
+// (under stream capture this is the usual fork / join).
+constexpr int kSide = 3;
+struct SideStreams {
+  bool init = false;
+  cudaStream_t s[kSide] = {};
+  cudaEvent_t fork = nullptr;
+  cudaEvent_t join[kSide] = {};
+};
+std::mutex g_side_mu;
+SideStreams g_side[64];
+
+class GroupFork {
+ public:
+  GroupFork(cudaStream_t user, int ngroups) : user_(user) {
+    if (ngroups <= 1) return;
+    int dev = 0;
+    if ((err_ = cudaGetDevice(&dev)) != cudaSuccess) return;
+    if (dev < 0 || dev >= 64) { err_ = cudaErrorInvalidDevice; return; }
+    lock_ = std::unique_lock<std::mutex>(g_side_mu);
+    SideStreams& S = g_side[dev];
+    if (!S.init) {
+      for (int q = 0; q < kSide && err_ == cudaSuccess; ++q)
+        if (!S.s[q]) err_ = cudaStreamCreateWithFlags(&S.s[q], cudaStreamNonBlocking);
+      if (err_ == cudaSuccess && !S.fork) err_ = cudaEventCreateWithFlags(&S.fork, cudaEventDisableTiming);
+      for (int q = 0; q < kSide && err_ == cudaSuccess; ++q)
+        if (!S.join[q]) err_ = cudaEventCreateWithFlags(&S.join[q], cudaEventDisableTiming);
+      if (err_ != cudaSuccess) return;
+      S.init = true;
+    }
+    if ((err_ = cudaEventRecord(S.fork, user)) != cudaSuccess) return;
+    st_ = &S;
+  }
+  cudaError_t error() const { return err_; }
+  // Stream of group g (0 = the caller's).
+  cudaStream_t stream(int g) {
+    if (!st_ || g == 0) return user_;
+    const int q = (g - 1) % kSide;
+    if (q >= used_) {
+      const cudaError_t e = cudaStreamWaitEvent(st_->s[q], st_->fork, 0);
+      if (e != cudaSuccess && err_ == cudaSuccess) err_ = e;
+      used_ = q + 1;
+    }
+    return st_->s[q];
+  }
+  // The caller's stream waits for every side stream used.
+  cudaError_t join() {
+    for (int q = 0; st_ && q < used_; ++q) {
+      cudaError_t e = cudaEventRecord(st_->join[q], st_->s[q]);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(user_, st_->join[q], 0);
+      if (e != cudaSuccess && err_ == cudaSuccess) err_ = e;
+    }
+    used_ = 0;
+    return err_;
+  }
+
+ private:
+  cudaStream_t user_;
+  SideStreams* st_ = nullptr;
+  std::unique_lock<std::mutex> lock_;
+  int used_ = 0;
+  cudaError_t err_ = cudaSuccess;
+};
+
+struct EncGroup {
+  tac::EncParams p;
+  int d, dt, na, nb, mode;
+};
+struct DecGroup {
+  tac::DecParams p;
+  int d, dt, na, nb, mode;
+};
+
+}  // namespace
+
 int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream) {
   static const char* who = "tac_encode_multi";
   if (njobs < 0) return fail(TAC_E_INVAL, "%s: njobs = %d", who, njobs);
@@ -279,13 +362,18 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
     return (((J.cfg.d * 4 + J.x.dtype) * 512 + J.cfg.n_angle) * 64 + J.cfg.norm_bits) * 4 + J.cfg.norm_mode;
   };
   std::stable_sort(live.begin(), live.end(), [&](int a, int b) { return kernel_key(a) < kernel_key(b); });
-  static thread_local tac::EncParams P;
+  static thread_local std::vector<EncGroup> groups;
+  groups.clear();
   size_t i = 0;
   while (i < live.size()) {
     const int key = kernel_key(live[i]);
     const tac_layer_cfg& c0 = jobs[live[i]].cfg;
     const int d = c0.d, dt = jobs[live[i]].x.dtype;
     const int na = c0.n_angle, nb = c0.norm_bits, mode = c0.norm_mode;
+    groups.emplace_back();
+    EncGroup& G = groups.back();
+    G.d = d; G.dt = dt; G.na = na; G.nb = nb; G.mode = mode;
+    tac::EncParams& P = G.p;
     std::memset(&P, 0, sizeof(P));
     int64_t tiles = 0;
     while (i < live.size() && P.njobs < TAC_MAX_JOBS && kernel_key(live[i]) == key) {
@@ -313,9 +401,22 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
     }
     if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many rows", who);
     P.ntiles = (int32_t)tiles;
-    cudaError_t e = tac::launch_encode(d, dt, na, nb, mode, P, sms, reinterpret_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
   }
+  // largest groups first: the small ones fill the tail of the large ones
+  std::stable_sort(groups.begin(), groups.end(),
+                   [](const EncGroup& a, const EncGroup& b) { return a.p.ntiles > b.p.ntiles; });
+  GroupFork fork(reinterpret_cast<cudaStream_t>(stream), (int)groups.size());
+  if (fork.error() != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(fork.error()));
+  for (size_t g = 0; g < groups.size(); ++g) {
+    const EncGroup& G = groups[g];
+    cudaError_t e = tac::launch_encode(G.d, G.dt, G.na, G.nb, G.mode, G.p, sms, fork.stream((int)g));
+    if (e != cudaSuccess) {
+      fork.join();
+      return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+    }
+  }
+  const cudaError_t e = fork.join();
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(e));
   return ok();
 }
 
@@ -351,13 +452,18 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
     return (((J.cfg.d * 4 + J.y.dtype) * 512 + J.cfg.n_angle) * 64 + J.cfg.norm_bits) * 4 + J.cfg.norm_mode;
   };
   std::stable_sort(live.begin(), live.end(), [&](int a, int b) { return kernel_key(a) < kernel_key(b); });
-  static thread_local tac::DecParams P;
+  static thread_local std::vector<DecGroup> groups;
+  groups.clear();
   size_t i = 0;
   while (i < live.size()) {
     const int key = kernel_key(live[i]);
     const tac_layer_cfg& c0 = jobs[live[i]].cfg;
     const int d = c0.d, dt = jobs[live[i]].y.dtype;
     const int na = c0.n_angle, nb = c0.norm_bits, mode = c0.norm_mode;
+    groups.emplace_back();
+    DecGroup& G = groups.back();
+    G.d = d; G.dt = dt; G.na = na; G.nb = nb; G.mode = mode;
+    tac::DecParams& P = G.p;
     std::memset(&P, 0, sizeof(P));
     int64_t tiles = 0;
     while (i < live.size() && P.njobs < TAC_MAX_JOBS && kernel_key(live[i]) == key) {
@@ -385,9 +491,21 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
     }
     if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many rows", who);
     P.ntiles = (int32_t)tiles;
-    cudaError_t e = tac::launch_decode(d, dt, na, nb, mode, P, sms, reinterpret_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
   }
+  std::stable_sort(groups.begin(), groups.end(),
+                   [](const DecGroup& a, const DecGroup& b) { return a.p.ntiles > b.p.ntiles; });
+  GroupFork fork(reinterpret_cast<cudaStream_t>(stream), (int)groups.size());
+  if (fork.error() != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(fork.error()));
+  for (size_t g = 0; g < groups.size(); ++g) {
+    const DecGroup& G = groups[g];
+    cudaError_t e = tac::launch_decode(G.d, G.dt, G.na, G.nb, G.mode, G.p, sms, fork.stream((int)g));
+    if (e != cudaSuccess) {
+      fork.join();
+      return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+    }
+  }
+  const cudaError_t e = fork.join();
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(e));
   return ok();
 }
 
