@@ -35,7 +35,8 @@
  *   - All device pointers must be 16-byte aligned; rows are row_stride elements
  *     apart and row_stride * sizeof(element) must be a multiple of 16.
  *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
- *     stream), allocate nothing, and never synchronize.
+ *     stream), allocate no device memory, and never synchronize (the batched
+ *     calls create their helper streams once, see tac_encode_multi).
  *   - Errors: a nonzero tac_status is returned and tac_last_error() gives a message
  *     (per host thread).  TAC_E_INVAL: a bad argument (nothing launched).
  *     TAC_E_UNSUPPORTED: a valid but unimplemented shape (nothing launched).
@@ -161,13 +162,19 @@ int tac_decode(const void* codes, const void* norms, const tac_layer_cfg* cfg, t
 /*
  * Batched encode.  Jobs may mix d, input dtypes and codebooks; jobs that share
  * the kernel shape (d, dtype, n_angle, norm_bits, norm_mode) run in one launch
- * (one per TAC_MAX_JOBS such jobs), the groups run back to back on `stream`.
- * With `slot` the rows of a decode step land at per-sequence record slots
- * (streaming append).  Jobs must not write overlapping slots.
+ * (one per TAC_MAX_JOBS such jobs).  With several launches they run
+ * concurrently, largest first: the first on `stream`, the others on
+ * library-owned streams that wait for `stream` at the call (an event), while
+ * `stream` waits for them before the call returns (events), so the call's work
+ * is ordered on `stream` as if it ran there alone and may be captured into a
+ * CUDA graph.  The first call with several launches on a device creates three
+ * streams and four events (kept for the process); make it outside stream
+ * capture.  With `slot` the rows of a decode step land at per-sequence record
+ * slots (streaming append).  Jobs must not write overlapping slots.
  */
 int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream);
 
-/* Batched decode, grouped into launches like tac_encode_multi. */
+/* Batched decode, grouped into launches (run concurrently) like tac_encode_multi. */
 int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream);
 
 /*
