@@ -657,7 +657,7 @@ def main():
             "pct_hbm_peak": 100.0 * value / world / hbm,
             "encode_gbs": enc_gbs, "decode_gbs": dec_gbs,
             "tokens_per_s": world * ws.tokens * w.layers * K / (total_ms / 1e3),
-            "roofline": {"bound": "hbm", "kernel": f"{dom} (tac_{dom}_multi, one launch)",
+            "roofline": {"bound": "hbm", "kernel": f"{dom} (one tac_{dom}_multi call: one launch per kernel shape, run concurrently)",
                          "achieved": dom_gbs, "peak": hbm, "unit": "GB/s", "frac": dom_gbs / hbm,
                          "peak_source": f"{peak_kind} hbm_gbs",
                          "traffic": measured_traffic(dom, ws.rows_per_launch),
