@@ -488,7 +488,7 @@ def run_attend(args):
                      "traffic": measured_traffic("attend", w.layers * w.heads * T),
                      "traffic_note": "attend_partial DRAM bytes per token-head (all launches of a step) from ncu "
                                      "at 4096 tokens, scaled by token-heads; null once the kernel source changes"},
-        "gpu_launches": 2 * args.steps * (1 + (len(jobs) - 1) // 96), "clocks": clocks}), flush=True)
+        "gpu_launches": 2 * args.steps * (1 + (len(jobs) - 1) // tac.ATTEND_MAX_JOBS), "clocks": clocks}), flush=True)
 
 
 def probe_rd(args):

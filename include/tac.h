@@ -189,6 +189,7 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
  * Results agree with decode-then-attend up to fp32 rounding (not bit-exact).
  */
 #define TAC_MAX_QUERIES 8      /* query rows per job (a GQA group) */
+#define TAC_ATTEND_MAX_JOBS 160 /* jobs per launch pair of tac_attend_multi */
 #define TAC_ATTEND_SPLIT 256   /* tokens per partial result in the workspace */
 
 typedef struct {
@@ -210,7 +211,10 @@ typedef struct {
  * job's part rounded up to 16 bytes.  Returns -1 for invalid jobs. */
 int64_t tac_attend_workspace_bytes(const tac_attend_job* jobs, int njobs);
 
-/* Attention for every job (jobs of one (d, dtype) share a launch pair).
+/* Attention for every job.  Jobs of one (d, dtype) share a launch pair (up to
+ * TAC_ATTEND_MAX_JOBS jobs each); several launch pairs run concurrently on
+ * `stream` and the helper streams of tac_encode_multi (fork / join by events),
+ * ordered on `stream` as a whole.
  * `workspace` (device, 16-byte aligned, >= tac_attend_workspace_bytes) is the
  * caller's; its contents need no initialisation and are overwritten.  Calls
  * that share a workspace must not overlap in time. */

@@ -33,6 +33,7 @@ BF16, FP32 = 0, 1
 MAX_D = 128
 MAX_JOBS = 96  # TAC_MAX_JOBS: jobs per kernel launch
 ATTEND_STATIC_WS_BYTES = 8 << 20  # TAC_ATTEND_STATIC_WS_BYTES: static attention workspace per device
+ATTEND_MAX_JOBS = 160  # TAC_ATTEND_MAX_JOBS: jobs per attention launch pair
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "_build", "libtac.so")

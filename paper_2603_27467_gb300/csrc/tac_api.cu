@@ -609,12 +609,24 @@ int check_attend_jobs(const tac_attend_job* jobs, int njobs, int64_t* need, cons
 }
 
 // Launches checked jobs, grouped by (d, dtype) in job order, up to
-// TAC_MAX_JOBS per launch pair; each job's workspace part follows the
-// previous one's.  Allocates nothing.
-int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st, const char* who) {
+// TAC_ATTEND_MAX_JOBS per launch pair; each job's workspace part follows the
+// previous one's.  `concurrent`: several launch pairs run concurrently
+// (GroupFork); otherwise back to back on `st`.  Allocates nothing.
+int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st, bool concurrent, const char* who) {
+  static_assert(sizeof(tac::AttParams) <= 32764, "kernel parameter limit");
   static thread_local tac::AttParams P;
   static const int kD[2] = {64, 128};
   static const int kDt[2] = {TAC_BF16, TAC_FP32};
+  int ngroups = 0;
+  for (int d : kD)
+    for (int dt : kDt) {
+      int c = 0;
+      for (int j = 0; j < njobs; ++j) c += jobs[j].cfg_k.d == d && jobs[j].q.dtype == dt;
+      ngroups += (c + TAC_ATTEND_MAX_JOBS - 1) / TAC_ATTEND_MAX_JOBS;
+    }
+  GroupFork fork(st, concurrent ? ngroups : 1);
+  if (fork.error() != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(fork.error()));
+  int g = 0;
   int64_t ws_off = 0;
   for (int d : kD) {
     for (int dt : kDt) {
@@ -628,7 +640,7 @@ int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st
         std::memset(&P, 0, sizeof(P));
         int64_t splits = 0;
         int nrows = 0, nq_max = 1;
-        while (i < njobs && P.njobs < TAC_MAX_JOBS) {
+        while (i < njobs && P.njobs < TAC_ATTEND_MAX_JOBS) {
           const tac_attend_job& J = jobs[i];
           const int64_t ns = (J.tokens + TAC_ATTEND_SPLIT - 1) / TAC_ATTEND_SPLIT;
           if (splits + ns > 0x7fffffff) break;   // CTAs (<= splits) are assigned at launch
@@ -665,14 +677,22 @@ int run_attend(const tac_attend_job* jobs, int njobs, float* ws, cudaStream_t st
           ++P.njobs;
           i = next(i + 1);
         }
-        if (P.njobs == 0) return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many tokens", who);
+        if (P.njobs == 0) {
+          fork.join();
+          return fail(TAC_E_UNSUPPORTED, "%s: a single job has too many tokens", who);
+        }
         P.nsplits = (int32_t)splits;
         P.q_bf16 = dt == TAC_BF16;
-        cudaError_t e = tac::launch_attend(d, dt, nq_max, P, nrows, ws, st);
-        if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+        cudaError_t e = tac::launch_attend(d, dt, nq_max, P, nrows, ws, fork.stream(g++));
+        if (e != cudaSuccess) {
+          fork.join();
+          return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+        }
       }
     }
   }
+  const cudaError_t e = fork.join();
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(e));
   return ok();
 }
 
@@ -688,7 +708,7 @@ int tac_attend_multi(const tac_attend_job* jobs, int njobs, void* workspace, int
   if (!workspace || !aligned16(workspace) || workspace_bytes < need)
     return fail(TAC_E_INVAL, "%s: workspace NULL, misaligned or smaller than %lld bytes", who, (long long)need);
   if (num_sms() <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
-  return run_attend(jobs, njobs, static_cast<float*>(workspace), reinterpret_cast<cudaStream_t>(stream), who);
+  return run_attend(jobs, njobs, static_cast<float*>(workspace), reinterpret_cast<cudaStream_t>(stream), true, who);
 }
 
 int tac_attend_multi_static(const tac_attend_job* jobs, int njobs, tac_stream_t stream) {
@@ -706,7 +726,7 @@ int tac_attend_multi_static(const tac_attend_job* jobs, int njobs, tac_stream_t 
   if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: static workspace: %s", who, cudaGetErrorString(e));
   if (njobs == 0) return ok();
   if (num_sms() <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
-  return run_attend(jobs, njobs, ws, reinterpret_cast<cudaStream_t>(stream), who);
+  return run_attend(jobs, njobs, ws, reinterpret_cast<cudaStream_t>(stream), false, who);
 }
 
 int tac_fwht_debug(const tac_rows* x, int d, const uint32_t* signs, float* y, tac_stream_t stream) {

@@ -30,7 +30,7 @@ struct AttParams {
   int32_t nctas;
   int32_t nsplits;
   int32_t q_bf16;                    // queries (and outputs) are bf16 rows, else fp32
-  AttJob job[TAC_MAX_JOBS];
+  AttJob job[TAC_ATTEND_MAX_JOBS];   // 200 bytes each: within the 32 KB of kernel parameters
 };
 
 // Per-split workspace record: max (log2 units), sum, accumulator (d floats).

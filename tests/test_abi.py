@@ -212,3 +212,19 @@ def test_attend_validation_and_workspace_size(tac_host):
     assert lib.tac_attend_multi(a, 1, 4096, 16, None) == tac_host.TAC_E_INVAL        # workspace too small
     assert lib.tac_attend_multi(a, 1, 4100, 1 << 30, None) == tac_host.TAC_E_INVAL   # misaligned workspace
     assert lib.tac_attend_multi(None, 0, None, 0, None) == tac_host.TAC_OK
+
+
+def test_binding_constants_match_header(tac_host):
+    """The binding's copies of the header's limits agree with include/tac.h."""
+    import os
+    import re
+    src = open(os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "tac.h")).read()
+
+    def define(name):
+        m = re.search(r"#define\s+" + name + r"\s+(\d+)\b", src)
+        assert m, name
+        return int(m.group(1))
+
+    assert define("TAC_MAX_JOBS") == tac_host.MAX_JOBS
+    assert define("TAC_ATTEND_MAX_JOBS") == tac_host.ATTEND_MAX_JOBS
+    assert define("TAC_ATTEND_SPLIT") == 256
