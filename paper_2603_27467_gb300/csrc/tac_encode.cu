@@ -355,24 +355,38 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
 
   // ---- row constants: stored header (Sec. 3.3), Eq. 2 as code = floor(f(s) qs + qo) ----
   constexpr float k2 = 2.0f / (float)D;
+  constexpr float rk2 = D == 16 ? 0.35355339059327379f : D == 32 ? 0.25f : D == 64 ? 0.17677669529663687f : 0.125f;
+  // sqrt(2/d) above.  Exact power-of-two scaling: sigma = 4^-k with
+  // smax * sigma in [1, 4) (at least 2^-25 for the smallest subnormal smax), so
+  // the square roots and logarithms of the row and of its pairs run on normal
+  // arguments in their flush-to-zero hardware forms and are scaled back
+  // exactly: sqrt(s) = 2^k sqrt(s sigma), log2 s = log2(s sigma) + 2k.
+  const int ek = ((int)((__float_as_uint(smax) >> 23) & 0xFFu) - 127) >> 1;
+  const int kk = ek < -62 ? -62 : (ek > 63 ? 63 : ek);
+  const float sigma = __uint_as_float((uint32_t)(127 - 2 * kk) << 23);
+  const float sr = __uint_as_float((uint32_t)(127 + kk) << 23);   // 2^k
+  const float smax_s = smax * sigma;
   float hmin = 0.f, hmax = 0.f, qs = 0.f, qo = 0.f, sfloor = 0.f;
   if constexpr (FP32N) {
     // no header: the norms are stored as they are (Sec. 3.1)
   } else if constexpr (MODE == TAC_NORM_LINEAR) {
-    hmin = sqrt_approx(smin * k2);
-    hmax = sqrt_approx(smax * k2);
+    hmin = sqrt_approx(smin * k2);              // smin * sigma may still be subnormal
+    hmax = sqrt_ftz(smax_s * k2) * sr;
     const float sc = (float)Lq * rcp_approx(hmax - hmin);
-    qs = sc * sqrt_approx(k2);                  // f(s) = sqrt(s)
+    qs = sc * rk2;                              // f(s) = sqrt(s)
     qo = __fmaf_rn(-hmin, sc, 0.5f);
     if (!(hmax > hmin) || !(sc <= 3.0e38f)) { qs = 0.f; qo = 0.5f; }
   } else {  // log-space, norms floored at 2^-24 r_max
     sfloor = smax * 3.5527136788005009e-15f;    // 2^-48 on the energy
-    hmin = sqrt_approx(fmaxf(smin, sfloor) * k2);
-    hmax = sqrt_approx(smax * k2);
-    const float lmin = lg2_approx(hmin);
-    const float sc = (float)Lq * rcp_approx(lg2_approx(hmax) - lmin);
+    const float hmin_s = sqrt_ftz(fmaxf(smin, sfloor) * sigma * k2);   // >= 2^-24 hmax_s: normal
+    const float hmax_s = sqrt_ftz(smax_s * k2);
+    hmin = hmin_s * sr;
+    hmax = hmax_s * sr;
+    const float lmin_s = lg2_ftz(hmin_s);
+    const float sc = (float)Lq * rcp_approx(lg2_ftz(hmax_s) - lmin_s);
     qs = 0.5f * sc;                             // f(s) = log2 s; log2 r = (log2 s + log2 k2)/2
-    qo = __fmaf_rn(0.5f * (float)(G::LOGD == 4 ? -3 : G::LOGD == 5 ? -4 : G::LOGD == 6 ? -5 : -6) - lmin,
+    qo = __fmaf_rn(0.5f * (float)(G::LOGD == 4 ? -3 : G::LOGD == 5 ? -4 : G::LOGD == 6 ? -5 : -6) -
+                       (lmin_s + (float)kk),
                    sc, 0.5f);
     if (!(hmax > hmin) || !(sc <= 3.0e38f)) { qs = 0.f; qo = 0.5f; }
   }
@@ -384,17 +398,12 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   // S = sum_i (E_i^2 + O_i^2) = d ||x||_2^2 / 2 (the factor 1.01 covers the
   // rounding of the computed S and the second-order terms).  The edge direction
   // (<= 1 ulp), the product and the fma add <= 4 u (|E| + |O|) <= 4 u sqrt(2 smax).
-  const float rmx = sqrt_approx(smax);
-  const float ty = (float)(G::LOGD - 1) * kU * 1.01f * sqrt_approx(ssum);
+  const float rmx = sqrt_ftz(smax_s) * sr;
+  const float ty = (float)(G::LOGD - 1) * kU * 1.01f * (sqrt_ftz(ssum * sigma) * sr);
   const float tau = ty + 5.f * kU * 1.4143f * rmx;
-  // Per-pair norm functions run on s * sigma, sigma = 4^-k an exact power of two
-  // with smax * sigma in [1, 4): sqrt(s) = 2^k sqrt(s sigma), log2 s =
-  // log2(s sigma) + 2k, so the flush-to-zero hardware forms see normal numbers
-  // (pairs below the log floor are clamped to it first).
-  const int ek = ((int)((__float_as_uint(smax) >> 23) & 0xFFu) - 127) >> 1;
-  const int kk = ek < -62 ? -62 : (ek > 63 ? 63 : ek);
-  const float sigma = __uint_as_float((uint32_t)(127 - 2 * kk) << 23);
-  if constexpr (MODE == TAC_NORM_LINEAR) qs *= __uint_as_float((uint32_t)(127 + kk) << 23);
+  // The per-pair norm functions below take s * sigma (pairs below the log
+  // floor are clamped to it first).
+  if constexpr (MODE == TAC_NORM_LINEAR) qs *= sr;
   else qo = __fmaf_rn((float)(2 * kk), qs, qo);
   const float sfl = sfloor * sigma;
   (void)qs; (void)qo; (void)sfl;
