@@ -345,6 +345,26 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   float smin = lmin_s;
   float smax = max3(max3(s[0], s[1], s[2]), max3(s[3], s[4], s[5]), fmaxf(s[6], s[7]));
   float ssum = ((s[0] + s[1]) + (s[2] + s[3])) + ((s[4] + s[5]) + (s[6] + s[7]));
+
+  // ---- angle codes (Alg. 1): they need no row constant, so they are decided
+  // before the row reductions (whose shuffle latency they cover) ----
+  uint32_t alo = 0, ahi = 0;
+  float am[8];                                  // |m|: each pair's certification margin
+  float mmin = __int_as_float(0x7f800000);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    float m;
+    const uint32_t k = edge_test<N, C::TABR>(v[j].x, v[j].y, et, m);
+    am[j] = fabsf(m);
+    mmin = fminf(mmin, am[j]);
+    // fields are disjoint and k < n: the adds are ORs (one IMAD each)
+    const int sa = j * W;
+    if (sa + W <= 32) alo += k << sa;
+    else if (sa >= 32) ahi += k << (sa - 32);
+    else { alo += k << sa; ahi += k >> (32 - sa); }
+  }
+
+  // ---- row min / max / sum over the row's L lanes ----
 #pragma unroll
   for (int off = 1; off < L; off <<= 1) {
     smin = fminf(smin, __shfl_xor_sync(0xffffffffu, smin, off));
@@ -412,20 +432,12 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   const float rthr = ty * (4.f * (float)n / 3.14159265f);
   const float sthr = rthr * rthr;
 
-  // ---- pass 2: angle codes (Alg. 1), norm codes (Eq. 2), packing ----
-  uint32_t alo = 0, ahi = 0, nlo = 0, nhi = 0;
+  // ---- pass 2: norm codes (Eq. 2), packing ----
+  uint32_t nlo = 0, nhi = 0;
   float rn[FP32N ? 8 : 1];                      // fp32 norms r_j = sqrt(2 s_j / d)
-  float mmin = __int_as_float(0x7f800000);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    float m;
-    const uint32_t k = edge_test<N, C::TABR>(v[j].x, v[j].y, et, m);
-    mmin = fminf(mmin, fabsf(m));
-    // fields are disjoint and k < n, c <= Lq: the adds are ORs (one IMAD each)
-    const int sa = j * W;
-    if (sa + W <= 32) alo += k << sa;
-    else if (sa >= 32) ahi += k << (sa - 32);
-    else { alo += k << sa; ahi += k >> (32 - sa); }
+    // fields are disjoint and c <= Lq: the adds are ORs (one IMAD each)
     if constexpr (FP32N) {
       rn[j] = sqrt_approx(s[j] * k2);
     } else {
@@ -441,11 +453,8 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; }
   else if (mmin < tau || lmin_s < sthr) {  // rare: name the uncertified pairs
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      float m;
-      edge_test<N, C::TABR>(v[j].x, v[j].y, et, m);
-      if (fabsf(m) < tau || s[j] < sthr) fm |= 1u << j;
-    }
+    for (int j = 0; j < 8; ++j)
+      if (am[j] < tau || s[j] < sthr) fm |= 1u << j;
   }
   if (!live) fm = 0;
 
