@@ -10,7 +10,7 @@
 namespace tac {
 
 constexpr int kThreads = 256;      // threads per CTA
-constexpr int kMinBlocks = 3;      // resident CTAs per SM the kernels are built for (24 warps)
+constexpr int kMinBlocks = 2;      // resident CTAs per SM the encode / decode kernels are built for (16 warps, <= 128 registers)
 constexpr int kPairsPerThread = 8; // each thread owns 8 consecutive angle pairs (16 elements)
 constexpr int kMaxW = 8;           // code bits <= 8 (n <= 256)
 // Tables holding one entry per bin for every supported n back to back:

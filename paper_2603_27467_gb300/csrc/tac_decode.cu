@@ -259,6 +259,8 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
 }
 
 template <int D, typename TOut, int N, int B, int MODE>
+// Two CTAs per SM (up to 128 registers), as for the encoder: the scheduling
+// room is worth more than a third CTA of warps.
 __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecParams p) {
   using C = Dec<D, TOut, N, B, MODE>;
   extern __shared__ __align__(128) uint8_t smem[];

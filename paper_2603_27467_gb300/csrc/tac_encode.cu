@@ -531,7 +531,7 @@ __device__ __noinline__ void copy_out_slow(const WarpJob* wj, const uint8_t* san
 template <int D, typename TIn, int N, int B, int MODE>
 // Two CTAs per SM (up to 128 registers): the encode's long per-pair chains
 // gain more from the scheduling room than from a third CTA of warps.
-__global__ void __launch_bounds__(kThreads, 2) encode_kernel(const __grid_constant__ EncParams p) {
+__global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __grid_constant__ EncParams p) {
   using C = Enc<D, TIn, N, B, MODE>;
   using IT = typename C::IT;
   extern __shared__ __align__(128) uint8_t smem[];
