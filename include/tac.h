@@ -111,8 +111,9 @@ typedef struct {
   const void* codes;     /* angle plane of the source cache (device) */
   const void* norms;     /* norm + header planes of the source cache (device) */
   int64_t capacity;      /* record slots in the source planes */
-  const int64_t* slot;   /* device, y.rows entries: source slot of output row i, each in
-                            [0, capacity) (not checked on the device); NULL means slot i */
+  const int64_t* slot;   /* device, y.rows entries: source slot of output row i; a slot
+                            outside [0, capacity) decodes as an all-zero record (the
+                            row r_min = r_max = 0: zeros); NULL means slot i */
   tac_rows y;            /* output rows (device), bf16 (round to nearest even) or fp32 */
 } tac_decode_job;
 
