@@ -9,8 +9,7 @@
 
 namespace tac {
 
-constexpr int kThreads = 256;      // threads per CTA
-constexpr int kMinBlocks = 2;      // resident CTAs per SM the encode / decode kernels are built for (16 warps, <= 128 registers)
+constexpr int kMinBlocks = 2;      // resident CTAs per SM the encode / decode kernels are built for
 constexpr int kPairsPerThread = 8; // each thread owns 8 consecutive angle pairs (16 elements)
 constexpr int kMaxW = 8;           // code bits <= 8 (n <= 256)
 // Tables holding one entry per bin for every supported n back to back:
@@ -52,8 +51,6 @@ __host__ __device__ constexpr int tab_n_of(int idx) {
 // pairs, so L = P/8 lanes share a row and a warp covers RW = 32/L rows (its
 // "warp tile").  Every warp runs its own pipeline over warp tiles.
 // ---------------------------------------------------------------------------
-constexpr int kWarps = kThreads / 32;
-
 template <int D>
 struct Geo {
   static constexpr int P = D / 2;

@@ -18,10 +18,10 @@
 //      E_i = WHT_i(x_even), O_i = WHT_i(x_odd) give (y_2i, y_2i+1) = (E+O, E-O),
 //      so r_i^2 = 2 (E_i^2 + O_i^2) / d and the angle test works on (E_i, O_i);
 //   3. Alg. 1's k_i = floor(n theta/2pi + 1/2) mod n is decided by an exact edge
-//      test: a candidate edge from an octant-reduced arctangent polynomial
-//      (max error 0.0038 rad: Rajan, Wang, Inkol, Joyal, "Efficient
-//      approximations for the arctangent function", IEEE SPM 2006), then the sign
-//      of the cross product of (E, O) with the edge direction.  The test is
+//      test: a candidate edge from an arctangent approximation (the angle of
+//      (|E|, |O|) is pi/4 + atan((|O| - |E|) / (|O| + |E|)), with an odd cubic
+//      for atan on [-1, 1], max error 0.00496 rad), then the sign of the cross
+//      product of (E, O) with the edge direction.  The test is
 //      certified by a rigorous bound on the fp32 error; the pairs it does not
 //      certify are re-decided by the warp from error-free double-float sums of
 //      the staged input (no fp64: the FP64 pipe is a small fraction of fp32 here);
@@ -52,6 +52,12 @@ constexpr DFEdgeTable make_df_edge_table() {
 __constant__ cx::DFEdgeTable g_edge_df = cx::make_df_edge_table();
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles in flight
+// CTA shape of the encode: 10 warps, two CTAs per SM (20 warps, up to 102
+// registers a thread): the encode is issue-bound, and the extra warps hide
+// more latency than the 128-register build's longer chains (3 % faster; 12
+// warps at 80 registers emit more instructions).
+constexpr int kEncWarps = 10;
+constexpr int kEncThreads = 32 * kEncWarps;
 
 // Shape of one kernel: n bins (W = ceil(log2 n) bits per angle code), B norm
 // bits (4, 8, or 32 for fp32 norms), MODE; HB header bytes per row (8, none
@@ -83,7 +89,7 @@ struct Enc {
   static constexpr int W_JOB = W_HDR + RW * HB;             // current job (WarpJob)
   static constexpr int WARP_B = W_JOB + 64;
   static constexpr int TABR = tab_copies(n, 8192);           // edge table copies
-  static constexpr int OFF_TAB = kWarps * WARP_B;           // fp32 edge table of this n (TABR copies)
+  static constexpr int OFF_TAB = kEncWarps * WARP_B;           // fp32 edge table of this n (TABR copies)
   static constexpr int SMEM = OFF_TAB + n * TABR * 8;
   static_assert((RW * AB) % 16 == 0 && (RW * NB) % 16 == 0 && (RW * HB) % 16 == 0, "record segments");
   static_assert(W_TP % 16 == 0 && W_ANG % 16 == 0 && W_JOB % 16 == 0 && WARP_B % 16 == 0, "alignment");
@@ -134,46 +140,64 @@ __device__ __forceinline__ int wrap_bin(int v) {
 }
 
 // Candidate edge for the pair (E, O) (butterfly halves, y = (E + O, E - O))
-// and n bins: Alg. 1's angle theta = pi/4 - angle(E, O) from the
-// octant-reduced arctangent polynomial, in bins, floored (M + n/8 - angle,
-// rounded down onto the integer grid of M = 1.5 * 2^23; for n not a multiple
-// of 8 the shift of M + n/8 onto that grid is below half a bin).  The true bin
-// is the candidate or the next one whenever the polynomial's error (0.0038
-// rad) is below half a bin, i.e. for every n <= 256.
+// and n bins, before the reduction mod n: Alg. 1's angle theta = pi/4 -
+// angle(E, O) in bins, floored (for n >= 8, M + n/8 - angle rounded down onto
+// the integer grid of M = 1.5 * 2^23, where n/8 is an integer and M + n/8
+// exact; for n = 2, 4, whose n/8 is not on that grid, a direct conversion
+// rounding down, which gives the same value less M).  The
+// angle of (|E|, |O|) is pi/4 + atan(t) with t = (|O| - |E|) / (|O| + |E|) in
+// [-1, 1], so no octant test is needed; atan(t) ~ t (a + b t^2) is an odd
+// cubic fitted minimax on [-1, 1] for this kernel (max error 0.00496 rad).  The
+// true bin is the candidate or the next one whenever that error is below half
+// a bin, i.e. for every n <= 256 (0.2 bins at n = 256).  A zero pair gives NaN
+// here: it is decided by the exact path, and the callers mask or clamp the
+// result before it indexes a table.
 template <int N>
-__device__ __forceinline__ int candidate_edge(float E, float O) {
+__device__ __forceinline__ int candidate_bits(float E, float O) {
   constexpr int n = N;
   constexpr float nb = (float)n * 0.15915494309189535f;  // bins per radian
-  constexpr float c1 = (0.78539816f + 0.273f) * nb;       // atan(t) ~ t (pi/4 + 0.273 (1 - t))
-  constexpr float c2 = 0.273f * nb;
+  constexpr float ca = 0.97239412f * nb, cb = -0.19194795f * nb;
   const float aE = fabsf(E), aO = fabsf(O);
-  const float mx = fmaxf(aE, aO), mn = fminf(aE, aO);
-  const float t = mn * rcp_approx(mx);
-  const float phi = t * __fmaf_rn(t, -c2, c1);                 // octant angle, bins
-  float fb = (aO > aE) ? (0.25f * n - phi) : phi;              // angle of (|E|, |O|)
-  fb = (E < 0.f) ? (0.5f * n - fb) : fb;                       // angle of (E, |O|)
+  const float t = (aO - aE) * rcp_approx(aO + aE);
+  const float q = __fmaf_rn(t, __fmaf_rn(t * t, cb, ca), 0.125f * n);   // angle of (|E|, |O|), bins
+  const float fb = (E < 0.f) ? (0.5f * n - q) : q;                      // angle of (E, |O|)
   const float ab = __uint_as_float(__float_as_uint(fb) ^ (__float_as_uint(O) & 0x80000000u));
-  const int bits = __float_as_int(__fadd_rd(12582912.0f + 0.125f * n, -ab));
+  if constexpr (n % 8 != 0) return __float2int_rd(0.125f * n - ab);
+  else return __float_as_int(__fadd_rd(12582912.0f + 0.125f * n, -ab));
+}
+
+// The candidate edge in [0, n).
+template <int N>
+__device__ __forceinline__ int candidate_edge(float E, float O) {
+  const int bits = candidate_bits<N>(E, O);
   if constexpr (is_pow2(N)) {
-    return bits & (n - 1);
+    return bits & (N - 1);
   } else {
-    // 0x4B400000 = bits of M.  A zero pair gives NaN here (its code is decided
-    // by the exact path); the clamp keeps every table index inside [0, n).
+    // 0x4B400000 = bits of M; the clamp keeps a zero pair's NaN inside [0, n).
     const int e = wrap_bin<N>(bits - 0x4B400000);
-    return (int)min((uint32_t)e, (uint32_t)(n - 1));
+    return (int)min((uint32_t)e, (uint32_t)(N - 1));
   }
 }
 
 // Alg. 1 bin of the pair (E, O) for n bins by the edge test: the candidate
 // edge, then the sign of the cross product with the edge direction (et: this
-// lane's copy of the replicated table, R copies).  Returns k; m is the signed
-// cross product (its magnitude is the certification margin).
+// lane's copy of the replicated table, R copies).  Returns k; m = O s - E c is
+// the cross product with the sign turned (k is the next bin when m < 0); its
+// magnitude is the certification margin, and a pair with m == 0 is never
+// certified, so which side the fast path gives it does not matter.
 template <int N, int R>
 __device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et, float& m) {
-  const int e = candidate_edge<N>(E, O);
-  const float2 dir = et[e * R];
-  m = __fmaf_rn(E, dir.x, -__fmul_rn(O, dir.y));
-  return (uint32_t)wrap_bin<N>(e + 1 + (__float_as_int(m) >> 31));
+  if constexpr (is_pow2(N)) {
+    const int bits = candidate_bits<N>(E, O);
+    const float2 dir = et[(bits & (N - 1)) * R];
+    m = __fmaf_rn(O, dir.y, -__fmul_rn(E, dir.x));
+    return (uint32_t)(bits + (int)(__float_as_uint(m) >> 31)) & (uint32_t)(N - 1);
+  } else {
+    const int e = candidate_edge<N>(E, O);
+    const float2 dir = et[e * R];
+    m = __fmaf_rn(O, dir.y, -__fmul_rn(E, dir.x));
+    return (uint32_t)wrap_bin<N>(e + (int)(__float_as_uint(m) >> 31));
+  }
 }
 
 // Exact re-decision of pair i of warp-tile row rr by the whole warp (all lanes
@@ -350,19 +374,19 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   // before the row reductions (whose shuffle latency they cover) ----
   uint32_t alo = 0, ahi = 0;
   float am[8];                                  // |m|: each pair's certification margin
-  float mmin = __int_as_float(0x7f800000);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     float m;
     const uint32_t k = edge_test<N, C::TABR>(v[j].x, v[j].y, et, m);
     am[j] = fabsf(m);
-    mmin = fminf(mmin, am[j]);
     // fields are disjoint and k < n: the adds are ORs (one IMAD each)
     const int sa = j * W;
     if (sa + W <= 32) alo += k << sa;
     else if (sa >= 32) ahi += k << (sa - 32);
     else { alo += k << sa; ahi += k >> (32 - sa); }
   }
+
+  const float mmin = min3(min3(am[0], am[1], am[2]), min3(am[3], am[4], am[5]), fminf(am[6], am[7]));
 
   // ---- row min / max / sum over the row's L lanes ----
 #pragma unroll
@@ -529,9 +553,8 @@ __device__ __noinline__ void copy_out_slow(const WarpJob* wj, const uint8_t* san
 }
 
 template <int D, typename TIn, int N, int B, int MODE>
-// Two CTAs per SM (up to 128 registers): the encode's long per-pair chains
-// gain more from the scheduling room than from a third CTA of warps.
-__global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __grid_constant__ EncParams p) {
+// Two CTAs of kEncWarps warps per SM (see kEncWarps).
+__global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const __grid_constant__ EncParams p) {
   using C = Enc<D, TIn, N, B, MODE>;
   using IT = typename C::IT;
   extern __shared__ __align__(128) uint8_t smem[];
@@ -540,7 +563,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
 
   // fp32 edge table of this n (shared by the CTA).
   float2* etab = reinterpret_cast<float2*>(smem + C::OFF_TAB);
-  for (int e = tid; e < C::n; e += kThreads) {
+  for (int e = tid; e < C::n; e += kEncThreads) {
     const float2 cs = cos_sin_q8(edge_q8(e, C::n), C::n);
 #pragma unroll
     for (int c = 0; c < C::TABR; ++c) etab[e * C::TABR + c] = cs;
@@ -550,7 +573,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) encode_kernel(const __gr
   // Each warp owns a contiguous range of warp tiles (balanced to +-1 tile), so
   // it meets a new job at most a few times per launch and walks its planes
   // with pointer increments.
-  const int Gw = gridDim.x * kWarps, gw = blockIdx.x * kWarps + warp;
+  const int Gw = gridDim.x * kEncWarps, gw = blockIdx.x * kEncWarps + warp;
   const int per = p.ntiles / Gw, extra = p.ntiles % Gw;
   int t = gw * per + min(gw, extra);
   const int t_end = t + per + (gw < extra ? 1 : 0);
@@ -718,14 +741,14 @@ static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_
     configured[dev] = 1;
   }
   int per_sm = 0;
-  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, C::SMEM);
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kEncThreads, C::SMEM);
   if (e != cudaSuccess) return e;
   if (per_sm < 1) per_sm = 1;
   int grid = grid_cap * per_sm;
-  const int need = (p.ntiles + kWarps - 1) / kWarps;
+  const int need = (p.ntiles + kEncWarps - 1) / kEncWarps;
   if (grid > need) grid = need;
   if (grid < 1) return cudaSuccess;
-  kern<<<grid, kThreads, C::SMEM, st>>>(p);
+  kern<<<grid, kEncThreads, C::SMEM, st>>>(p);
   return cudaGetLastError();
 }
 

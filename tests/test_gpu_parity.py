@@ -202,6 +202,29 @@ def test_exact_bin_centres_and_ties(tac_gpu, orc):
             assert np.all(k[0] == 1) and np.all(k[1] == 0) and np.all(k[2] == 1) and np.all(k[3] == 2)
 
 
+@pytest.mark.parametrize("n", [2, 4, 8, 16, 64, 256])
+def test_pairs_next_to_bin_edges(tac_gpu, orc, n):
+    """Pairs a small angle (1e-6 .. 1e-2 rad, either side) from a bin edge of
+    Alg. 1, theta = (k + 1/2) 2 pi / n: a candidate edge one bin off would be
+    decided wrong there, by the fast test or the exact path.  fp32 rows
+    x = D H y; the oracle sees the same rounded inputs, every code must match."""
+    torch = _torch()
+    d, rows = 128, 64
+    P = d // 2
+    rng = np.random.default_rng(100 + n)
+    k = rng.integers(0, n, size=(rows, P))
+    delta = rng.choice([1e-6, 1e-5, 1e-4, 1e-3, 1e-2], size=(rows, P)) * rng.choice([-1.0, 1.0], size=(rows, P))
+    theta = (k + 0.5) * 2.0 * np.pi / n + delta
+    r = 0.5 + rng.random((rows, P))
+    y = np.zeros((rows, d))
+    y[:, 0::2], y[:, 1::2] = r * np.cos(theta), r * np.sin(theta)
+    s = orc.signs(0, 0, 0, d)
+    x = (orc.transform(y, np.ones(d, dtype=np.int8)) * s).astype(np.float32)
+    st = check_roundtrip(tac_gpu, orc, torch.tensor(x).cuda(), d, n, 8, 0, label=f"near edges n={n}",
+                         decode_dtypes=("fp32",))
+    assert st["angle_mismatch"] == 0, st
+
+
 @pytest.mark.parametrize("d,n,b,mode", [(128, 64, 8, 0), (128, 256, 4, 1), (64, 128, 8, 0)])
 def test_many_tiles_per_cta_every_row(tac_gpu, orc, d, n, b, mode):
     """Enough rows that every CTA of the persistent grid loops over many tiles
