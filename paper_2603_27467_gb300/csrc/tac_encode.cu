@@ -159,8 +159,10 @@ __device__ __forceinline__ int candidate_bits(float E, float O) {
   constexpr float ca = 0.97239412f * nb, cb = -0.19194795f * nb;
   const float aE = fabsf(E), aO = fabsf(O);
   const float t = (aO - aE) * rcp_approx(aO + aE);
-  const float q = __fmaf_rn(t, __fmaf_rn(t * t, cb, ca), 0.125f * n);   // angle of (|E|, |O|), bins
-  const float fb = (E < 0.f) ? (0.5f * n - q) : q;                      // angle of (E, |O|)
+  // angle of (|E|, |O|) less n/4, in bins: in [-n/4, 0]
+  const float dq = __fmaf_rn(t, __fmaf_rn(t * t, cb, ca), -0.125f * n);
+  // angle of (E, |O|): n/4 + dq, or n/2 - (n/4 + dq) = n/4 - dq when E < 0
+  const float fb = 0.25f * n + __uint_as_float(__float_as_uint(dq) ^ (__float_as_uint(E) & 0x80000000u));
   const float ab = __uint_as_float(__float_as_uint(fb) ^ (__float_as_uint(O) & 0x80000000u));
   if constexpr (n % 8 != 0) return __float2int_rd(0.125f * n - ab);
   else return __float_as_int(__fadd_rd(12582912.0f + 0.125f * n, -ab));
@@ -288,7 +290,10 @@ __device__ __forceinline__ void patch_code(uint8_t* rec, int i, int k) {
 template <int D, typename TIn, int N, int B, int MODE>
 __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const float2* et, int nrows,
                                           int lane, const uint2 (&msk)[8], const uint32_t* signs) {
-  // (for bf16 only msk[m].x is used; the .y words are constant zero)
+  // bf16: msk[m].x holds the sign bits of the pair's two elements (bits 15
+  // and 31), msk[m].y the low element's bit moved to bit 31.  The low element
+  // widens as w * 2^16 + msk.y (adding bit 31 is an XOR of it: one integer
+  // multiply-add), the high one as (w ^ msk.x) & 0xFFFF0000 (one logic op).
   using C = Enc<D, TIn, N, B, MODE>;
   using G = Geo<D>;
   using IT = typename C::IT;
@@ -315,8 +320,9 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
         const uint32_t u[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          const uint32_t w = u[j] ^ msk[4 * h + j].x;
-          v[4 * h + j] = make_float2(bf16lo(w), bf16hi(w));
+          const uint2 mk = msk[4 * h + j];
+          v[4 * h + j] = make_float2(__uint_as_float(u[j] * 65536u + mk.y),
+                                     __uint_as_float((u[j] ^ mk.x) & 0xFFFF0000u));
         }
       } else {
 #pragma unroll
@@ -334,8 +340,8 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
 #pragma unroll
     for (int m = 0; m < 8; ++m) {
       if constexpr (C::ESZ == 2) {
-        const uint32_t u = *reinterpret_cast<const uint32_t*>(row + 4 * L * m) ^ msk[m].x;
-        v[m] = make_float2(bf16lo(u), bf16hi(u));
+        const uint32_t u = *reinterpret_cast<const uint32_t*>(row + 4 * L * m);
+        v[m] = make_float2(__uint_as_float(u * 65536u + msk[m].y), __uint_as_float((u ^ msk[m].x) & 0xFFFF0000u));
       } else {
         const uint2 u = *reinterpret_cast<const uint2*>(row + 8 * L * m);
         v[m] = make_float2(__uint_as_float(u.x ^ msk[m].x), __uint_as_float(u.y ^ msk[m].y));
@@ -690,7 +696,10 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
         }
         const int l = lane % C::L;
 #pragma unroll
-        for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, slot_pair<D>(l + C::L * m));
+        for (int m = 0; m < 8; ++m) {
+          msk[m] = pair_sign_mask<C::ESZ>(J.signs, slot_pair<D>(l + C::L * m));
+          if constexpr (C::ESZ == 2) msk[m].y = msk[m].x << 16;
+        }
         __syncwarp();
       }
     }
