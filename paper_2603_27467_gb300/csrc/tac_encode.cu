@@ -657,57 +657,78 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
   // the current (dense) job and the prefetched tile a full tile of the issue
   // job inside the warp's range.  Set by the general iterations.
   int fast = 0;
-  for (; t < t_end; ++t) {
-    cp_async_wait<kNS - 2>();   // this warp tile has landed
-    __syncwarp();               // ... and every lane is done with the previous one
-    const int ns = (stage + kNS - 1) & (kNS - 1);
-    const bool fast_tile = fast > 0;
-    if (fast_tile) {
-      --fast;
-      uint8_t* dst = in_dst + ns * IT::BYTES;
+  const float2* const etl = etab + (lane % C::TABR);
+  while (t < t_end) {
+    if (fast > 0) {
+      // A stretch of `fast` tiles, each a full tile of the current dense job
+      // whose prefetch is a full tile of the issue job: no per-tile checks, the
+      // cursors are settled once after it.
+      const int t_stop = t + fast;
+      for (; t < t_stop; ++t) {
+        cp_async_wait<kNS - 2>();   // this warp tile has landed
+        __syncwarp();               // ... and every lane is done with the previous one
+        uint8_t* dst = in_dst + ((stage + kNS - 1) & (kNS - 1)) * IT::BYTES;
 #pragma unroll
-      for (int q = 0; q < C::CHUNKS; ++q) cp_async16(dst + q * C::RPQ * IT::STRIDE, i_src + q * i_qstep, 16);
-      cp_async_commit();
-      i_src += i_step;
-      i_left -= C::RW;
-      ++it;
-    } else {
-      issue(ns);
-      if (t >= c_end) {  // next job
-        const int cj = find_job(p, t);
-        const EncJob& J = p.job[cj];
-        c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
-        const int rel = t - J.tile0;
-        c_row0 = (int64_t)rel * C::RW;
-        c_left = J.rows - c_row0;
-        c_dense = J.slot == nullptr;
+        for (int q = 0; q < C::CHUNKS; ++q) cp_async16(dst + q * C::RPQ * IT::STRIDE, i_src + q * i_qstep, 16);
+        cp_async_commit();
+        i_src += i_step;
+        tile_body<D, TIn, N, B, MODE>(wsm + C::W_IN + stage * IT::BYTES, wsm, etl, C::RW, lane, msk, wj->signs);
+        __syncwarp();
 #pragma unroll
         for (int q = 0; q < C::ROUNDS; ++q) {
           const int ch = q * 32 + lane;
-          if (ch < C::NA) { o_dst[q] = J.codes + 16 * ch; o_step[q] = C::RW * C::AB; }
-          else if (ch < C::NA + C::NN) { o_dst[q] = J.norms + 16 * (ch - C::NA); o_step[q] = C::RW * C::NB; }
-          else { o_dst[q] = J.hdr + 16 * (ch - C::NA - C::NN); o_step[q] = C::RW * C::HB; }
-          o_dst[q] += (int64_t)rel * o_step[q];
+          if (ch < C::NCH)
+            *reinterpret_cast<uint4*>(o_dst[q]) = *reinterpret_cast<const uint4*>(wsm + C::W_ANG + 16 * ch);
+          o_dst[q] += o_step[q];
         }
-        if (lane == 0) {
-          wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot; wj->capacity = J.capacity;
-#pragma unroll
-          for (int q = 0; q < 4; ++q) wj->signs[q] = J.signs[q];
-        }
-        const int l = lane % C::L;
-#pragma unroll
-        for (int m = 0; m < 8; ++m) {
-          msk[m] = pair_sign_mask<C::ESZ>(J.signs, slot_pair<D>(l + C::L * m));
-          if constexpr (C::ESZ == 2) msk[m].y = msk[m].x << 16;
-        }
-        __syncwarp();
+        stage = (stage + 1) & (kNS - 1);
       }
+      const int64_t adv = (int64_t)fast * C::RW;
+      c_row0 += adv;
+      c_left -= adv;
+      i_left -= adv;
+      it += fast;
+      fast = 0;
+      continue;
     }
-    const int nrows = (fast_tile || c_left >= C::RW) ? C::RW : (int)c_left;
-    const uint8_t* in = wsm + C::W_IN + stage * IT::BYTES;
-    tile_body<D, TIn, N, B, MODE>(in, wsm, etab + (lane % C::TABR), nrows, lane, msk, wj->signs);
+
+    // ---- general tile: a job's first tile, tails, scattered slots, range ends ----
+    cp_async_wait<kNS - 2>();
     __syncwarp();
-    if (fast_tile || (c_dense && nrows == C::RW)) {
+    issue((stage + kNS - 1) & (kNS - 1));
+    if (t >= c_end) {  // next job
+      const int cj = find_job(p, t);
+      const EncJob& J = p.job[cj];
+      c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
+      const int rel = t - J.tile0;
+      c_row0 = (int64_t)rel * C::RW;
+      c_left = J.rows - c_row0;
+      c_dense = J.slot == nullptr;
+#pragma unroll
+      for (int q = 0; q < C::ROUNDS; ++q) {
+        const int ch = q * 32 + lane;
+        if (ch < C::NA) { o_dst[q] = J.codes + 16 * ch; o_step[q] = C::RW * C::AB; }
+        else if (ch < C::NA + C::NN) { o_dst[q] = J.norms + 16 * (ch - C::NA); o_step[q] = C::RW * C::NB; }
+        else { o_dst[q] = J.hdr + 16 * (ch - C::NA - C::NN); o_step[q] = C::RW * C::HB; }
+        o_dst[q] += (int64_t)rel * o_step[q];
+      }
+      if (lane == 0) {
+        wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot; wj->capacity = J.capacity;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) wj->signs[q] = J.signs[q];
+      }
+      const int l = lane % C::L;
+#pragma unroll
+      for (int m = 0; m < 8; ++m) {
+        msk[m] = pair_sign_mask<C::ESZ>(J.signs, slot_pair<D>(l + C::L * m));
+        if constexpr (C::ESZ == 2) msk[m].y = msk[m].x << 16;
+      }
+      __syncwarp();
+    }
+    const int nrows = c_left >= C::RW ? C::RW : (int)c_left;
+    tile_body<D, TIn, N, B, MODE>(wsm + C::W_IN + stage * IT::BYTES, wsm, etl, nrows, lane, msk, wj->signs);
+    __syncwarp();
+    if (c_dense && nrows == C::RW) {
 #pragma unroll
       for (int q = 0; q < C::ROUNDS; ++q) {
         const int ch = q * 32 + lane;
@@ -722,14 +743,13 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
     c_row0 += C::RW;
     c_left -= C::RW;
     stage = (stage + 1) & (kNS - 1);
-    if (!fast_tile) {
-      // c_left now counts the rows of the compute job from tile t + 1, i_left
-      // those of the issue job from tile it (the next to prefetch).
-      const int64_t cf = c_dense ? c_left / C::RW : 0;
-      const int64_t pf = min(min((int64_t)(p_end - it), i_left / C::RW), (int64_t)(t_end - it));
-      const int64_t f = min(cf, pf);
-      fast = f > 0 ? (int)f : 0;
-    }
+    ++t;
+    // c_left now counts the rows of the compute job from tile t, i_left those
+    // of the issue job from tile it (the next to prefetch).
+    const int64_t cf = c_dense ? c_left / C::RW : 0;
+    const int64_t pf = min(min((int64_t)(p_end - it), i_left / C::RW), (int64_t)(t_end - it));
+    const int64_t f = min(cf, pf);
+    fast = f > 0 ? (int)f : 0;
   }
   cp_async_wait<0>();
 }
