@@ -361,53 +361,63 @@ __global__ void __launch_bounds__(Dec<D, TOut, N, B, MODE>::THREADS, kMinBlocks)
   // the current job and the prefetched tile a full tile of the (contiguous)
   // issue job inside the warp's range.  Set by the general iterations.
   int fast = 0;
-  for (; t < t_end; ++t) {
-    cp_async_wait<kNS - 2>();   // this warp tile's records have landed
-    __syncwarp();               // ... and every lane is done with the previous tile
-    const int ns = (stage + kNS - 1) & (kNS - 1);
-    const bool fast_tile = fast > 0;
-    if (fast_tile) {
-      --fast;
-      uint8_t* dst = wsm + C::W_REC + ns * C::REC_W;
+  while (t < t_end) {
+    if (fast > 0) {
+      // A stretch of `fast` tiles, each a full tile of the current job whose
+      // prefetch is a full tile of the (contiguous) issue job: no per-tile
+      // checks, the cursors are settled once after it.
+      const int t_stop = t + fast;
+      for (; t < t_stop; ++t) {
+        cp_async_wait<kNS - 2>();   // this warp tile's records have landed
+        __syncwarp();               // ... and every lane is done with the previous tile
+        uint8_t* dst = wsm + C::W_REC + ((stage + kNS - 1) & (kNS - 1)) * C::REC_W;
 #pragma unroll
-      for (int q = 0; q < C::ROUNDS; ++q) {
-        const int ch = q * 32 + lane;
-        if (ch < C::NCH) cp_async16(dst + 16 * ch, i_src[q], 16);
-        i_src[q] += i_step[q];
+        for (int q = 0; q < C::ROUNDS; ++q) {
+          const int ch = q * 32 + lane;
+          if (ch < C::NCH) cp_async16(dst + 16 * ch, i_src[q], 16);
+          i_src[q] += i_step[q];
+        }
+        cp_async_commit();
+        decode_body<D, TOut, N, B, MODE>(wsm + C::W_REC + stage * C::REC_W, wsm, ttab, lane, msk, o_row, true);
+        o_row += c_step;
+        stage = (stage + 1) & (kNS - 1);
       }
-      cp_async_commit();
-      i_row0 += C::RW;
-      i_left -= C::RW;
-      ++it;
-    } else {
-      issue(ns);
-      if (t >= c_end) {  // next job
-        const int cj = find_job(p, t);
-        const DecJob& J = p.job[cj];
-        c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
-        const int64_t row0 = (int64_t)(t - J.tile0) * C::RW;
-        c_left = J.rows - row0;
-        const int64_t sb = J.stride * C::ESZ;
-        c_step = C::RW * sb;
-        o_row = reinterpret_cast<uint8_t*>(J.y) + (row0 + r) * sb + (run_layout<D>() ? 8 : 2) * C::ESZ * l;
-#pragma unroll
-        for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, slot_pair<D>(l + C::L * m));
-      }
+      const int64_t adv = (int64_t)fast * C::RW;
+      i_row0 += adv;
+      i_left -= adv;
+      it += fast;
+      c_left -= adv;
+      fast = 0;
+      continue;
     }
-    const uint8_t* rec = wsm + C::W_REC + stage * C::REC_W;
-    decode_body<D, TOut, N, B, MODE>(rec, wsm, ttab, lane, msk, o_row,
-                                     fast_tile || r < c_left);
+
+    // ---- general tile: a job's first tile, tails, gathered slots, range ends ----
+    cp_async_wait<kNS - 2>();
+    __syncwarp();
+    issue((stage + kNS - 1) & (kNS - 1));
+    if (t >= c_end) {  // next job
+      const int cj = find_job(p, t);
+      const DecJob& J = p.job[cj];
+      c_end = (cj + 1 < p.njobs) ? p.job[cj + 1].tile0 : p.ntiles;
+      const int64_t row0 = (int64_t)(t - J.tile0) * C::RW;
+      c_left = J.rows - row0;
+      const int64_t sb = J.stride * C::ESZ;
+      c_step = C::RW * sb;
+      o_row = reinterpret_cast<uint8_t*>(J.y) + (row0 + r) * sb + (run_layout<D>() ? 8 : 2) * C::ESZ * l;
+#pragma unroll
+      for (int m = 0; m < 8; ++m) msk[m] = pair_sign_mask<C::ESZ>(J.signs, slot_pair<D>(l + C::L * m));
+    }
+    decode_body<D, TOut, N, B, MODE>(wsm + C::W_REC + stage * C::REC_W, wsm, ttab, lane, msk, o_row, r < c_left);
     o_row += c_step;
     c_left -= C::RW;
     stage = (stage + 1) & (kNS - 1);
-    if (!fast_tile) {
-      // c_left now counts the rows of the compute job from tile t + 1, i_left
-      // those of the issue job from tile it (the next to prefetch).
-      const int64_t cf = c_left / C::RW;
-      const int64_t pf = p_dense ? min(min((int64_t)(p_end - it), i_left / C::RW), (int64_t)(t_end - it)) : 0;
-      const int64_t f = min(cf, pf);
-      fast = f > 0 ? (int)f : 0;
-    }
+    ++t;
+    // c_left now counts the rows of the compute job from tile t, i_left those
+    // of the issue job from tile it (the next to prefetch).
+    const int64_t cf = c_left / C::RW;
+    const int64_t pf = p_dense ? min(min((int64_t)(p_end - it), i_left / C::RW), (int64_t)(t_end - it)) : 0;
+    const int64_t f = min(cf, pf);
+    fast = f > 0 ? (int)f : 0;
   }
   cp_async_wait<0>();
 }
