@@ -41,8 +41,11 @@
  *     (per host thread).  TAC_E_INVAL: a bad argument (nothing launched).
  *     TAC_E_UNSUPPORTED: a valid but unimplemented shape (nothing launched).
  *     TAC_E_CUDA: the launch failed (cudaGetLastError after the launch).
- *   - Inputs must be finite with |x_j| <= 2^56; other values give unspecified codes
- *     but never out-of-bounds accesses.
+ *   - Inputs must be finite with |x_j| <= 2^56, and each nonzero |x_j| >= 2^-53
+ *     for bf16 rows (>= 2^-37 for fp32 rows): then every nonzero pair energy
+ *     E^2 + O^2 of the butterfly is a normal fp32 number and the codes and header
+ *     match the definitions within the stated tolerances.  Other values give
+ *     unspecified codes but never out-of-bounds accesses.
  */
 #ifndef TAC_H_
 #define TAC_H_

@@ -416,12 +416,17 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   const float sigma = __uint_as_float((uint32_t)(127 - 2 * kk) << 23);
   const float sr = __uint_as_float((uint32_t)(127 + kk) << 23);   // 2^k
   const float smax_s = smax * sigma;
+  // sqrt(smax sigma); for d = 32, 128 the factor 2/d of r^2 is an even power of
+  // two, so sqrt(smax sigma 2/d) is taken as this times sqrt(2/d), an exact
+  // product (one hardware square root, about 1 ulp, either way).
+  constexpr bool kEvenK2 = D == 32 || D == 128;
+  const float rms = sqrt_ftz(smax_s);
   float hmin = 0.f, hmax = 0.f, qs = 0.f, qo = 0.f, sfloor = 0.f;
   if constexpr (FP32N) {
     // no header: the norms are stored as they are (Sec. 3.1)
   } else if constexpr (MODE == TAC_NORM_LINEAR) {
     hmin = sqrt_approx(smin * k2);              // smin * sigma may still be subnormal
-    hmax = sqrt_ftz(smax_s * k2) * sr;
+    hmax = (kEvenK2 ? rms * rk2 : sqrt_ftz(smax_s * k2)) * sr;
     const float sc = (float)Lq * rcp_approx(hmax - hmin);
     qs = sc * rk2;                              // f(s) = sqrt(s)
     qo = __fmaf_rn(-hmin, sc, 0.5f);
@@ -429,7 +434,7 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   } else {  // log-space, norms floored at 2^-24 r_max
     sfloor = smax * 3.5527136788005009e-15f;    // 2^-48 on the energy
     const float hmin_s = sqrt_ftz(fmaxf(smin, sfloor) * sigma * k2);   // >= 2^-24 hmax_s: normal
-    const float hmax_s = sqrt_ftz(smax_s * k2);
+    const float hmax_s = kEvenK2 ? rms * rk2 : sqrt_ftz(smax_s * k2);
     hmin = hmin_s * sr;
     hmax = hmax_s * sr;
     const float lmin_s = lg2_ftz(hmin_s);
@@ -448,7 +453,7 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   // S = sum_i (E_i^2 + O_i^2) = d ||x||_2^2 / 2 (the factor 1.01 covers the
   // rounding of the computed S and the second-order terms).  The edge direction
   // (<= 1 ulp), the product and the fma add <= 4 u (|E| + |O|) <= 4 u sqrt(2 smax).
-  const float rmx = sqrt_ftz(smax_s) * sr;
+  const float rmx = rms * sr;
   const float ty = (float)(G::LOGD - 1) * kU * 1.01f * (sqrt_ftz(ssum * sigma) * sr);
   const float tau = ty + 5.f * kU * 1.4143f * rmx;
   // The per-pair norm functions below take s * sigma (pairs below the log

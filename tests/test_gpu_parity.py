@@ -202,6 +202,34 @@ def test_exact_bin_centres_and_ties(tac_gpu, orc):
             assert np.all(k[0] == 1) and np.all(k[1] == 0) and np.all(k[2] == 1) and np.all(k[3] == 2)
 
 
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+@pytest.mark.parametrize("b,mode", [(8, 0), (4, 1)])
+def test_magnitude_range_limits(tac_gpu, orc, dt, b, mode):
+    """Rows at the ends of the documented input range, every nonzero |x_j| in
+    [2^-53, 2^56] (bf16) or [2^-37, 2^56] (fp32), where every nonzero pair
+    energy E^2 + O^2 is a normal fp32 number: rows of the smallest values, rows
+    of the largest (whose energy sum overflows, so every pair takes the exact
+    path) and rows spread over the whole range with zeros."""
+    torch = _torch()
+    d = 128
+    lo = -53 if dt == "bf16" else -37
+    rng = np.random.default_rng(7 + b + 2 * mode)
+
+    def row(elo, ehi, zero_frac=0.0):
+        e = rng.integers(elo, ehi + 1, size=d).astype(np.float64)
+        x = np.where(rng.random(d) < 0.5, -1.0, 1.0) * (1.0 + rng.random(d)) * np.exp2(e)
+        x[rng.random(d) < zero_frac] = 0.0
+        return x
+
+    rows = [row(lo, lo + 3) for _ in range(8)] + [row(52, 55) for _ in range(8)]
+    rows += [row(lo, 55, 0.1) for _ in range(16)]
+    x = torch.tensor(np.array(rows), dtype=torch.float32)
+    x = (x.to(torch.bfloat16) if dt == "bf16" else x).cuda()
+    xa = np.abs(parity.to_f64(x))
+    assert xa.max() <= 2.0**56 and xa[xa > 0].min() >= 2.0**lo
+    check_roundtrip(tac_gpu, orc, x, d, 64, b, mode, label=f"range {dt} b={b} m={mode}")
+
+
 @pytest.mark.parametrize("n", [2, 4, 8, 16, 64, 256])
 def test_pairs_next_to_bin_edges(tac_gpu, orc, n):
     """Pairs a small angle (1e-6 .. 1e-2 rad, either side) from a bin edge of
