@@ -456,12 +456,11 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   const float rmx = rms * sr;
   const float ty = (float)(G::LOGD - 1) * kU * 1.01f * (sqrt_ftz(ssum * sigma) * sr);
   const float tau = ty + 5.f * kU * 1.4143f * rmx;
-  // The per-pair norm functions below take s * sigma (pairs below the log
-  // floor are clamped to it first).
-  if constexpr (MODE == TAC_NORM_LINEAR) qs *= sr;
-  else qo = __fmaf_rn((float)(2 * kk), qs, qo);
-  const float sfl = sfloor * sigma;
-  (void)qs; (void)qo; (void)sfl;
+  // The per-pair norm functions below take s itself (pairs below the log floor
+  // are clamped to it first), against the true-scale qs, qo: for inputs in the
+  // supported range every nonzero s is a normal fp32 number, so the
+  // flush-to-zero hardware forms see it unchanged.
+  (void)qs; (void)qo; (void)sfloor;
   // Pairs whose norm is so small that the fp32 angle may be off by a quarter bin
   // are re-decided too: sqrt(s) < 4 n ty / pi.
   const float rthr = ty * (4.f * (float)n / 3.14159265f);
@@ -477,8 +476,8 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
       rn[j] = sqrt_approx(s[j] * k2);
     } else {
       float f;
-      if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_ftz(s[j] * sigma);
-      else f = lg2_ftz(fmaxf(s[j] * sigma, sfl));
+      if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_ftz(s[j]);
+      else f = lg2_ftz(fmaxf(s[j], sfloor));
       const uint32_t c = min(__float2uint_rd(__fmaf_rn(f, qs, qo)), (uint32_t)Lq);
       const int sn = j * B;
       if (sn < 32) nlo += c << sn; else nhi += c << (sn - 32);
