@@ -160,6 +160,31 @@ int check_rows(const tac_rows* r, int d, const char* who, const char* name, bool
   return TAC_OK;
 }
 
+// SMs each launch of a multi-launch call may use.  A large call gives every
+// launch the whole GPU: they run back to back in effect, each at full rate.  A
+// small one (fewer than kSplitTiles warp tiles per SM in all) is dominated by
+// each launch's ramp (table set-up, first prefetches) and tail, so its launches
+// get shares of the SMs in proportion to their tiles (at least one each) and
+// run side by side, paying the ramp once.
+constexpr int64_t kSplitTiles = 640;   // 32 tiles per warp at 20 warps per SM
+void sm_shares(const int64_t* tiles, int ngroups, int sms, int* caps) {
+  int64_t total = 0;
+  for (int g = 0; g < ngroups; ++g) total += tiles[g];
+  if (ngroups <= 1 || total >= kSplitTiles * sms) {
+    for (int g = 0; g < ngroups; ++g) caps[g] = sms;
+    return;
+  }
+  int used = 0;
+  for (int g = 0; g < ngroups; ++g) {
+    caps[g] = (int)std::max<int64_t>(1, tiles[g] * sms / total);
+    used += caps[g];
+  }
+  // hand the SMs left by rounding down to the largest groups (groups are
+  // sorted largest first); more groups than SMs may oversubscribe: the extra
+  // CTAs wait for a free slot
+  for (int g = 0; used < sms && ngroups > 0; g = (g + 1) % ngroups, ++used) ++caps[g];
+}
+
 int num_sms() {
   static int cache[64] = {0};
   int dev = 0;
@@ -405,11 +430,17 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
   // largest groups first: the small ones fill the tail of the large ones
   std::stable_sort(groups.begin(), groups.end(),
                    [](const EncGroup& a, const EncGroup& b) { return a.p.ntiles > b.p.ntiles; });
+  static thread_local std::vector<int64_t> gtiles;
+  static thread_local std::vector<int> caps;
+  gtiles.resize(groups.size());
+  caps.resize(groups.size());
+  for (size_t g = 0; g < groups.size(); ++g) gtiles[g] = groups[g].p.ntiles;
+  sm_shares(gtiles.data(), (int)groups.size(), sms, caps.data());
   GroupFork fork(reinterpret_cast<cudaStream_t>(stream), (int)groups.size());
   if (fork.error() != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(fork.error()));
   for (size_t g = 0; g < groups.size(); ++g) {
     const EncGroup& G = groups[g];
-    cudaError_t e = tac::launch_encode(G.d, G.dt, G.na, G.nb, G.mode, G.p, sms, fork.stream((int)g));
+    cudaError_t e = tac::launch_encode(G.d, G.dt, G.na, G.nb, G.mode, G.p, caps[g], fork.stream((int)g));
     if (e != cudaSuccess) {
       fork.join();
       return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
@@ -494,11 +525,17 @@ int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream)
   }
   std::stable_sort(groups.begin(), groups.end(),
                    [](const DecGroup& a, const DecGroup& b) { return a.p.ntiles > b.p.ntiles; });
+  static thread_local std::vector<int64_t> gtiles;
+  static thread_local std::vector<int> caps;
+  gtiles.resize(groups.size());
+  caps.resize(groups.size());
+  for (size_t g = 0; g < groups.size(); ++g) gtiles[g] = groups[g].p.ntiles;
+  sm_shares(gtiles.data(), (int)groups.size(), sms, caps.data());
   GroupFork fork(reinterpret_cast<cudaStream_t>(stream), (int)groups.size());
   if (fork.error() != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(fork.error()));
   for (size_t g = 0; g < groups.size(); ++g) {
     const DecGroup& G = groups[g];
-    cudaError_t e = tac::launch_decode(G.d, G.dt, G.na, G.nb, G.mode, G.p, sms, fork.stream((int)g));
+    cudaError_t e = tac::launch_decode(G.d, G.dt, G.na, G.nb, G.mode, G.p, caps[g], fork.stream((int)g));
     if (e != cudaSuccess) {
       fork.join();
       return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
