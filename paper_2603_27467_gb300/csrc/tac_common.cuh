@@ -57,14 +57,21 @@ struct Geo {
   static constexpr int L = P / kPairsPerThread;
   static constexpr int RW = 32 / L;
   static constexpr int LOGD = (D == 16) ? 4 : (D == 32) ? 5 : (D == 64) ? 6 : 7;
-  // Transpose buffer (L > 1): pair i of warp-tile row r at
-  //   r*ST + (i / L)*SM + (i % L)*8.
-  // Lane l writes pairs l + L*m (m = 0..7: offsets m*SM, a linear stride) and
-  // reads pairs 8l..8l+7 as four 16-byte granules at (8/L)*l*SM + fixed offsets.
-  // SM and ST are padded so both patterns are bank-conflict free (d = 32..128).
-  static constexpr int SM = 8 * L + 16;
-  static constexpr int ST = 8 * SM + (L == 8 ? 64 : 16);
+  // Transpose buffer (L > 1): pair i of warp-tile row r at r*ST + the offset
+  // of i in its pair row, (i / L)*SM + 8*((i % L) ^ s), where for L = 4 the two
+  // 16-byte granules of pair rows 4..7 trade places (s = 2 there, else 0).
+  // Two patterns use it: lane l touches pairs l + L*m (m = 0..7, 8-byte
+  // accesses at m*SM + 8*(l ^ swa(m))) and pairs 8l..8l+7 as four 16-byte
+  // granules (at (8/L)*l*SM + tp_pair(2q ^ swb(l))).  SM, ST and the swap make
+  // both patterns free of bank conflicts (a shared-memory model of 16-lane
+  // phases for 8-byte and 8-lane phases for 16-byte accesses: 16 wavefronts
+  // each per warp tile); for L = 4 no padding alone does (one of the two then
+  // takes 32).
+  static constexpr int SM = L == 8 ? 80 : L == 4 ? 32 : 16;
+  static constexpr int ST = L == 8 ? 704 : L == 4 ? 288 : 144;
   static constexpr int TP_W = (L > 1) ? RW * ST : 0;
+  __host__ __device__ static constexpr int swa(int m) { return L == 4 ? ((m >> 1) & 2) : 0; }
+  __host__ __device__ static constexpr int swb(int l) { return L == 4 ? (l & 2) : 0; }
   __host__ __device__ static constexpr int tp_pair(int i) { return (i / L) * SM + (i % L) * 8; }
 };
 

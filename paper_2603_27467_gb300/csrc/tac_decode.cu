@@ -209,11 +209,11 @@ __device__ __forceinline__ void decode_body(const uint8_t* rec, uint8_t* wsm, co
     uint8_t* tpl = tpr + (8 / L) * l * G::SM;
 #pragma unroll
     for (int q = 0; q < 4; ++q)
-      *reinterpret_cast<float4*>(tpl + G::tp_pair(2 * q)) =
+      *reinterpret_cast<float4*>(tpl + G::tp_pair((2 * q) ^ G::swb(l))) =
           make_float4(v[2 * q].x, v[2 * q].y, v[2 * q + 1].x, v[2 * q + 1].y);
     __syncwarp();
 #pragma unroll
-    for (int m = 0; m < 8; ++m) v[m] = *reinterpret_cast<const float2*>(tpr + m * G::SM + 8 * l);
+    for (int m = 0; m < 8; ++m) v[m] = *reinterpret_cast<const float2*>(tpr + m * G::SM + 8 * (l ^ G::swa(m)));
     // Stages on pair-index bits 3..log2(P)-1 (this lane now holds pairs l + L*m).
     butterfly8<8, 8 / L>(v);
   }

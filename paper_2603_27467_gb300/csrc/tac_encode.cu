@@ -354,12 +354,12 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
     // ---- transpose within the warp: lane l now owns pairs 8l..8l+7 ----
     uint8_t* tpr = wsm + C::W_TP + r * G::ST;
 #pragma unroll
-    for (int m = 0; m < 8; ++m) *reinterpret_cast<float2*>(tpr + m * G::SM + 8 * l) = v[m];
+    for (int m = 0; m < 8; ++m) *reinterpret_cast<float2*>(tpr + m * G::SM + 8 * (l ^ G::swa(m))) = v[m];
     __syncwarp();
     const uint8_t* tpl = tpr + (8 / L) * l * G::SM;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      const float4 t = *reinterpret_cast<const float4*>(tpl + G::tp_pair(2 * q));
+      const float4 t = *reinterpret_cast<const float4*>(tpl + G::tp_pair((2 * q) ^ G::swb(l)));
       v[2 * q] = make_float2(t.x, t.y);
       v[2 * q + 1] = make_float2(t.z, t.w);
     }
