@@ -23,8 +23,8 @@
 //      for atan on [-1, 1], max error 0.00496 rad), then the sign of the cross
 //      product of (E, O) with the edge direction.  The test is
 //      certified by a rigorous bound on the fp32 error; the pairs it does not
-//      certify are re-decided by the warp from error-free double-float sums of
-//      the staged input (no fp64: the FP64 pipe is a small fraction of fp32 here);
+//      certify (about 1e-4 of them) are re-decided by the warp from fp64 sums
+//      of the staged input;
 //   4. Eq. 2 norm codes (linear, or on log2 r) against the stored fp32 (r_min, r_max);
 //   5. each lane packs its 8 codes LSB-first; the warp stages its records in
 //      shared memory and writes them with one 16-byte store per lane (contiguous
@@ -33,23 +33,20 @@
 
 namespace tac {
 
-// Edge directions (cos psi_e, sin psi_e) for every supported n as double-float
-// pairs (c = ch + cl, s = sh + sl), read warp-uniformly by the exact path.
+// Edge directions (cos psi_e, sin psi_e) for every supported n in fp64, read
+// warp-uniformly by the exact path.
 namespace cx {
-struct DF4 { float ch, cl, sh, sl; };
-struct DFEdgeTable { DF4 v[kTabEntries]; };
-constexpr DFEdgeTable make_df_edge_table() {
-  DFEdgeTable t{};
+struct DEdgeTable { CS v[kTabEntries]; };
+constexpr DEdgeTable make_d_edge_table() {
+  DEdgeTable t{};
   for (int idx = 0; idx < kTabEntries; ++idx) {
     const int n = tab_n_of(idx), e = idx - tab_offset_n(n);
-    const CS d = cos_sin_q8(8 * e + 4 + n, n);
-    const float ch = (float)d.c, sh = (float)d.s;
-    t.v[idx] = DF4{ch, (float)(d.c - (double)ch), sh, (float)(d.s - (double)sh)};
+    t.v[idx] = cos_sin_q8(8 * e + 4 + n, n);
   }
   return t;
 }
 }  // namespace cx
-__constant__ cx::DFEdgeTable g_edge_df = cx::make_df_edge_table();
+__constant__ cx::DEdgeTable g_edge_d = cx::make_d_edge_table();
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles in flight
 // CTA shape of the encode: 10 warps, two CTAs per SM (20 warps, up to 102
@@ -125,13 +122,6 @@ __device__ __forceinline__ void store_bytes(uint8_t* dst, uint32_t lo, uint32_t 
   }
 }
 
-// Error-free transformation: s + e == a + b exactly (Knuth's TwoSum).
-__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
-  s = __fadd_rn(a, b);
-  const float bb = __fsub_rn(s, a);
-  e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
-}
-
 // v mod n for v in [-n, 2n).
 template <int N>
 __device__ __forceinline__ int wrap_bin(int v) {
@@ -205,12 +195,13 @@ __device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et
 // Exact re-decision of pair i of warp-tile row rr by the whole warp (all lanes
 // call it with the same arguments); returns k in every lane.  E_i = sum_j
 // +-x_2j and O_i = sum_j +-x_2j+1 (each term an exactly representable signed
-// input element) are accumulated as double-float values with TwoSum; their
-// relative error is of order 64 u^2, far inside the 1e-5 rad band the angle
-// parity tolerates.  The candidate edge comes from the polynomial on the sums
-// rounded to fp32 (scaled by a power of two when tiny, so the reciprocal sees
-// a normal number), the edge test m = E cos psi - O sin psi is evaluated in
-// double-float against the double-float edge direction.
+// input element) are summed in fp64 across the warp: relative error at most
+// (P - 1) 2^-53 of ||x||_1, far inside the 1e-5 rad band the angle parity
+// tolerates (the FP64 pipe is slow, but this path takes about 1e-4 of the
+// pairs).  The candidate edge comes from the fp32 polynomial on the sums
+// rounded to fp32 (scaled by a power of two when tiny, so that the reciprocal
+// sees a normal number); the edge test m = E cos psi - O sin psi is evaluated
+// in fp64 against the fp64 edge direction.
 template <int D, typename TIn, int N>
 __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uint8_t* in, int rr, int i,
                                                 int lane) {
@@ -218,7 +209,7 @@ __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uin
   using IT = RowTile<D, (int)sizeof(TIn)>;
   constexpr int ESZ = (int)sizeof(TIn);
   constexpr int P = G::P;
-  float eh = 0.f, el = 0.f, oh = 0.f, ol = 0.f;
+  double e = 0.0, o = 0.0;
   const int ip = slot_pair<D>(i);   // the pair held in slot i
   const uint8_t* row = in + rr * IT::STRIDE;
 #pragma unroll
@@ -237,39 +228,21 @@ __device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uin
       const bool neg = __popc((unsigned)(ip & jj)) & 1;
       if (((signs[e0 >> 5] >> (e0 & 31)) & 1u) != (uint32_t)neg) x0 = -x0;
       if (((signs[e1 >> 5] >> (e1 & 31)) & 1u) != (uint32_t)neg) x1 = -x1;
-      float t;
-      two_sum(eh, x0, eh, t); el = __fadd_rn(el, t);
-      two_sum(oh, x1, oh, t); ol = __fadd_rn(ol, t);
+      e += (double)x0;
+      o += (double)x1;
     }
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
-    const float a = __shfl_xor_sync(0xffffffffu, eh, off), b = __shfl_xor_sync(0xffffffffu, el, off);
-    const float c = __shfl_xor_sync(0xffffffffu, oh, off), d = __shfl_xor_sync(0xffffffffu, ol, off);
-    float t;
-    two_sum(eh, a, eh, t); el = __fadd_rn(__fadd_rn(el, b), t);
-    two_sum(oh, c, oh, t); ol = __fadd_rn(__fadd_rn(ol, d), t);
+    e += __shfl_xor_sync(0xffffffffu, e, off);
+    o += __shfl_xor_sync(0xffffffffu, o, off);
   }
-  two_sum(eh, el, eh, el);  // renormalize: eh == 0 now means E == 0
-  two_sum(oh, ol, oh, ol);
-  if (eh == 0.f && oh == 0.f) return 0;  // pair (0, 0) -> bin 0
-  if (fmaxf(fabsf(eh), fabsf(oh)) < 1e-30f) {  // exact power-of-two rescale
-    eh *= 18446744073709551616.f; el *= 18446744073709551616.f;
-    oh *= 18446744073709551616.f; ol *= 18446744073709551616.f;
-  }
-  const int e = candidate_edge<N>(eh, oh);
-  const cx::DF4 dir = g_edge_df.v[tab_offset_n(N) + e];
-  const float p1 = __fmul_rn(eh, dir.ch), q1 = __fmaf_rn(eh, dir.ch, -p1);
-  const float p2 = __fmul_rn(oh, dir.sh), q2 = __fmaf_rn(oh, dir.sh, -p2);
-  float dd, t;
-  two_sum(p1, -p2, dd, t);
-  float rest = __fadd_rn(t, __fsub_rn(q1, q2));
-  rest = __fmaf_rn(eh, dir.cl, rest);
-  rest = __fmaf_rn(el, dir.ch, rest);
-  rest = __fmaf_rn(-oh, dir.sl, rest);
-  rest = __fmaf_rn(-ol, dir.sh, rest);
-  const float m = __fadd_rn(dd, rest);
-  return wrap_bin<N>(e + (m >= 0.f ? 1 : 0));
+  if (e == 0.0 && o == 0.0) return 0;  // pair (0, 0) -> bin 0
+  const double sc = (fabs(e) + fabs(o) < 1e-30) ? 18446744073709551616.0 : 1.0;   // exact 2^64
+  const int ec = candidate_edge<N>((float)(e * sc), (float)(o * sc));
+  const cx::CS dir = g_edge_d.v[tab_offset_n(N) + ec];
+  const double m = fma(e, dir.c, -(o * dir.s));
+  return wrap_bin<N>(ec + (m >= 0.0 ? 1 : 0));
 }
 
 // Patch code i (W bits) of a staged angle record (one lane).
