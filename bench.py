@@ -2,15 +2,18 @@
 """TurboAngle KV-cache encode/decode benchmark on GB300 (libtac, sm_103a).
 
 One step = encode every (layer, K/V) block of a synthetic KV cache into packed
-records (tac_encode_multi, one launch) and decode every record back to bf16
-(tac_decode_multi, one launch).  Default workload: the Mistral-7B-shaped cache
+records (one tac_encode_multi call: one launch per kernel shape, run
+concurrently) and decode every record back to bf16 (one tac_decode_multi call).
+Default workload: the Mistral-7B-shaped cache
 (32 layers x 8 KV heads x 32768 tokens x d 128, bf16; early-boost n = 256 on
 layers 0-3, n = 64 elsewhere; K 8-bit linear / V 4-bit log norms).
 
 value = algorithmic bytes moved per step (bf16 rows in + packed records out for
 encode, records in + bf16 rows out for decode) / step time, summed over ranks.
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tac|reference]
-       [--config mistral7b|llama1b|append|longctx]
+       [--config mistral7b|llama1b|append|longctx|mistral7b_angle|mistral7b_norm8|
+                 tinyllama_n56|attend] [--tokens T] [--graph on|off]
+       [--no-e2e] [--no-cpu-baseline] [--probe rd]
 """
 from __future__ import annotations
 
