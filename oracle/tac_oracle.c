@@ -25,11 +25,14 @@
  *   R2 Rounding in Alg. 1: k = floor(n theta/(2 pi) + 1/2) mod n, theta in (-pi, pi]
  *      from atan2; a value exactly halfway rounds up.
  *   R3 A pair (0, 0) gets k = 0.
- *   R4 The stored header is (float)r_min, (float)r_max (round to nearest); Eq. 2 is
- *      evaluated against these stored values, in fp64, then rounded half up and
- *      clamped to [0, 2^b - 1].
- *   R5 If the stored r_max equals the stored r_min every norm code is 0 and decode
- *      returns r_min for every pair (an all-zero vector decodes to zero).
+ *   R4 Eq. 2 takes r_min and r_max as what the formula names: the minimum and the
+ *      maximum of the vector's pair norms themselves (their fp64 values here).  Sec. 3.3
+ *      stores the two in fp32 for the decoder: the header holds (float)r_min and
+ *      (float)r_max (round to nearest), and decode dequantizes against those stored
+ *      values.  Eq. 2's value is rounded half up and clamped to [0, 2^b - 1].
+ *   R5 If r_max equals r_min every norm code is 0; if the stored r_max equals the
+ *      stored r_min, decode returns the stored r_min for every pair (an all-zero vector
+ *      decodes to zero).
  *   R6 Log-space: norms are floored at 2^-24 * r_max before the logarithm (so a zero
  *      pair norm has a finite code) and the stored r_min is that floored minimum;
  *      log base 2.
@@ -142,7 +145,7 @@ static int32_t fp32_bits(double v) {
   return b;
 }
 
-/* Eq. 2 with clamp (reading R4); returns the pre-round value in *pre. */
+/* Eq. 2 with clamp (readings R4, R5); returns the pre-round value in *pre. */
 static int32_t norm_code(double val, double lo, double hi, int b, double* pre) {
   int32_t L = (1 << b) - 1;
   if (hi == lo) { *pre = 0.0; return 0; }           /* reading R5 */
@@ -200,25 +203,23 @@ int orc_encode(const double* x, int64_t rows, int d, const int8_t* s, int n, int
         if (pre) pre[i] = 0.0;
       }
     } else if (mode == 0) {
-      float hmin = (float)rmin, hmax = (float)rmax;        /* Sec. 3.3: fp32 min/max */
-      hdr_out[2 * row] = hmin;
-      hdr_out[2 * row + 1] = hmax;
+      hdr_out[2 * row] = (float)rmin;                         /* Sec. 3.3: stored in fp32 */
+      hdr_out[2 * row + 1] = (float)rmax;
       for (int i = 0; i < P; ++i) {
         double pv;
-        c_out[row * P + i] = norm_code(r[i], (double)hmin, (double)hmax, b, &pv);
+        c_out[row * P + i] = norm_code(r[i], rmin, rmax, b, &pv);   /* Eq. 2, reading R4 */
         if (pre) pre[i] = pv;
       }
     } else {
       double floor_r = ldexp(rmax, -24);                     /* reading R6 */
       double lo = rmin < floor_r ? floor_r : rmin;
-      float hmin = (float)lo, hmax = (float)rmax;
-      hdr_out[2 * row] = hmin;
-      hdr_out[2 * row + 1] = hmax;
-      double lmin = (hmin > 0.0f) ? log2((double)hmin) : 0.0;
-      double lmax = (hmax > 0.0f) ? log2((double)hmax) : 0.0;
+      hdr_out[2 * row] = (float)lo;                           /* Sec. 3.3: stored in fp32 */
+      hdr_out[2 * row + 1] = (float)rmax;
+      double lmin = (lo > 0.0) ? log2(lo) : 0.0;
+      double lmax = (rmax > 0.0) ? log2(rmax) : 0.0;
       for (int i = 0; i < P; ++i) {
         double pv;
-        if (hmax == hmin) {
+        if (rmax == lo) {                                     /* reading R5 */
           c_out[row * P + i] = 0;
           pv = 0.0;
         } else {

@@ -246,6 +246,112 @@ def test_norm_endpoints_and_error_bound(orc, b, mode):
         assert np.all(np.abs(lhat - lr) <= step[:, None] / 2 + 1e-6)
 
 
+def test_eq2_takes_the_exact_extremes(orc):
+    """Reading R4: Eq. 2 normalizes by the vector's own minimum and maximum norm,
+    so the argmax pair's value is exactly 2^b - 1 and the argmin pair's exactly 0
+    (against the fp32-rounded header they would be off by ~1e-8 relative).  The
+    header still holds the fp32 roundings of both."""
+    d = 128
+    w = workloads.CONFIGS["mistral7b"]
+    x = np.asarray(workloads.block(w, 2, 0, tokens=40).float().numpy(), dtype=np.float64)
+    rows = np.arange(len(x))
+    for b, mode in ((8, 0), (4, 1), (8, 1)):
+        s = orc.signs(0, 2, mode, d)
+        out = orc.encode(x, s, 64, b, mode)
+        r, pre = out["r"], out["pre"]
+        L = (1 << b) - 1
+        assert np.all(pre[rows, r.argmax(axis=1)] == L)
+        if mode == 0:
+            assert np.all(pre[rows, r.argmin(axis=1)] == 0.0)
+        assert np.array_equal(out["hdr"][:, 1], r.max(axis=1).astype(np.float32))
+        # rows whose extremes are not fp32 numbers exist, so the two readings differ here
+        assert np.any(r.max(axis=1) != r.max(axis=1).astype(np.float32).astype(np.float64))
+
+
+def _pairs_at_axes(orc, norms, n, s):
+    """Rows with pair i = norms[i] * (cos, sin)(2 pi k_i / n), k_i on the axes
+    (multiples of n/4), so that x = D H y is exact at d = 64 (H = +-1/8)."""
+    rows, P = norms.shape
+    rng = np.random.default_rng(7)
+    q = rng.integers(0, 4, size=(rows, P))
+    k = q * (n // 4)
+    y = np.zeros((rows, 2 * P))
+    y[:, 0::2] = norms * np.array([1.0, 0.0, -1.0, 0.0])[q]
+    y[:, 1::2] = norms * np.array([0.0, 1.0, 0.0, -1.0])[q]
+    return _x_from_y(orc, y, s), y, k
+
+
+@pytest.mark.parametrize("b,base", [(4, 0), (4, -10), (3, 5), (2, -3)])
+def test_log_dequant_exact_at_powers_of_two(orc, b, base):
+    """Sec. 3.3 log-space variant with reading R7: pair norms 2^(base + j),
+    j = 0 .. 2^b - 1 (both extremes present), span exactly 2^b - 1 octaves, so
+    Eq. 2 on log r gives the integer code j with no rounding, and decode must
+    return 2^(base + c) exactly: a wrong log base or exp base, 2^b instead of
+    2^b - 1 levels, or swapped l_min / l_max all break it."""
+    d, n = 64, 16
+    L = (1 << b) - 1
+    rng = np.random.default_rng(b * 100 + base)
+    j = rng.integers(0, L + 1, size=(12, d // 2))
+    j[:, 0], j[:, 1] = 0, L
+    s = orc.signs(0, 1, 1, d)
+    x, y, k = _pairs_at_axes(orc, 2.0 ** (base + j), n, s)
+    out = orc.encode(x, s, n, b, 1)
+    assert np.array_equal(out["c"], j.astype(np.int32))
+    assert np.array_equal(out["k"], k.astype(np.int32))
+    assert np.all(out["hdr"][:, 0] == np.float32(2.0**base)) and np.all(out["hdr"][:, 1] == np.float32(2.0 ** (base + L)))
+    xh = orc.decode(out["k"], out["c"], out["hdr"], s, n, b, 1)
+    assert np.allclose(xh, x, rtol=0, atol=1e-12 * np.abs(x).max())
+
+
+def test_log_dequant_floor(orc):
+    """Reading R6: norms below 2^-24 r_max are floored there before the log, and
+    the header's r_min is that floor.  With b = 2 and norms 2^0 .. 2^24 in steps
+    of 2^8 plus one pair at 2^-5, the floored pair takes code 0 and decodes to
+    the floor 2^0, the others decode exactly."""
+    d, n = 64, 16
+    j = np.tile(np.array([0, 8, 16, 24]), (3, 8)).astype(np.float64)
+    norms = 2.0**j
+    norms[:, 5] = 2.0**-5
+    s = orc.signs(2, 0, 1, d)
+    x, y, k = _pairs_at_axes(orc, norms, n, s)
+    out = orc.encode(x, s, n, 2, 1)
+    want = (j // 8).astype(np.int32)
+    want[:, 5] = 0
+    assert np.array_equal(out["c"], want)
+    assert np.all(out["hdr"][:, 0] == 1.0) and np.all(out["hdr"][:, 1] == np.float32(2.0**24))
+    xh = orc.decode(out["k"], out["c"], out["hdr"], s, n, 2, 1)
+    yh = orc.transform(xh, s)
+    rh = np.hypot(yh[:, 0::2], yh[:, 1::2])
+    expect = norms.copy()
+    expect[:, 5] = 1.0
+    # the re-transform rounds at the scale of the largest pair (2^24)
+    assert np.allclose(rh, expect, rtol=1e-12, atol=1e-12 * 2.0**24)
+
+
+@pytest.mark.parametrize("b", [4, 8])
+def test_log_dequant_half_step(orc, b):
+    """Decoded norms in log-space mode lie within half a log step of log2 r
+    (floored at 2^-24 r_max): |log2 r^ - log2 r| <= (l_max - l_min) / (2 (2^b - 1)),
+    up to the fp32 rounding of the stored header.  r^ is measured on the decoded
+    vector itself (y^ = H D x^), not recomputed from the codes."""
+    d, n = 128, 64
+    w = workloads.CONFIGS["mistral7b"]
+    x = np.asarray(workloads.block(w, 7, 1, tokens=48).float().numpy(), dtype=np.float64)
+    s = orc.signs(0, 7, 1, d)
+    out = orc.encode(x, s, n, b, 1)
+    xh = orc.decode(out["k"], out["c"], out["hdr"], s, n, b, 1)
+    yh = orc.transform(xh, s)
+    rh = np.hypot(yh[:, 0::2], yh[:, 1::2])
+    r = np.maximum(out["r"], out["r"].max(axis=1, keepdims=True) * 2.0**-24)
+    hmin, hmax = out["hdr"][:, 0].astype(np.float64), out["hdr"][:, 1].astype(np.float64)
+    half = (np.log2(hmax) - np.log2(hmin)) / (2 * ((1 << b) - 1))
+    err = np.abs(np.log2(rh) - np.log2(r))
+    assert np.all(err <= half[:, None] + 2e-7), float((err - half[:, None]).max())
+    assert np.all(rh >= hmin[:, None] * (1 - 1e-12)) and np.all(rh <= hmax[:, None] * (1 + 1e-12))
+    # the bound is attained up to a small factor (the test would catch a zero step)
+    assert float((err / half[:, None]).max()) > 0.9
+
+
 def test_norm_monotone(orc):
     d = 64
     rng = np.random.default_rng(9)
