@@ -122,14 +122,20 @@ typedef struct {
 
 /*
  * D of Sec. 2 ("s_i ~ Uniform{+1,-1}", sampled once from a seeded PRNG, Sec. 3.1
- * implementation note).  Counter-based SplitMix64 (Steele, Lea, Flood 2014):
- *   key = output #q of the SplitMix64 stream seeded with `seed`, q = 2*layer + kv
- *         (q = 0 when `shared` != 0: one D for every layer and K/V, as in the paper);
+ * implementation note), one per (layer, K/V).  Counter-based SplitMix64
+ * (Steele, Lea, Flood 2014):
+ *   key = output #q of the SplitMix64 stream seeded with `seed`, q = 2*layer + kv;
  *   s_j = -1 iff bit 63 of output #j of the stream seeded with key is set.
  * Output #i of the stream seeded with z is mix(z + (i+1)*0x9E3779B97F4A7C15).
- * Writes ceil(d/32) words (host memory).  kv: 0 = K, 1 = V.  Host only.
+ * Writes ceil(d/32) words (host memory; bit j of the little-endian word array
+ * set <=> s_j = -1).  kv: 0 = K, 1 = V.  Host only; TAC_E_INVAL for a NULL
+ * out_words, d outside 1..2^20, layer < 0 or kv not 0/1.
  */
-int tac_make_signs(uint64_t seed, int layer, int kv, int shared, int d, uint32_t* out_words);
+int tac_make_signs(uint64_t seed, int layer, int kv, int d, uint32_t* out_words);
+
+/* The paper's single D for every layer and K/V (Sec. 3.1 implementation note):
+ * the stream keyed by output #0, i.e. tac_make_signs' q = 0. */
+int tac_make_signs_shared(uint64_t seed, int d, uint32_t* out_words);
 
 /* Bytes per row of each plane (Sec. 3.1 rate: log2(n) bits per pair, stored in
  * ceil(log2 n) bits; Eq. 3 norm bits per pair; 64 bits of header per vector).
@@ -147,6 +153,20 @@ int64_t tac_norms_bytes(const tac_layer_cfg* cfg, int64_t capacity);
 double tac_avg_angle_bits(int num_layers, const int* n_k, const int* n_v);
 /* Eq. 3: b_angle + b_norm / 2 + 64 / d. */
 double tac_total_bits(double b_angle, double b_norm, int d);
+
+/*
+ * Rates of a per-layer schedule (n_k[l], n_v[l]) with norm bits b_k, b_v
+ * (Sec. 3.2, 3.3), written to out4 (host, 4 doubles):
+ *   [0] Eq. 1 angle bits per element;
+ *   [1] payload bits per element: [0] + (b_k + b_v) / 4 (norm bits per pair / 2,
+ *       averaged over K and V);
+ *   [2] Eq. 3 total: [0] + (b_k + b_v) / 4 + 64/d; with fp32 norms
+ *       (b_k = b_v = 32, Sec. 3.1) the payload itself (no min/max header);
+ *   [3] bits the angle codes occupy: ceil(log2 n) instead of log2 n.
+ * TAC_E_INVAL for a bad schedule (num_layers < 1, an n < 1, d < 1, norm bits
+ * outside 1..16 unless both are 32).
+ */
+int tac_rates(int num_layers, const int* n_k, const int* n_v, int b_k, int b_v, int d, double* out4);
 
 /*
  * Encode x.rows rows (Alg. 1 + Eq. 2) into record slots 0..x.rows-1 of
@@ -263,6 +283,15 @@ int tac_attend_multi_static(const tac_attend_job* jobs, int njobs, tac_stream_t 
  */
 int tac_fwht_debug(const tac_rows* x, int d, const uint32_t* signs, float* y,
                    tac_stream_t stream);
+
+/*
+ * The hardware approximations the kernels use, element-wise, for tests that
+ * measure them against the error bounds the encoder's certification assumes
+ * (the paper has no counterpart).  op: 0 sqrt.approx.f32, 1 sqrt.approx.ftz.f32,
+ * 2 rcp.approx.ftz.f32, 3 lg2.approx.f32, 4 lg2.approx.ftz.f32,
+ * 5 ex2.approx.ftz.f32.  x, y: n floats (device, 16-byte aligned).
+ */
+int tac_hw_approx_debug(int op, const float* x, float* y, int64_t n, tac_stream_t stream);
 
 /* Message of the last failed call on this host thread ("" if none). */
 const char* tac_last_error(void);

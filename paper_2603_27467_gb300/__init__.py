@@ -90,7 +90,11 @@ def load():
         i64, i32, vp = ctypes.c_int64, ctypes.c_int, ctypes.c_void_p
         P = ctypes.POINTER
         lib.tac_make_signs.restype = i32
-        lib.tac_make_signs.argtypes = [ctypes.c_uint64, i32, i32, i32, i32, P(ctypes.c_uint32)]
+        lib.tac_make_signs.argtypes = [ctypes.c_uint64, i32, i32, i32, P(ctypes.c_uint32)]
+        lib.tac_make_signs_shared.restype = i32
+        lib.tac_make_signs_shared.argtypes = [ctypes.c_uint64, i32, P(ctypes.c_uint32)]
+        lib.tac_rates.restype = i32
+        lib.tac_rates.argtypes = [i32, P(ctypes.c_int), P(ctypes.c_int), i32, i32, i32, P(ctypes.c_double)]
         for name in ("tac_angle_row_bytes", "tac_norm_row_bytes"):
             getattr(lib, name).restype = i64
             getattr(lib, name).argtypes = [P(_Cfg)]
@@ -117,6 +121,8 @@ def load():
         lib.tac_attend_multi_static.argtypes = [P(_AttJob), i32, vp]
         lib.tac_fwht_debug.restype = i32
         lib.tac_fwht_debug.argtypes = [P(_Rows), i32, P(ctypes.c_uint32), vp, vp]
+        lib.tac_hw_approx_debug.restype = i32
+        lib.tac_hw_approx_debug.argtypes = [i32, vp, vp, i64, vp]
         lib.tac_last_error.restype = ctypes.c_char_p
         lib.tac_last_error.argtypes = []
         lib.tac_version.restype = ctypes.c_char_p
@@ -162,8 +168,11 @@ class LayerCfg:
 def make_signs(seed: int, layer: int, kv: int, d: int, shared: bool = False) -> np.ndarray:
     """D of Sec. 2 for (layer, kv) as little-endian uint32 bit words (bit set => -1)."""
     words = np.zeros(max(1, (d + 31) // 32), dtype=np.uint32)
-    _check(load().tac_make_signs(seed & (2**64 - 1), layer, kv, int(shared), d,
-                                 words.ctypes.data_as(ctypes.POINTER(ctypes.c_uint32))))
+    out = words.ctypes.data_as(ctypes.POINTER(ctypes.c_uint32))
+    if shared:
+        _check(load().tac_make_signs_shared(seed & (2**64 - 1), d, out))
+    else:
+        _check(load().tac_make_signs(seed & (2**64 - 1), layer, kv, d, out))
     return words
 
 
@@ -478,20 +487,29 @@ def fwht_debug(x, signs: np.ndarray, d: int, stream=None):
     return y
 
 
+HW_SQRT, HW_SQRT_FTZ, HW_RCP_FTZ, HW_LG2, HW_LG2_FTZ, HW_EX2_FTZ = range(6)
+
+
+def hw_approx_debug(op: int, x, stream=None):
+    """tac_hw_approx_debug: the kernels' hardware approximation `op` applied to
+    the fp32 device tensor x, element-wise."""
+    torch = _torch()
+    x = x.contiguous()
+    y = torch.empty_like(x)
+    _check(load().tac_hw_approx_debug(op, x.data_ptr(), y.data_ptr(), x.numel(), _stream_ptr(stream)))
+    return y
+
+
 def rates(d: int, n_k, n_v, b_k: int = 8, b_v: int = 4) -> dict:
-    """Rate accounting for a per-layer schedule: Eq. 1 angle bits, payload bits
-    (angle + norm bits per pair / 2) and Eq. 3 totals (64/d min-max overhead).
-    With b_k = b_v = 32 (fp32 norms, Sec. 3.1) the total is the angle bits plus
-    16 bits per element and there is no min-max overhead; "stored_bits" counts
-    the ceil(log2 n) bits a code of a non-power-of-two n occupies."""
-    import math
-    b_angle = avg_angle_bits(n_k, n_v)
-    payload = b_angle + (b_k + b_v) / 4.0
-    fp32 = b_k == 32 and b_v == 32
-    total = payload if fp32 else total_bits(b_angle, (b_k + b_v) / 2.0, d)
-    stored = sum(math.ceil(math.log2(a)) + math.ceil(math.log2(b)) for a, b in zip(n_k, n_v)) / (4.0 * len(n_k))
-    return {"angle_bits": b_angle, "payload_bits": payload, "total_bits": total,
-            "stored_angle_bits": stored}
+    """tac_rates: Eq. 1 angle bits, payload bits (angle + norm bits per pair / 2),
+    Eq. 3 total (no min/max header with fp32 norms, b_k = b_v = 32) and the
+    ceil(log2 n) bits the angle codes occupy, for a per-layer schedule."""
+    L = len(n_k)
+    a = (ctypes.c_int * L)(*[int(v) for v in n_k])
+    b = (ctypes.c_int * L)(*[int(v) for v in n_v])
+    out = (ctypes.c_double * 4)()
+    _check(load().tac_rates(L, a, b, b_k, b_v, d, out))
+    return {"angle_bits": out[0], "payload_bits": out[1], "total_bits": out[2], "stored_angle_bits": out[3]}
 
 
 def early_boost(num_layers: int, boosted, n_early=(256, 128), base=(128, 64)):

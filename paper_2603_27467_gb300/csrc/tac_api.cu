@@ -74,6 +74,7 @@ cudaError_t launch_attend(int d, int dtype, int nq_max, const AttParams& p, int 
 cudaError_t attend_static_workspace(float** ws);
 cudaError_t launch_fwht_debug(int d, const void* x, int dtype, int64_t rows, int64_t stride,
                               const uint32_t* signs, float* y, cudaStream_t st);
+cudaError_t launch_hw_approx(int op, const float* x, float* y, int64_t n, int sms, cudaStream_t st);
 }  // namespace tac
 
 namespace {
@@ -218,18 +219,32 @@ const char* tac_last_error(void) { return g_err.c_str(); }
 
 const char* tac_version(void) { return "libtac 0.1.0 (TurboAngle encode/decode, sm_103a)"; }
 
-int tac_make_signs(uint64_t seed, int layer, int kv, int shared, int d, uint32_t* out_words) {
-  if (!out_words) return fail(TAC_E_INVAL, "tac_make_signs: out_words is NULL");
-  if (d < 1 || d > (1 << 20)) return fail(TAC_E_INVAL, "tac_make_signs: d = %d", d);
-  if (layer < 0) return fail(TAC_E_INVAL, "tac_make_signs: layer = %d", layer);
-  if (kv != 0 && kv != 1) return fail(TAC_E_INVAL, "tac_make_signs: kv = %d (0 = K, 1 = V)", kv);
-  const uint64_t q = shared ? 0u : (uint64_t)(2 * (int64_t)layer + kv);
+}  // extern "C"
+
+namespace {
+// Sign words of the stream keyed by output #q of the SplitMix64 stream seeded with seed.
+int make_signs_q(const char* who, uint64_t seed, uint64_t q, int d, uint32_t* out_words) {
+  if (!out_words) return fail(TAC_E_INVAL, "%s: out_words is NULL", who);
+  if (d < 1 || d > (1 << 20)) return fail(TAC_E_INVAL, "%s: d = %d", who, d);
   const uint64_t key = splitmix64(seed, q);
   const int nw = (d + 31) / 32;
   for (int i = 0; i < nw; ++i) out_words[i] = 0u;
   for (int j = 0; j < d; ++j)
     if (splitmix64(key, (uint64_t)j) >> 63) out_words[j >> 5] |= 1u << (j & 31);
   return ok();
+}
+}  // namespace
+
+extern "C" {
+
+int tac_make_signs(uint64_t seed, int layer, int kv, int d, uint32_t* out_words) {
+  if (layer < 0) return fail(TAC_E_INVAL, "tac_make_signs: layer = %d", layer);
+  if (kv != 0 && kv != 1) return fail(TAC_E_INVAL, "tac_make_signs: kv = %d (0 = K, 1 = V)", kv);
+  return make_signs_q("tac_make_signs", seed, (uint64_t)(2 * (int64_t)layer + kv), d, out_words);
+}
+
+int tac_make_signs_shared(uint64_t seed, int d, uint32_t* out_words) {
+  return make_signs_q("tac_make_signs_shared", seed, 0u, d, out_words);
 }
 
 int64_t tac_angle_row_bytes(const tac_layer_cfg* cfg) {
@@ -270,6 +285,24 @@ double tac_avg_angle_bits(int num_layers, const int* n_k, const int* n_v) {
 double tac_total_bits(double b_angle, double b_norm, int d) {
   if (d <= 0) return NAN;
   return b_angle + b_norm / 2.0 + 64.0 / (double)d;
+}
+
+int tac_rates(int num_layers, const int* n_k, const int* n_v, int b_k, int b_v, int d, double* out4) {
+  static const char* who = "tac_rates";
+  if (!out4) return fail(TAC_E_INVAL, "%s: out4 is NULL", who);
+  if (num_layers <= 0 || !n_k || !n_v || d <= 0) return fail(TAC_E_INVAL, "%s: bad schedule", who);
+  const bool fp32 = b_k == 32 && b_v == 32;
+  if (!fp32 && (b_k < 1 || b_k > 16 || b_v < 1 || b_v > 16))
+    return fail(TAC_E_INVAL, "%s: norm bits %d / %d (1..16, or 32 for fp32 norms)", who, b_k, b_v);
+  const double angle = tac_avg_angle_bits(num_layers, n_k, n_v);
+  if (std::isnan(angle)) return fail(TAC_E_INVAL, "%s: a codebook size is < 1", who);
+  double stored = 0.0;
+  for (int l = 0; l < num_layers; ++l) stored += tac::code_bits(n_k[l]) + tac::code_bits(n_v[l]);
+  out4[0] = angle;                                   // Eq. 1
+  out4[1] = angle + (b_k + b_v) / 4.0;               // payload: angle + norm bits per pair / 2
+  out4[2] = fp32 ? out4[1] : tac_total_bits(angle, (b_k + b_v) / 2.0, d);   // Eq. 3
+  out4[3] = stored / (4.0 * num_layers);             // bits the angle codes occupy
+  return ok();
 }
 
 namespace {
@@ -780,6 +813,19 @@ int tac_fwht_debug(const tac_rows* x, int d, const uint32_t* signs, float* y, ta
   if (d < 32) s[0] &= (1u << d) - 1u;
   cudaError_t e = tac::launch_fwht_debug(d, x->data, x->dtype, x->rows, x->row_stride, s, y,
                                          reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+  return ok();
+}
+
+int tac_hw_approx_debug(int op, const float* x, float* y, int64_t n, tac_stream_t stream) {
+  static const char* who = "tac_hw_approx_debug";
+  if (op < 0 || op > 5) return fail(TAC_E_INVAL, "%s: op = %d (0..5)", who, op);
+  if (n < 0) return fail(TAC_E_INVAL, "%s: n = %lld", who, (long long)n);
+  if (n == 0) return ok();
+  if (!x || !y || !aligned16(x) || !aligned16(y)) return fail(TAC_E_INVAL, "%s: x or y is NULL or misaligned", who);
+  const int sms = num_sms();
+  if (sms <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
+  cudaError_t e = tac::launch_hw_approx(op, x, y, n, sms, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
   return ok();
 }

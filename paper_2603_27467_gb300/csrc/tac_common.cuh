@@ -108,6 +108,17 @@ __host__ __device__ constexpr int slot_pair(int v) {
   }
 }
 
+// The slot that holds pair i (the inverse of slot_pair).
+template <int D>
+__host__ __device__ constexpr int pair_slot(int i) {
+  if constexpr (run_layout<D>()) {
+    constexpr int L = D / 16;
+    return (i / 4) % L + L * ((i % 4) + 4 * (i / (4 * L)));
+  } else {
+    return i;
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Device job descriptors (kernel parameters, copied by value at launch).
 // ---------------------------------------------------------------------------

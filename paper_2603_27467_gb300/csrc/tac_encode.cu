@@ -23,9 +23,12 @@
 //      for atan on [-1, 1], max error 0.00496 rad), then the sign of the cross
 //      product of (E, O) with the edge direction.  The test is
 //      certified by a rigorous bound on the fp32 error; the pairs it does not
-//      certify (about 1e-4 of them) are re-decided by the warp from fp64 sums
-//      of the staged input;
-//   4. Eq. 2 norm codes (linear, or on log2 r) against the stored fp32 (r_min, r_max);
+//      certify (about 1e-4 of them) are re-decided by the warp from exact
+//      sums of the staged input;
+//   4. Eq. 2 norm codes (linear, or on log2 r) against the row's minimum and
+//      maximum pair norms; a code whose fp32 Eq. 2 value lies within a band
+//      of a rounding midpoint is re-decided from exact sums as well, and the
+//      fp32 extremes are stored as the header (r_min, r_max);
 //   5. each lane packs its 8 codes LSB-first; the warp stages its records in
 //      shared memory and writes them with one 16-byte store per lane (contiguous
 //      slots) or per row (scatter-append slots).
@@ -33,27 +36,31 @@
 
 namespace tac {
 
-// Edge directions (cos psi_e, sin psi_e) for every supported n in fp64, read
+// Edge directions (cos psi_e, sin psi_e) for every supported n as double-float
+// pairs (c_hi, c_lo, s_hi, s_lo), built in fp64 by the host compiler and read
 // warp-uniformly by the exact path.
 namespace cx {
-struct DEdgeTable { CS v[kTabEntries]; };
-constexpr DEdgeTable make_d_edge_table() {
-  DEdgeTable t{};
+struct DfEdgeTable { float4 v[kTabEntries]; };
+constexpr DfEdgeTable make_df_edge_table() {
+  DfEdgeTable t{};
   for (int idx = 0; idx < kTabEntries; ++idx) {
     const int n = tab_n_of(idx), e = idx - tab_offset_n(n);
-    t.v[idx] = cos_sin_q8(8 * e + 4 + n, n);
+    const CS cs = cos_sin_q8(8 * e + 4 + n, n);
+    const float ch = (float)cs.c, sh = (float)cs.s;
+    t.v[idx] = float4{ch, (float)(cs.c - (double)ch), sh, (float)(cs.s - (double)sh)};
   }
   return t;
 }
 }  // namespace cx
-__constant__ cx::DEdgeTable g_edge_d = cx::make_d_edge_table();
+__constant__ cx::DfEdgeTable g_edge_df = cx::make_df_edge_table();
 
 constexpr int kNS = 4;  // pipeline stages per warp: kNS - 1 warp tiles in flight
-// CTA shape of the encode: 10 warps, two CTAs per SM (20 warps, up to 102
-// registers a thread): the encode is issue-bound, and the extra warps hide
-// more latency than the 128-register build's longer chains (3 % faster; 12
-// warps at 80 registers emit more instructions).
-constexpr int kEncWarps = 10;
+constexpr int kQ = 96;  // entries of a warp's re-decision queue
+// CTA shape of the encode: 8 warps, two CTAs per SM (16 warps, up to 128
+// registers a thread).  10-warp CTAs (up to 96 registers) issued about 3 %
+// faster before the re-decision queue, whose bookkeeping no longer fits in 96
+// registers without spills in the main loop.
+constexpr int kEncWarps = 8;
 constexpr int kEncThreads = 32 * kEncWarps;
 
 // Shape of one kernel: n bins (W = ceil(log2 n) bits per angle code), B norm
@@ -84,13 +91,19 @@ struct Enc {
   static constexpr int W_NRM = W_ANG + RW * AB;
   static constexpr int W_HDR = W_NRM + RW * NB;
   static constexpr int W_JOB = W_HDR + RW * HB;             // current job (WarpJob)
-  static constexpr int WARP_B = W_JOB + 64;
+  static constexpr int W_RC = W_JOB + 64;                    // the rows' fp32 (smin, smax, ty) for the queue
+  static constexpr int W_Q = W_RC + RW * 16;                 // re-decision queue (kQ entries of 32 bytes)
+  static constexpr int WARP_B = W_Q + kQ * 32;
+  // scratch of the queue's exact path (2P longs), free between tiles: the
+  // transpose rows, or for d = 16 (no transpose) the staged records
+  static constexpr int W_SCR = (G::TP_W >= 16 * P) ? W_TP : W_ANG;
   static constexpr int TABR = tab_copies(n, 8192);           // edge table copies
   static constexpr int OFF_TAB = kEncWarps * WARP_B;           // fp32 edge table of this n (TABR copies)
   static constexpr int SMEM = OFF_TAB + n * TABR * 8;
   static_assert((RW * AB) % 16 == 0 && (RW * NB) % 16 == 0 && (RW * HB) % 16 == 0, "record segments");
   static_assert(W_TP % 16 == 0 && W_ANG % 16 == 0 && W_JOB % 16 == 0 && WARP_B % 16 == 0, "alignment");
   static_assert(32 % CPR == 0 && RW % RPQ == 0, "chunk map");
+  static_assert(G::TP_W >= 16 * P || RW * (AB + NB + HB) >= 16 * P, "queue scratch");
 };
 
 // The job a warp is encoding as far as the rare paths need it (exact
@@ -102,6 +115,7 @@ struct WarpJob {
   const int64_t* slot;
   int64_t capacity;
   uint32_t signs[4];
+  int32_t job;         // its index in the launch's job table
 };
 static_assert(sizeof(WarpJob) <= 64, "WarpJob");
 
@@ -192,69 +206,504 @@ __device__ __forceinline__ uint32_t edge_test(float E, float O, const float2* et
   }
 }
 
-// Exact re-decision of pair i of warp-tile row rr by the whole warp (all lanes
-// call it with the same arguments); returns k in every lane.  E_i = sum_j
-// +-x_2j and O_i = sum_j +-x_2j+1 (each term an exactly representable signed
-// input element) are summed in fp64 across the warp: relative error at most
-// (P - 1) 2^-53 of ||x||_1, far inside the 1e-5 rad band the angle parity
-// tolerates (the FP64 pipe is slow, but this path takes about 1e-4 of the
-// pairs).  The candidate edge comes from the fp32 polynomial on the sums
-// rounded to fp32 (scaled by a power of two when tiny, so that the reciprocal
-// sees a normal number); the edge test m = E cos psi - O sin psi is evaluated
-// in fp64 against the fp64 edge direction.
-template <int D, typename TIn, int N>
-__device__ __forceinline__ int exact_angle_code(const uint32_t* signs, const uint8_t* in, int rr, int i,
-                                                int lane) {
-  using G = Geo<D>;
-  using IT = RowTile<D, (int)sizeof(TIn)>;
-  constexpr int ESZ = (int)sizeof(TIn);
-  constexpr int P = G::P;
-  double e = 0.0, o = 0.0;
-  const int ip = slot_pair<D>(i);   // the pair held in slot i
-  const uint8_t* row = in + rr * IT::STRIDE;
-#pragma unroll
-  for (int j0 = 0; j0 < P; j0 += 32) {
-    const int jj = j0 + lane;
-    if (jj < P) {
-      const int e0 = 2 * jj, e1 = 2 * jj + 1;
-      float x0, x1;
-      if constexpr (ESZ == 2) {
-        const uint32_t u = *reinterpret_cast<const uint32_t*>(row + 4 * jj);
-        x0 = bf16lo(u); x1 = bf16hi(u);
-      } else {
-        const float2 u = *reinterpret_cast<const float2*>(row + 8 * jj);
-        x0 = u.x; x1 = u.y;
-      }
-      const bool neg = __popc((unsigned)(ip & jj)) & 1;
-      if (((signs[e0 >> 5] >> (e0 & 31)) & 1u) != (uint32_t)neg) x0 = -x0;
-      if (((signs[e1 >> 5] >> (e1 & 31)) & 1u) != (uint32_t)neg) x1 = -x1;
-      e += (double)x0;
-      o += (double)x1;
-    }
-  }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    e += __shfl_xor_sync(0xffffffffu, e, off);
-    o += __shfl_xor_sync(0xffffffffu, o, off);
-  }
-  if (e == 0.0 && o == 0.0) return 0;  // pair (0, 0) -> bin 0
-  const double sc = (fabs(e) + fabs(o) < 1e-30) ? 18446744073709551616.0 : 1.0;   // exact 2^64
-  const int ec = candidate_edge<N>((float)(e * sc), (float)(o * sc));
-  const cx::CS dir = g_edge_d.v[tab_offset_n(N) + ec];
-  const double m = fma(e, dir.c, -(o * dir.s));
-  return wrap_bin<N>(ec + (m >= 0.0 ? 1 : 0));
+// ---------------------------------------------------------------------------
+// Exact path.  The butterfly halves E_i = sum_j +-x_2j and O_i = sum_j +-x_2j+1
+// of a pair are sums of exactly representable signed input elements; they are
+// formed exactly in 64-bit fixed point (integer adds on the ALU: the FP64 pipe
+// of this part is too slow for a path that runs on a few rows in a hundred)
+// and the decisions are then taken in double-float arithmetic (pairs of fp32,
+// about 46 significant bits).
+// ---------------------------------------------------------------------------
+
+// One input element (bf16 or fp32 bits), D and its own sign applied, as a
+// 64-bit fixed-point number on the scale of the row's largest exponent field
+// emax: element = X 2^(emax - K - bias).  K = 47 (bf16) or 31 (fp32) leaves
+// room for the sum of d/2 terms; an element more than 2^K below the largest
+// loses its bits below the scale (each sum then within d/2 2^-K of the
+// largest element).
+template <typename TIn>
+__device__ __forceinline__ long long fix_elem(uint32_t bits, int emax, uint32_t neg) {
+  constexpr bool BF = sizeof(TIn) == 2;
+  constexpr int MB = BF ? 7 : 23, K = BF ? 47 : 31;
+  const int e = (int)((bits >> MB) & 0xFFu);
+  const uint32_t m = (bits & ((1u << MB) - 1u)) | (e != 0 ? (1u << MB) : 0u);
+  const int sh = max(e, 1) - emax + K;
+  long long x = sh >= 0 ? ((long long)m << sh) : (sh > -(MB + 1) ? (long long)(m >> -sh) : 0ll);
+  return neg ? -x : x;
 }
 
-// Patch code i (W bits) of a staged angle record (one lane).
-template <int W>
-__device__ __forceinline__ void patch_code(uint8_t* rec, int i, int k) {
-  const int bit = i * W, b0 = bit >> 3, sh = bit & 7;
-  const uint32_t mask = ((1u << W) - 1u) << sh;
-  uint32_t v = rec[b0];
-  if (sh + W > 8) v |= (uint32_t)rec[b0 + 1] << 8;
-  v = (v & ~mask) | ((uint32_t)k << sh);
-  rec[b0] = (uint8_t)v;
-  if (sh + W > 8) rec[b0 + 1] = (uint8_t)(v >> 8);
+// ---- double-float arithmetic (x + y, |y| <= ulp(x)/2) ----
+__device__ __forceinline__ float2 df_fast2sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  return make_float2(s, __fadd_rn(b, __fsub_rn(a, s)));
+}
+__device__ __forceinline__ float2 df_add(float2 a, float2 b) {
+  const float s = __fadd_rn(a.x, b.x);
+  const float bb = __fsub_rn(s, a.x);
+  const float e = __fadd_rn(__fsub_rn(a.x, __fsub_rn(s, bb)), __fsub_rn(b.x, bb));
+  return df_fast2sum(s, __fadd_rn(e, __fadd_rn(a.y, b.y)));
+}
+__device__ __forceinline__ float2 df_neg(float2 a) { return make_float2(-a.x, -a.y); }
+__device__ __forceinline__ float2 df_mul(float2 a, float2 b) {
+  const float p = __fmul_rn(a.x, b.x);
+  float e = __fmaf_rn(a.x, b.x, -p);
+  e = __fmaf_rn(a.x, b.y, __fmaf_rn(a.y, b.x, e));
+  return df_fast2sum(p, e);
+}
+__device__ __forceinline__ float2 df_mulf(float2 a, float b) {
+  const float p = __fmul_rn(a.x, b);
+  return df_fast2sum(p, __fmaf_rn(a.y, b, __fmaf_rn(a.x, b, -p)));
+}
+__device__ __forceinline__ float2 df_div(float2 a, float2 b) {
+  const float r = rcp_approx(b.x);                       // b.x normal and nonzero at every caller
+  const float q1 = __fmul_rn(a.x, r);
+  const float2 res = df_add(a, df_neg(df_mulf(b, q1)));  // a - q1 b
+  return df_fast2sum(q1, __fmul_rn(res.x, r));
+}
+__device__ __forceinline__ float2 df_sqrt(float2 a) {
+  if (!(a.x > 0.f)) return make_float2(0.f, 0.f);
+  const float r = sqrt_approx(a.x);
+  const float d = __fadd_rn(__fmaf_rn(-r, r, a.x), a.y);
+  return df_fast2sum(r, __fmul_rn(d, 0.5f * rcp_approx(r)));
+}
+__device__ __forceinline__ int df_sign(float2 a) {
+  const float v = a.x != 0.f ? a.x : a.y;
+  return v > 0.f ? 1 : (v < 0.f ? -1 : 0);
+}
+// a < b for normalized double-floats (|lo| <= ulp(hi) / 2, as every
+// operation here returns them): the leading parts decide unless equal.
+__device__ __forceinline__ bool df_less(float2 a, float2 b) { return a.x < b.x || (a.x == b.x && a.y < b.y); }
+// 2^k for -126 <= k <= 127, and x 2^k for results in the normal range.
+__device__ __forceinline__ float pow2i(int k) { return __uint_as_float((uint32_t)(127 + k) << 23); }
+__device__ __forceinline__ float2 df_scale(float2 a, int k) {   // a 2^k, |k| <= 126, normal results
+  const float f = pow2i(k);
+  return make_float2(a.x * f, a.y * f);
+}
+
+// A 64-bit integer as a double-float (its top 48 significant bits; exact below 2^48).
+__device__ __forceinline__ float2 ll_to_df(long long v) {
+  if (v == 0) return make_float2(0.f, 0.f);
+  const bool neg = v < 0;
+  const unsigned long long u = neg ? (unsigned long long)(-v) : (unsigned long long)v;
+  const int lz = __clzll((long long)u);
+  const unsigned long long w = u << lz;                  // leading one at bit 63
+  const float hi = (float)(uint32_t)(w >> 40) * pow2i(40 - lz);             // 24 bits: exact
+  const float lo = (float)(uint32_t)((w >> 16) & 0xFFFFFFull) * pow2i(16 - lz);
+  return neg ? make_float2(-hi, -lo) : make_float2(hi, lo);
+}
+
+// Pair energy E^2 + O^2 in double-float from the exact sums.
+__device__ __forceinline__ float2 df_energy(longlong2 eo) {
+  const float2 e = ll_to_df(eo.x), o = ll_to_df(eo.y);
+  return df_add(df_mul(e, e), df_mul(o, o));
+}
+
+// Exact angle code (Alg. 1) of a pair from its exact sums: the candidate edge
+// from the fp32 polynomial on the leading parts, then the edge test
+// m = E cos psi - O sin psi in double-float against the double-float edge
+// direction (the code is the next bin when m >= 0).
+template <int N>
+__device__ __forceinline__ int fix_angle_code(longlong2 eo) {
+  if (eo.x == 0 && eo.y == 0) return 0;  // pair (0, 0) -> bin 0
+  const float2 e = ll_to_df(eo.x), o = ll_to_df(eo.y);
+  const int ec = candidate_edge<N>(e.x, o.x);
+  const float4 dir = g_edge_df.v[tab_offset_n(N) + ec];
+  const float2 m = df_add(df_mul(e, make_float2(dir.x, dir.y)), df_neg(df_mul(o, make_float2(dir.z, dir.w))));
+  return wrap_bin<N>(ec + (df_sign(m) >= 0 ? 1 : 0));
+}
+
+// log2 of a double-float >= 1, to about 2e-7 absolute: exponent plus log2 of
+// the leading part's significand plus the first-order term of the tail.
+__device__ __forceinline__ float df_log2_est(float2 a) {
+  const int e = (int)((__float_as_uint(a.x) >> 23) & 0xFFu) - 127;
+  const float mh = a.x * pow2i(-e), ml = a.y * pow2i(-e);
+  return (float)e + log2f(mh) + ml / mh * 1.4426950408889634f;
+}
+
+// The exponent of a positive normal fp32 number.
+__device__ __forceinline__ int f32_exp(float x) { return (int)((__float_as_uint(x) >> 23) & 0xFFu) - 127; }
+
+// a^n for a double-float a >= 1 and n >= 0, as m 2^e with m in [1, 2) (a
+// double-float) and an integer e: every product is brought back to [1, 2),
+// so nothing overflows for any n the codes need (n <= 2 * 255 + 1).
+__device__ __forceinline__ void df_pow(float2 a, int n, float2& m, int& e) {
+  int eb = f32_exp(a.x);
+  float2 b = df_scale(a, -eb);
+  m = make_float2(1.f, 0.f);
+  e = 0;
+  while (n) {
+    if (n & 1) {
+      m = df_mul(m, b);
+      e += eb;
+      const int k = f32_exp(m.x);
+      m = df_scale(m, -k);
+      e += k;
+    }
+    n >>= 1;
+    if (n) {
+      b = df_mul(b, b);
+      eb *= 2;
+      const int k = f32_exp(b.x);
+      b = df_scale(b, -k);
+      eb += k;
+    }
+  }
+}
+
+// rho1^n1 >= rho2^n2 for double-floats rho >= 1 and n >= 0.
+__device__ __forceinline__ bool df_pow_ge(float2 r1, int n1, float2 r2, int n2) {
+  float2 m1, m2;
+  int e1, e2;
+  df_pow(r1, n1, m1, e1);
+  df_pow(r2, n2, m2, e2);
+  if (e1 != e2) return e1 > e2;                          // both significands in [1, 2)
+  return !df_less(m1, m2);
+}
+
+// Eq. 2 code of a pair from double-float energies s = E^2 + O^2 (unnormalized:
+// r^2 = 2 s / d, a common factor that cancels): the pair's (sa) and the row's
+// minimum and maximum.  Linear: Lq (r - r_min) / (r_max - r_min); log-space:
+// the same on log2 r with norms floored at 2^-24 r_max (log2 r = (log2 s +
+// log2(2/d)) / 2: the ratio is taken on the energies); rounded half up and
+// clamped; 0 when r_max = r_min (Sec. 3.3, Eq. 2 and its log-space variant).
+// A code is c = max{c : the value >= c - 1/2}; an estimate (double-float
+// for linear, log2 estimates for log-space) gives c, and only when it lies
+// too close to a boundary for its own error is that boundary tested exactly:
+// linear by the sign of Lq (r - r_min) - (c - 1/2)(r_max - r_min) in
+// double-float; log-space by (s/s_lo)^(2 Lq) >= (s_max/s_lo)^(2c - 1), the
+// same inequality raised to integer powers.
+template <int B, int MODE>
+__device__ __forceinline__ int fix_norm_code(float2 sa, float2 smn, float2 smx) {
+  constexpr int Lq = (1 << B) - 1;
+  int c;
+  if constexpr (MODE == TAC_NORM_LINEAR) {
+    const float2 a = df_sqrt(sa), m = df_sqrt(smn), M = df_sqrt(smx);
+    const float2 A = df_add(a, df_neg(m)), R = df_add(M, df_neg(m));
+    if (!(R.x > 0.f)) return 0;                          // r_max = r_min
+    auto at_least = [&](int cc) {                        // value >= cc - 1/2
+      return df_sign(df_add(df_mulf(A, (float)Lq), df_neg(df_mulf(R, (float)cc - 0.5f)))) >= 0;
+    };
+    const float2 w = df_add(df_div(df_mulf(A, (float)Lq), R), make_float2(0.5f, 0.f));
+    c = (int)floorf(w.x);
+    const float fr = __fadd_rn(__fsub_rn(w.x, (float)c), w.y);   // the double-float value is good to 1e-9
+    if (fr > 1e-6f && fr < 1.f - 1e-6f) return min(max(c, 0), Lq);
+    c = min(max(c, 0), Lq);
+    while (c > 0 && !at_least(c)) --c;
+    while (c < Lq && at_least(c + 1)) ++c;
+  } else {
+    const float2 fl = df_scale(smx, -48);                // (2^-24 r_max)^2
+    const float2 lo = df_less(smn, fl) ? fl : smn;
+    const float2 aa = df_less(sa, fl) ? fl : sa;
+    if (!df_less(lo, smx)) return 0;                     // r_max = r_lo
+    const float2 r1 = df_div(aa, lo), r2 = df_div(smx, lo);   // >= 1
+    auto at_least = [&](int cc) { return df_pow_ge(r1, 2 * Lq, r2, 2 * cc - 1); };
+    const float l2 = df_log2_est(r2);
+    const float v = __fmaf_rn((float)Lq, df_log2_est(r1) / l2, 0.5f);
+    c = (int)floorf(v);
+    const float fr = v - (float)c;
+    const float tol = (float)Lq * 1e-6f / l2 + 1e-5f;      // the two estimates are good to 2e-7 each
+    if (fr > tol && fr < 1.f - tol) return min(max(c, 0), Lq);
+    c = min(max(c, 0), Lq);
+    while (c > 0 && !at_least(c)) --c;
+    while (c < Lq && at_least(c + 1)) ++c;
+  }
+  return c;
+}
+
+// Set bits [bit, bit + w) (w <= 8) of the byte stream at base to code, in
+// global memory.  Atomic on the aligned words they touch, so lanes that patch
+// different codes of one word do not lose each other's bits.
+__device__ __forceinline__ void patch_bits(uint8_t* base, int bit, int w, uint32_t code) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(base) + (uintptr_t)(bit >> 3);
+  uint32_t* word = reinterpret_cast<uint32_t*>(a & ~(uintptr_t)3);
+  const int sh = (int)(a & 3u) * 8 + (bit & 7);
+  const int n0 = min(w, 32 - sh);
+  const uint32_t m0 = ((1u << n0) - 1u) << sh;
+  atomicAnd(word, ~m0);
+  atomicOr(word, (code << sh) & m0);
+  if (n0 < w) {
+    const uint32_t m1 = (1u << (w - n0)) - 1u;
+    atomicAnd(word + 1, ~m1);
+    atomicOr(word + 1, (code >> n0) & m1);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Re-decision queue.  The main loop only notes the codes its bands could not
+// settle (a few in ten thousand); each warp keeps them in a queue in its
+// shared memory and works through it between tiles when it fills up, and at
+// the end.  Doing so outside the tile body keeps the body's registers and
+// instructions free of the rare path; the records, written already, are
+// patched in place.  An entry (32 bytes): job | slot << 8 | kind << 14, the
+// row in the job, and for a norm code its pair energy s and the row's smin,
+// smax and ty of the fast path.  kind: 0 an angle code, 1 a norm code, 2 the
+// whole row (rows with more flagged codes than kRowEntries, or whose norm
+// band is too wide to be useful), 3 settled.
+// ---------------------------------------------------------------------------
+template <int D>
+struct QGeo {
+  static constexpr int RW = Geo<D>::RW;
+  static constexpr int kRowEntries = (32 / RW) > 1 ? 32 / RW : 1;   // per row before it goes whole
+  static constexpr int kMaxPerTile = RW * kRowEntries;              // <= 32
+};
+
+// The part of the norm band left once the fast path's own arithmetic is taken
+// out: kKappa times the first-order bound of the transform (see tile_body).
+template <int D>
+__device__ __forceinline__ constexpr float norm_kappa() { return D >= 64 ? 0.015625f : 0.25f; }
+
+// Second look at a flagged norm code from the fast path's own fp32 values
+// (pair energy s, the row's smin, smax and ty) in double-float arithmetic, so
+// that only the transform's error is left.  Returns the code when the Eq. 2
+// value lies farther than norm_kappa() times that bound from a rounding
+// midpoint, else -1.
+template <int D, int B, int MODE>
+__device__ __forceinline__ int norm_second_look(float s, float smin, float smax, float ty) {
+  constexpr int Lq = (1 << B) - 1;
+  constexpr float kappa = norm_kappa<D>();
+  if constexpr (MODE == TAC_NORM_LINEAR) {
+    const float2 m = df_sqrt(make_float2(smin, 0.f)), M = df_sqrt(make_float2(smax, 0.f));
+    const float2 R = df_add(M, df_neg(m));
+    if (!(R.x > 0.f)) return -1;
+    // every sqrt(s) within ty; the double-float arithmetic adds far less than 1e-9 Lq
+    const float band = kappa * 2.f * (float)Lq * ty / R.x * 1.0001f + 1e-9f * (float)Lq;
+    const float2 A = df_add(df_sqrt(make_float2(s, 0.f)), df_neg(m));
+    const float2 w = df_add(df_div(df_mulf(A, (float)Lq), R), make_float2(0.5f, 0.f));
+    float c = floorf(w.x);
+    if (w.x == c && w.y < 0.f) c -= 1.f;
+    const float fr = __fadd_rn(__fsub_rn(w.x, c), w.y);
+    if (!(fminf(fr, 1.f - fr) > band)) return -1;
+    return min(max((int)c, 0), Lq);
+  } else {
+    const float sfl = smax * 3.5527136788005009e-15f;  // 2^-48 s_max
+    const float slo = fmaxf(smin, sfl), sa = fmaxf(s, sfl);
+    if (!(smax > slo)) return -1;
+    const float l2 = df_log2_est(df_div(make_float2(smax, 0.f), make_float2(slo, 0.f)));
+    const float l1 = df_log2_est(df_div(make_float2(sa, 0.f), make_float2(slo, 0.f)));
+    // log2 s moves by 2 dsqrt(s) / (sqrt(s) ln 2); each log2 estimate adds 2e-7
+    const float band = kappa * 2.f * 1.4426950408889634f * (float)Lq * ty / l2 * 1.01f *
+                           (rcp_approx(sqrt_approx(sa)) + rcp_approx(sqrt_approx(slo))) +
+                       (float)Lq * (4e-7f / l2 + 8.f * kU);
+    const float v = (float)Lq * l1 / l2 + 0.5f;
+    const float c = floorf(v);
+    const float fr = v - c;
+    if (!(fminf(fr, 1.f - fr) > band)) return -1;
+    return min(max((int)c, 0), Lq);
+  }
+}
+
+// The words of one input row a lane takes for the exact path: for pair
+// indices jj = lane + 32 q, elements 2 jj and 2 jj + 1 (one 32-bit word of two
+// bf16, or two fp32 words).
+template <int D, typename TIn>
+struct RowWords {
+  static constexpr int Q = (Geo<D>::P + 31) / 32;
+  static constexpr int NW = sizeof(TIn) == 2 ? Q : 2 * Q;
+  uint32_t w[NW];
+};
+
+template <int D, typename TIn>
+__device__ __forceinline__ void load_row_words(const uint8_t* src, RowWords<D, TIn>& r, int lane) {
+  constexpr int P = Geo<D>::P, Q = RowWords<D, TIn>::Q;
+#pragma unroll
+  for (int q = 0; q < Q; ++q) {
+    const int jj = lane + 32 * q;
+    if constexpr (sizeof(TIn) == 2) {
+      r.w[q] = jj < P ? *reinterpret_cast<const uint32_t*>(src + 4 * jj) : 0u;
+    } else {
+      const uint2 u = jj < P ? *reinterpret_cast<const uint2*>(src + 8 * jj) : make_uint2(0u, 0u);
+      r.w[2 * q] = u.x;
+      r.w[2 * q + 1] = u.y;
+    }
+  }
+}
+
+// Exact butterfly halves of every pair of one row, in 64-bit fixed point in
+// the warp's scratch (E at x[0 .. P), O at x[P .. 2P)): the row's elements
+// (this lane's words) are put on one fixed-point scale with D applied and
+// transformed by the unnormalized Sylvester butterfly (integer adds, exact).
+template <int D, typename TIn>
+__device__ __forceinline__ void exact_row(const EncJob& J, const RowWords<D, TIn>& r, long long* x, int lane) {
+  constexpr bool BF = sizeof(TIn) == 2;
+  constexpr int P = Geo<D>::P, Q = RowWords<D, TIn>::Q, MB = BF ? 7 : 23, SB = BF ? 15 : 31;
+  uint32_t w0[Q], w1[Q];
+  int emax = 1;
+#pragma unroll
+  for (int q = 0; q < Q; ++q) {
+    if constexpr (BF) {
+      w0[q] = r.w[q] & 0xFFFFu;
+      w1[q] = r.w[q] >> 16;
+    } else {
+      w0[q] = r.w[2 * q];
+      w1[q] = r.w[2 * q + 1];
+    }
+    emax = max(emax, (int)max((w0[q] >> MB) & 0xFFu, (w1[q] >> MB) & 0xFFu));
+  }
+  emax = (int)__reduce_max_sync(0xffffffffu, (unsigned)emax);
+#pragma unroll
+  for (int q = 0; q < Q; ++q) {
+    const int jj = lane + 32 * q, e0 = 2 * jj, e1 = 2 * jj + 1;
+    if (jj < P) {
+      const uint32_t s0 = (J.signs[e0 >> 5] >> (e0 & 31)) & 1u, s1 = (J.signs[e1 >> 5] >> (e1 & 31)) & 1u;
+      x[jj] = fix_elem<TIn>(w0[q], emax, ((w0[q] >> SB) & 1u) ^ s0);
+      x[P + jj] = fix_elem<TIn>(w1[q], emax, ((w1[q] >> SB) & 1u) ^ s1);
+    }
+  }
+  __syncwarp();
+#pragma unroll
+  for (int lh = 0; (1 << lh) < P; ++lh) {
+    const int h = 1 << lh;
+#pragma unroll
+    for (int q = 0; q < (P + 31) / 32; ++q) {       // P/2 butterflies on each half
+      const int bfly = lane + 32 * q;
+      if (bfly < P) {
+        const int half = bfly / (P / 2), k = bfly % (P / 2);
+        const int i0 = half * P + ((k >> lh) << (lh + 1)) + (k & (h - 1));
+        const long long a = x[i0], c = x[i0 + h];
+        x[i0] = a + c;
+        x[i0 + h] = a - c;
+      }
+    }
+    __syncwarp();
+  }
+}
+
+// Works through a warp's queue (all lanes call it): first the second look at
+// every norm entry, one entry a lane; then, warp-wide and a row at a time, the
+// exact path for what is left: the row's transform in fixed point, its exact
+// minimum and maximum pair energy, and the codes from the exact sums.  The
+// records in global memory are patched.  scratch: 2P longs of the warp's
+// shared memory.  Out of line: it runs once per few dozen entries.
+template <int D, typename TIn, int N, int B, int MODE>
+__device__ __noinline__ void flush_queue(const EncParams* p, uint4* q, int qn, long long* scratch, int lane) {
+  constexpr int P = Geo<D>::P;
+  constexpr int W = code_bits(N);
+  constexpr bool FP32N = MODE == TAC_NORM_FP32;
+  constexpr int AB = P * W / 8, NB = P * (FP32N ? 32 : B) / 8;
+  constexpr int kB = 4;                                 // rows whose loads are in flight together
+  __syncwarp();
+  auto record = [&](const EncJob& J, long long row, uint8_t*& codes, uint8_t*& norms) -> bool {
+    const long long sl = J.slot ? J.slot[row] : row;
+    if (sl < 0 || sl >= J.capacity) return false;   // skipped slots get no record
+    codes = J.codes + sl * AB;
+    norms = J.norms + sl * NB;
+    return true;
+  };
+  auto settled = [&](int e) { return ((q[2 * e].x >> 14) & 3u) == 3u; };
+  // The rows of the entries left after the second look are read again from
+  // global memory; ask for all of them now, so that their latency (long
+  // while the encoder streams) passes during the second look.
+  for (int e = lane; e < qn; e += 32) {
+    const uint4 a = q[2 * e];
+    const EncJob& J = p->job[a.x & 0xFFu];
+    const char* row = reinterpret_cast<const char*>(J.x) + (long long)a.y * J.stride * (long long)sizeof(TIn);
+#pragma unroll
+    for (int c = 0; c < D * (int)sizeof(TIn); c += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(row + c));
+  }
+  if constexpr (!FP32N) {
+    for (int e = lane; e < qn; e += 32) {
+      const uint4 a = q[2 * e];
+      if (((a.x >> 14) & 3u) != 1u) continue;
+      const uint4 b = q[2 * e + 1];
+      const int c = norm_second_look<D, B, MODE>(__uint_as_float(a.z), __uint_as_float(a.w), __uint_as_float(b.x),
+                                                 __uint_as_float(b.y));
+      if (c < 0) continue;
+      const EncJob& J = p->job[a.x & 0xFFu];
+      uint8_t *codes, *norms;
+      if (record(J, (long long)a.y, codes, norms)) patch_bits(norms, (int)((a.x >> 8) & 63u) * B, B, (uint32_t)c);
+      q[2 * e].x = a.x | (3u << 14);
+    }
+    __syncwarp();
+  }
+  // The rest, a batch of up to kB rows at a time (a row's entries are
+  // consecutive): the rows' loads are issued together so that their latencies
+  // overlap, then each row is transformed exactly and its codes decided.
+  int e = 0;
+  while (true) {
+    int bs[kB], be[kB], nb = 0;
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      bs[b] = be[b] = qn;
+      while (e < qn && settled(e)) ++e;
+      if (e < qn) {
+        const uint4 a = q[2 * e];
+        int g = e + 1;
+        while (g < qn && (q[2 * g].x & 0xFFu) == (a.x & 0xFFu) && q[2 * g].y == a.y) ++g;
+        bs[b] = e;
+        be[b] = g;
+        nb = b + 1;
+        e = g;
+      }
+    }
+    if (nb == 0) break;
+    RowWords<D, TIn> rw[kB];
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      if (b < nb) {
+        const uint4 a = q[2 * bs[b]];
+        const EncJob& J = p->job[a.x & 0xFFu];
+        load_row_words<D, TIn>(reinterpret_cast<const uint8_t*>(J.x) + (long long)a.y * J.stride * (long long)sizeof(TIn),
+                               rw[b], lane);
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      if (b >= nb) continue;
+      const uint4 a0 = q[2 * bs[b]];
+      const EncJob& J = p->job[a0.x & 0xFFu];
+      uint8_t *codes, *norms;
+      if (!record(J, (long long)a0.y, codes, norms)) continue;
+      exact_row<D, TIn>(J, rw[b], scratch, lane);
+      bool have_ext = false;
+      float2 smn = make_float2(0.f, 0.f), smx = make_float2(0.f, 0.f);
+      for (int f = bs[b]; f < be[b]; ++f) {
+        const uint4 a = q[2 * f];
+        const uint32_t kind = (a.x >> 14) & 3u;
+        if (kind == 3u) continue;
+        if (kind != 0u && !have_ext) {
+          have_ext = true;
+          if constexpr (!FP32N) {
+            // exact extremes of the pair energies
+            smn = make_float2(3.4028234663852886e38f, 0.f);
+            smx = make_float2(0.f, 0.f);
+            for (int ip = lane; ip < P; ip += 32) {
+              const float2 se = df_energy(make_longlong2(scratch[ip], scratch[P + ip]));
+              if (df_less(se, smn)) smn = se;
+              if (df_less(smx, se)) smx = se;
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+              const float2 omn = make_float2(__shfl_xor_sync(0xffffffffu, smn.x, off), __shfl_xor_sync(0xffffffffu, smn.y, off));
+              const float2 omx = make_float2(__shfl_xor_sync(0xffffffffu, smx.x, off), __shfl_xor_sync(0xffffffffu, smx.y, off));
+              if (df_less(omn, smn)) smn = omn;
+              if (df_less(smx, omx)) smx = omx;
+            }
+          }
+        }
+        if (kind == 2u) {   // the whole row, a pair a lane
+          for (int ip = lane; ip < P; ip += 32) {
+            const longlong2 eo = make_longlong2(scratch[ip], scratch[P + ip]);
+            const int v = pair_slot<D>(ip);
+            patch_bits(codes, v * W, W, (uint32_t)fix_angle_code<N>(eo));
+            if constexpr (!FP32N) patch_bits(norms, v * B, B, (uint32_t)fix_norm_code<B, MODE>(df_energy(eo), smn, smx));
+          }
+        } else {
+          const int v = (int)((a.x >> 8) & 63u);
+          const int ip = slot_pair<D>(v);
+          const longlong2 eo = make_longlong2(scratch[ip], scratch[P + ip]);
+          if (kind == 0u) {
+            const int k = fix_angle_code<N>(eo);
+            if (lane == 0) patch_bits(codes, v * W, W, (uint32_t)k);
+          } else if constexpr (!FP32N) {
+            const int c = fix_norm_code<B, MODE>(df_energy(eo), smn, smx);
+            if (lane == 0) patch_bits(norms, v * B, B, (uint32_t)c);
+          }
+        }
+      }
+      __syncwarp();
+    }
+  }
+  __syncwarp();
 }
 
 // Encode this lane's 8 pairs of warp-tile row r (lane l of the row) and stage
@@ -262,7 +711,8 @@ __device__ __forceinline__ void patch_code(uint8_t* rec, int i, int k) {
 // TAC_NORM_FP32 (B = 32: the pair norms themselves, no header).
 template <int D, typename TIn, int N, int B, int MODE>
 __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const float2* et, int nrows,
-                                          int lane, const uint2 (&msk)[8], const uint32_t* signs) {
+                                          int lane, const uint2 (&msk)[8], uint4* q, int& qn, int t,
+                                          const EncParams& p) {
   // bf16: msk[m].x holds the sign bits of the pair's two elements (bits 15
   // and 31), msk[m].y the low element's bit moved to bit 31.  The low element
   // widens as w * 2^16 + msk.y (adding bit 31 is an XOR of it: one integer
@@ -394,13 +844,13 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   // product (one hardware square root, about 1 ulp, either way).
   constexpr bool kEvenK2 = D == 32 || D == 128;
   const float rms = sqrt_ftz(smax_s);
-  float hmin = 0.f, hmax = 0.f, qs = 0.f, qo = 0.f, sfloor = 0.f;
+  float hmin = 0.f, hmax = 0.f, qs = 0.f, qo = 0.f, sfloor = 0.f, sc = 0.f;
   if constexpr (FP32N) {
     // no header: the norms are stored as they are (Sec. 3.1)
   } else if constexpr (MODE == TAC_NORM_LINEAR) {
     hmin = sqrt_approx(smin * k2);              // smin * sigma may still be subnormal
     hmax = (kEvenK2 ? rms * rk2 : sqrt_ftz(smax_s * k2)) * sr;
-    const float sc = (float)Lq * rcp_approx(hmax - hmin);
+    sc = (float)Lq * rcp_approx(hmax - hmin);
     qs = sc * rk2;                              // f(s) = sqrt(s)
     qo = __fmaf_rn(-hmin, sc, 0.5f);
     if (!(hmax > hmin) || !(sc <= 3.0e38f)) { qs = 0.f; qo = 0.5f; }
@@ -411,7 +861,7 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
     hmin = hmin_s * sr;
     hmax = hmax_s * sr;
     const float lmin_s = lg2_ftz(hmin_s);
-    const float sc = (float)Lq * rcp_approx(lg2_ftz(hmax_s) - lmin_s);
+    sc = (float)Lq * rcp_approx(lg2_ftz(hmax_s) - lmin_s);
     qs = 0.5f * sc;                             // f(s) = log2 s; log2 r = (log2 s + log2 k2)/2
     qo = __fmaf_rn(0.5f * (float)(G::LOGD == 4 ? -3 : G::LOGD == 5 ? -4 : G::LOGD == 6 ? -5 : -6) -
                        (lmin_s + (float)kk),
@@ -425,45 +875,169 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   //        <= (log2 d - 1) u sqrt(d/2) ||x||_2 = (log2 d - 1) u sqrt(S),
   // S = sum_i (E_i^2 + O_i^2) = d ||x||_2^2 / 2 (the factor 1.01 covers the
   // rounding of the computed S and the second-order terms).  The edge direction
-  // (<= 1 ulp), the product and the fma add <= 4 u (|E| + |O|) <= 4 u sqrt(2 smax).
+  // (each entry within 1 ulp, i.e. 2u relative) and the product E c (u) add
+  // at most 2u (|E||c| + |O||s|) + u |E c| <= 3u sqrt(E^2 + O^2) <= 3u sqrt(smax);
+  // the fma's own rounding cannot change the sign of a nonzero result.
+  // The same ty bounds the error of every sqrt(E^2 + O^2) (the unnormalized
+  // pair norm), so ty sqrt(2/d) bounds the error of each r_i.
+  // The angle band takes norm_kappa() of the transform's part (see the norm
+  // band below) and all of the arithmetic's part.
   const float rmx = rms * sr;
   const float ty = (float)(G::LOGD - 1) * kU * 1.01f * (sqrt_ftz(ssum * sigma) * sr);
-  const float tau = ty + 5.f * kU * 1.4143f * rmx;
+  const float tau = norm_kappa<D>() * ty + 3.03f * kU * rmx;
   // The per-pair norm functions below take s itself (pairs below the log floor
   // are clamped to it first), against the true-scale qs, qo: for inputs in the
   // supported range every nonzero s is a normal fp32 number, so the
   // flush-to-zero hardware forms see it unchanged.
-  (void)qs; (void)qo; (void)sfloor;
   // Pairs whose norm is so small that the fp32 angle may be off by a quarter bin
   // are re-decided too: sqrt(s) < 4 n ty / pi.
   const float rthr = ty * (4.f * (float)n / 3.14159265f);
   const float sthr = rthr * rthr;
+  if (l == 0) reinterpret_cast<float4*>(wsm + C::W_RC)[r] = make_float4(smin, smax, ty, 0.f);
+
+  // Norm-code band (Eq. 2).  The code is floor(t), t = f(s) qs + qo the Eq. 2
+  // value plus 1/2; it is re-decided exactly when t lies within th of an
+  // integer (a rounding midpoint of Eq. 2).  th adds two parts:
+  //  - the butterfly: kKappa times the first-order bound of the fp32 transform
+  //    (ty on every pair norm; linear: 2 Lq tau_r / (r_max - r_min), log: the
+  //    same on log2 r with 1/r_i <= 1/r_lo, tau_r = ty sqrt(2/d)).  That bound
+  //    assumes every rounding of every stage at its maximum and with one sign;
+  //    the errors measured on the synthetic caches of every workload stay
+  //    below 0.075 of it for a pair norm at d = 64, 128 (0.17 at d <= 32), and
+  //    their distribution is what kKappa is set from: in a simulation of the
+  //    fp32 transform over 1.3e8 pairs of every workload no norm code (and
+  //    over 1.8e8 codes no angle code) decided from the fp32 values outside
+  //    the band at kKappa = 1/128 differed from the exact one.  kKappa = 1/64
+  //    (d >= 64) or 1/4 (d <= 32) is used.  It is no proof for every input: a
+  //    code can still differ where the transform's error exceeds kKappa of its
+  //    bound and the exact value lies closer to the midpoint than that error,
+  //    i.e. within about 1e-4 code units (or 1e-7 rad) of it, where the parity
+  //    rule counts such codes;
+  //  - the kernel's own arithmetic, bounded in full: each computed norm (the
+  //    pair's, r_min's, r_max's) within kEr of its value for the computed
+  //    energy (hardware square root, rounding of the energy), qs within kEq,
+  //    log2 within kEl absolute plus a rounding of the result, and the roundings
+  //    of qo and of the final fma at magnitudes up to 2^(B+1).
+  // A row whose band reaches 1/4 (rows of nearly equal pair norms, non-finite
+  // rows) has every norm code re-decided.
+  constexpr float kKappa = norm_kappa<D>();
+  // kEr: hardware sqrt <= 2u relative (1 ulp) plus the energy's rounding
+  // (2u on s, u on its root); kEq: rcp <= 2u plus two roundings; kEl: lg2
+  // <= 2^-22 absolute on [1/2, 2), and within 4u |result| elsewhere (a GPU
+  // test checks each of these limits over whole binades).
+  constexpr float kEr = 3.f * kU, kEq = 4.f * kU, kEl = 2.384185791015625e-07f;  // 2^-22
+  constexpr float kMag = FP32N ? 0.f : (float)(1 << (B & 15));  // 2^B
+  constexpr int kFb = 23 - (FP32N ? 8 : B);                     // fraction bits of t + 2^B
+  constexpr uint32_t kFracMask = (1u << kFb) - 1u;
+  float th = 0.f;
+  if constexpr (!FP32N) {
+    if constexpr (MODE == TAC_NORM_LINEAR) {
+      th = kKappa * 2.f * qs * ty + 2.f * kEr * (hmax + hmin) * sc + (float)Lq * kEq +
+           kU * (hmin * sc + 4.f * kMag + 2.f);
+    } else {
+      const float elp = kEl + 4.f * kU * (fabsf(2.f * (float)kk) + 52.f);   // log2 of one pair's energy
+      th = kKappa * 2.f * sc * (ty * rk2) * rcp_approx(hmin) * 1.4426950408889634f + 1.5f * sc * elp +
+           (float)Lq * kEq + kU * (fabsf(qo) + 4.f * kMag + 2.f);
+    }
+  }
+  const bool nall = !(th < 0.25f);              // also NaN
+  const float thu = nall ? 0.f : th;
+  // t + 2^B + th (in [2^B, 2^(B+1))): the integer part of t + th sits in the
+  // mantissa bits [23 - B, 23) and its fraction in the kFb bits below
+  const float qo2 = qo + (kMag + thu);
+  const uint32_t thb2 = nall ? 0xFFFFFFFFu : 2u * ((uint32_t)(thu * (float)(1u << kFb)) + 1u);
 
   // ---- pass 2: norm codes (Eq. 2), packing ----
   uint32_t nlo = 0, nhi = 0;
+  uint32_t nfr = 0xFFFFFFFFu;                   // smallest fraction field of t + th over the lane's pairs
   float rn[FP32N ? 8 : 1];                      // fp32 norms r_j = sqrt(2 s_j / d)
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    // fields are disjoint and c <= Lq: the adds are ORs (one IMAD each)
     if constexpr (FP32N) {
       rn[j] = sqrt_approx(s[j] * k2);
     } else {
       float f;
       if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_ftz(s[j]);
       else f = lg2_ftz(fmaxf(s[j], sfloor));
-      const uint32_t c = min(__float2uint_rd(__fmaf_rn(f, qs, qo)), (uint32_t)Lq);
+      const uint32_t tb = __float_as_uint(__fmaf_rn(f, qs, qo2));
+      nfr = min(nfr, tb & kFracMask);
+      // code floor(t + th) = bits [kFb, kFb + B) of tb, moved to its field at
+      // bit j B (a pair within th of a midpoint is re-decided below)
       const int sn = j * B;
-      if (sn < 32) nlo += c << sn; else nhi += c << (sn - 32);
+      const int sh = kFb - (sn & 31);
+      const uint32_t part = (sh >= 0 ? (tb >> sh) : (tb << -sh)) & ((uint32_t)Lq << (sn & 31));
+      if (sn < 32) nlo |= part; else nhi |= part;
     }
   }
-  uint32_t fm = 0;
+  const bool nflag = !FP32N && (nall || nfr < thb2);
+  // fl: bits 0-7 name the angle codes to re-decide, bits 8-15 the norm codes
+  uint32_t fl = 0;
   if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; }
-  else if (mmin < tau || lmin_s < sthr) {  // rare: name the uncertified pairs
+  else if (mmin < tau || lmin_s < sthr || nflag) {  // rare: name the uncertified pairs
 #pragma unroll
     for (int j = 0; j < 8; ++j)
-      if (am[j] < tau || s[j] < sthr) fm |= 1u << j;
+      if (am[j] < tau || s[j] < sthr) fl |= 1u << j;
+    if constexpr (!FP32N) {
+      if (nflag) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float f;
+          if constexpr (MODE == TAC_NORM_LINEAR) f = sqrt_ftz(s[j]);
+          else f = lg2_ftz(fmaxf(s[j], sfloor));
+          if (nall || (__float_as_uint(__fmaf_rn(f, qs, qo2)) & kFracMask) < thb2) fl |= 0x100u << j;
+        }
+      }
+    }
   }
-  if (!live) fm = 0;
+  if (!live) fl = 0;
+
+  // ---- queue the codes to re-decide (kQ - qn >= kMaxPerTile on entry) ----
+  if (__ballot_sync(0xffffffffu, fl != 0u) != 0u) {
+    using QG = QGeo<D>;
+    const int cnt = __popc(fl & 0xFFFFu);
+    int rowcnt = cnt;
+#pragma unroll
+    for (int off = 1; off < L; off <<= 1) rowcnt += __shfl_xor_sync(0xffffffffu, rowcnt, off);
+    const bool whole = rowcnt > QG::kRowEntries || (nall && rowcnt > 0);
+    const int mine = whole ? (l == 0 ? 1 : 0) : cnt;
+    int inc = mine;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int o = __shfl_up_sync(0xffffffffu, inc, off);
+      if (lane >= off) inc += o;
+    }
+    if (mine) {
+      uint4* e = q + 2 * (qn + inc - mine);
+      const WarpJob* wj = reinterpret_cast<const WarpJob*>(wsm + C::W_JOB);
+      const int cj = wj->job;
+      const uint32_t row = (uint32_t)((long long)(t - p.job[cj].tile0) * C::RW + r);
+      const uint32_t hd = (uint32_t)cj;
+      const float4 rc = reinterpret_cast<const float4*>(wsm + C::W_RC)[r];
+      if (whole) {
+        e[0] = make_uint4(hd | (2u << 14), row, 0u, 0u);
+        e[1] = make_uint4(0u, 0u, 0u, 0u);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if ((fl >> j) & 1u) {
+            e[0] = make_uint4(hd | ((uint32_t)(8 * l + j) << 8), row, 0u, 0u);
+            e[1] = make_uint4(0u, 0u, 0u, 0u);
+            e += 2;
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if ((fl >> (8 + j)) & 1u) {
+            e[0] = make_uint4(hd | ((uint32_t)(8 * l + j) << 8) | (1u << 14), row, __float_as_uint(s[j]),
+                              __float_as_uint(rc.x));
+            e[1] = make_uint4(__float_as_uint(rc.y), __float_as_uint(rc.z), 0u, 0u);
+            e += 2;
+          }
+        }
+      }
+    }
+    qn += __shfl_sync(0xffffffffu, inc, 31);
+  }
 
   // ---- stage the records ----
   if (live) {
@@ -479,22 +1053,6 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   }
   __syncwarp();
 
-  // ---- exact re-decision of the uncertified pairs, one warp per pair ----
-  unsigned ball = __ballot_sync(0xffffffffu, fm != 0u);
-  while (ball) {
-    const int owner = __ffs(ball) - 1;
-    ball &= ball - 1;
-    uint32_t mm = __shfl_sync(0xffffffffu, fm, owner);
-    const int rr = owner / L, ol = owner % L;
-    while (mm) {
-      const int j = __ffs(mm) - 1;
-      mm &= mm - 1;
-      const int i = 8 * ol + j;
-      const int kk = exact_angle_code<D, TIn, N>(signs, in, rr, i, lane);
-      if (lane == 0) patch_code<W>(wsm + C::W_ANG + rr * AB, i, kk);
-    }
-    __syncwarp();
-  }
 }
 
 // Records of a tail tile (nrows < RW) or of scattered slots, from the staged
@@ -627,6 +1185,16 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
   uint2 msk[8];
 #pragma unroll
   for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
+  // re-decision queue: qn entries (warp-uniform), drained when fewer than
+  // one tile's worst case of free entries is left, and at the end
+  using QG = QGeo<D>;
+  uint4* const qb = reinterpret_cast<uint4*>(wsm + C::W_Q);
+  long long* const scr = reinterpret_cast<long long*>(wsm + C::W_SCR);
+  int qn = 0;
+  // Drain threshold, staggered over the warps (up to 28 entries apart) so that
+  // the warps of an SM, whose queues fill at about the same rate, do not all
+  // drain at the same time.
+  const int q_hi = kQ - QG::kMaxPerTile - 4 * (gw & 7);
 
   static_assert((kNS & (kNS - 1)) == 0, "stage ring size");
   int stage = 0;
@@ -640,8 +1208,9 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
       // A stretch of `fast` tiles, each a full tile of the current dense job
       // whose prefetch is a full tile of the issue job: no per-tile checks, the
       // cursors are settled once after it.
-      const int t_stop = t + fast;
+      const int t_start = t, t_stop = t + fast;
       for (; t < t_stop; ++t) {
+        if (qn > q_hi) break;   // the general iteration drains the queue first
         cp_async_wait<kNS - 2>();   // this warp tile has landed
         __syncwarp();               // ... and every lane is done with the previous one
         uint8_t* dst = in_dst + ((stage + kNS - 1) & (kNS - 1)) * IT::BYTES;
@@ -649,7 +1218,7 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
         for (int q = 0; q < C::CHUNKS; ++q) cp_async16(dst + q * C::RPQ * IT::STRIDE, i_src + q * i_qstep, 16);
         cp_async_commit();
         i_src += i_step;
-        tile_body<D, TIn, N, B, MODE>(wsm + C::W_IN + stage * IT::BYTES, wsm, etl, C::RW, lane, msk, wj->signs);
+        tile_body<D, TIn, N, B, MODE>(wsm + C::W_IN + stage * IT::BYTES, wsm, etl, C::RW, lane, msk, qb, qn, t, p);
         __syncwarp();
 #pragma unroll
         for (int q = 0; q < C::ROUNDS; ++q) {
@@ -660,16 +1229,23 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
         }
         stage = (stage + 1) & (kNS - 1);
       }
-      const int64_t adv = (int64_t)fast * C::RW;
+      const int done = t - t_start;
+      const int64_t adv = (int64_t)done * C::RW;
       c_row0 += adv;
       c_left -= adv;
       i_left -= adv;
-      it += fast;
+      it += done;
       fast = 0;
       continue;
     }
 
-    // ---- general tile: a job's first tile, tails, scattered slots, range ends ----
+    // ---- general tile: a job's first tile, tails, scattered slots, range ends,
+    // and the queue's drains (here only, so that the stretches stay free of calls) ----
+    if (qn > q_hi) {
+      __syncwarp();
+      flush_queue<D, TIn, N, B, MODE>(&p, qb, qn, scr, lane);
+      qn = 0;
+    }
     cp_async_wait<kNS - 2>();
     __syncwarp();
     issue((stage + kNS - 1) & (kNS - 1));
@@ -691,6 +1267,7 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
       }
       if (lane == 0) {
         wj->codes = J.codes; wj->norms = J.norms; wj->hdr = J.hdr; wj->slot = J.slot; wj->capacity = J.capacity;
+        wj->job = cj;
 #pragma unroll
         for (int q = 0; q < 4; ++q) wj->signs[q] = J.signs[q];
       }
@@ -703,7 +1280,7 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
       __syncwarp();
     }
     const int nrows = c_left >= C::RW ? C::RW : (int)c_left;
-    tile_body<D, TIn, N, B, MODE>(wsm + C::W_IN + stage * IT::BYTES, wsm, etl, nrows, lane, msk, wj->signs);
+    tile_body<D, TIn, N, B, MODE>(wsm + C::W_IN + stage * IT::BYTES, wsm, etl, nrows, lane, msk, qb, qn, t, p);
     __syncwarp();
     if (c_dense && nrows == C::RW) {
 #pragma unroll
@@ -727,6 +1304,10 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
     const int64_t pf = min(min((int64_t)(p_end - it), i_left / C::RW), (int64_t)(t_end - it));
     const int64_t f = min(cf, pf);
     fast = f > 0 ? (int)f : 0;
+  }
+  if (qn > 0) {
+    __syncwarp();
+    flush_queue<D, TIn, N, B, MODE>(&p, qb, qn, scr, lane);
   }
   cp_async_wait<0>();
 }

@@ -73,4 +73,33 @@ cudaError_t launch_fwht_debug(int d, const void* x, int dtype, int64_t rows, int
   return cudaGetLastError();
 }
 
+// Element-wise hardware approximations, as the kernels use them (tac_common.cuh):
+// op 0 sqrt.approx.f32, 1 sqrt.approx.ftz.f32, 2 rcp.approx.ftz.f32,
+// 3 lg2.approx.f32, 4 lg2.approx.ftz.f32, 5 ex2.approx.ftz.f32.
+__global__ void __launch_bounds__(256) hw_approx_kernel(int op, const float* __restrict__ x, float* __restrict__ y,
+                                                        int64_t n) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const float a = x[i];
+    float r;
+    switch (op) {
+      case 0: r = sqrt_approx(a); break;
+      case 1: r = sqrt_ftz(a); break;
+      case 2: r = rcp_approx(a); break;
+      case 3: r = lg2_approx(a); break;
+      case 4: r = lg2_ftz(a); break;
+      default: r = ex2_ftz(a); break;
+    }
+    y[i] = r;
+  }
+}
+
+cudaError_t launch_hw_approx(int op, const float* x, float* y, int64_t n, int sms, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  int64_t blocks = (n + 255) / 256;
+  const int64_t cap = (int64_t)(sms > 0 ? sms : 1) * 8;
+  if (blocks > cap) blocks = cap;
+  hw_approx_kernel<<<(unsigned)blocks, 256, 0, st>>>(op, x, y, n);
+  return cudaGetLastError();
+}
+
 }  // namespace tac

@@ -1,20 +1,23 @@
 """Element-by-element comparison of the CUDA path with the CPU oracle.
 
-Rules (derived in the design notes from the fp32 arithmetic of the kernels):
+Rules:
 
 angle codes   bit-exact wherever the oracle's angle lies 1e-5 rad or more from a
               bin edge; inside that band a differing code is counted, and the
               count must not exceed 1e-6 of all codes (below 10^6 codes: zero).
-header        |r_gpu - r_oracle| <= eps_h, eps_h = (2/sqrt d) gamma + 4 u r_max,
-              gamma = (log2 d - 1) u ||x||_1: the first-order bound of the fp32
-              butterfly's rounding on a pair (u = 2^-24), plus the energy's
-              rounding and the hardware square root (<= 2 ulp).
-norm codes    bit-exact wherever the oracle's Eq. 2 pre-round value lies more than
-              beta_i from a rounding midpoint, beta_i the propagated bound of the
-              fp32 norm, header and Eq. 2 arithmetic; inside, a code may differ by
-              one level and is counted (rate reported, must stay <= 1e-4).
-fp32 norms    (mode 2, Sec. 3.1) |r_gpu - r| <= (2/sqrt d) gamma + 4 u r, r the oracle's
-              exact pair norm; there is no header.
+norm codes    the same rule on Eq. 2: bit-exact wherever the oracle's Eq. 2
+              value lies more than 1e-4 code units from a rounding midpoint;
+              inside, a code may differ by one level, is counted, and the count
+              must not exceed 1e-6 of all codes (below 10^6 codes: zero).
+              Structured rows (constants, one-hots) get no exemption.
+header        the stored (r_min, r_max) are floating-point outputs:
+              |r_gpu - r_oracle| <= (2/sqrt d) gamma + (E_SQRT + 2u) r_max,
+              gamma = (log2 d - 1) u ||x||_1 the first-order bound of the fp32
+              butterfly on a pair (u = 2^-24), 2u the rounding of the pair
+              energy and of the stored value, E_SQRT the hardware square root's
+              relative error (a GPU test measures it against this bound).
+fp32 norms    (mode 2, Sec. 3.1) the same bound with r in place of r_max; there
+              is no header.
 decode        on identical codes: fp32 out |y - v| <= 1e-5 ||x^||;
               bf16 out |y - v| <= ulp_bf16(v)/2 + 1e-3 ||x^||  (v = oracle fp64 output).
 """
@@ -25,7 +28,10 @@ import math
 import numpy as np
 
 U = 2.0**-24
-ANGLE_BAND = 1e-5
+ANGLE_BAND = 1e-5      # rad: angle codes may differ only this close to a bin edge
+NORM_BAND = 1e-4       # code units: norm codes may differ only this close to a midpoint
+MISMATCH_RATE = 1e-6   # largest share of codes allowed to differ inside a band
+E_SQRT = 2.0**-23      # relative error bound of the hardware square root the kernels use
 
 
 def to_f64(t) -> np.ndarray:
@@ -65,32 +71,36 @@ def _gamma(x64: np.ndarray) -> np.ndarray:
     return (math.log2(d) - 1) * U * np.abs(x64).sum(axis=1)
 
 
-def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, mode: int,
-                   label: str = "", structured: bool = False) -> dict:
-    """Check GPU codes (k, c, hdr) against oracle output `ref` for input rows x64.
+def _allowed(codes: int) -> int:
+    """Mismatches allowed inside a band: 1e-6 of the codes, rounded down (0 below 10^6)."""
+    return int(MISMATCH_RATE * codes)
 
-    `structured`: hand-built rows (constants, one-hots) put Eq. 2 values exactly on
-    rounding midpoints, so only the band rule (not the statistical rate) applies."""
+
+def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, mode: int,
+                   label: str = "") -> dict:
+    """Check GPU codes (k, c, hdr) against oracle output `ref` for input rows x64;
+    returns the counts (band populations and mismatches)."""
     rows, d = x64.shape
     P = d // 2
-    L = (1 << b) - 1
     st = {"label": label, "rows": rows, "codes": rows * P}
 
     # ---- angle codes ----
     mism = k != ref["k"]
-    outside = mism & (ref["edge"] >= ANGLE_BAND)
+    in_band = ref["edge"] < ANGLE_BAND
+    outside = mism & ~in_band
     st["angle_mismatch"] = int(mism.sum())
     st["angle_mismatch_outside_band"] = int(outside.sum())
-    st["angle_band_population"] = int((ref["edge"] < ANGLE_BAND).sum())
+    st["angle_band_population"] = int(in_band.sum())
     assert st["angle_mismatch_outside_band"] == 0, (label, np.argwhere(outside)[:5])
-    assert st["angle_mismatch"] <= 1e-6 * st["codes"], (label, st)
+    assert st["angle_mismatch"] <= _allowed(st["codes"]), (label, st)
 
     gam = _gamma(x64)
+    assert np.all(np.isfinite(gam)), (label, "non-finite input row")
     if mode == FP32_MODE:
         # ---- fp32 norms: values, not codes ----
         r = ref["r"]
         rg = np.ascontiguousarray(c, dtype=np.int32).view(np.float32).astype(np.float64)
-        eps_r = (2.0 / math.sqrt(d)) * gam[:, None] + 4 * U * r + 1e-45
+        eps_r = (2.0 / math.sqrt(d)) * gam[:, None] + (E_SQRT + 2 * U) * r + 1e-45
         err = np.abs(rg - r)
         st["norm_max_err_over_bound"] = float((err / eps_r).max()) if rows else 0.0
         assert np.all(err <= eps_r), (label, st)
@@ -98,40 +108,25 @@ def compare_encode(orc, x64: np.ndarray, ref: dict, k, c, hdr, n: int, b: int, m
 
     # ---- header ----
     hmax_o = ref["hdr"][:, 1].astype(np.float64)
-    eps_h = (2.0 / math.sqrt(d)) * gam + 4 * U * hmax_o + 1e-45
+    eps_h = (2.0 / math.sqrt(d)) * gam + (E_SQRT + 2 * U) * hmax_o + 1e-45
     dh = np.abs(hdr.astype(np.float64) - ref["hdr"].astype(np.float64))
     st["header_max_err_over_bound"] = float((dh / eps_h[:, None]).max()) if rows else 0.0
+    hmax_ulp = np.spacing(np.abs(ref["hdr"]).astype(np.float32)).astype(np.float64)
+    st["header_max_err_ulp"] = float((dh / hmax_ulp).max()) if rows else 0.0
     assert np.all(dh <= eps_h[:, None]), (label, st)
 
     # ---- norm codes ----
-    hmin_o = ref["hdr"][:, 0].astype(np.float64)
-    r = ref["r"]
-    eps_r = (2.0 / math.sqrt(d)) * gam[:, None] + 4 * U * r
-    dh_range = np.maximum(hmax_o - hmin_o, 1e-300)
-    if mode == 0:
-        beta = L * (eps_r + 3 * eps_h[:, None]) / dh_range[:, None] + 4 * U * L
-    else:
-        floor_r = np.maximum(r, hmax_o[:, None] * 2.0**-24)
-        lmin = np.log2(np.maximum(hmin_o, 1e-300))
-        lmax = np.log2(np.maximum(hmax_o, 1e-300))
-        lrange = np.maximum(lmax - lmin, 1e-300)
-        # hardware log2: absolute error <= 2^-21 (plus relative rounding of the result)
-        dl = (eps_r / floor_r + 2 * U) / math.log(2) + 4 * U * np.abs(np.log2(floor_r)) + 2.0**-21
-        dlmin = (eps_h / np.maximum(hmin_o, 1e-300) + 2 * U) / math.log(2) + 4 * U * np.abs(lmin) + 2.0**-21
-        dlmax = (eps_h / np.maximum(hmax_o, 1e-300) + 2 * U) / math.log(2) + 4 * U * np.abs(lmax) + 2.0**-21
-        beta = L * (dl + 3 * np.maximum(dlmin, dlmax)[:, None]) / lrange[:, None] + 4 * U * L
-    flat = (ref["hdr"][:, 0] == ref["hdr"][:, 1])
-    beta[flat] = 0.0
     pre = ref["pre"]
+    assert np.all(np.isfinite(pre)), (label, "non-finite Eq. 2 value")
     dist_mid = np.abs(pre - (np.floor(pre) + 0.5))  # distance to the nearest rounding midpoint
+    in_band = dist_mid <= NORM_BAND
     nm = c != ref["c"]
+    bad = nm & ((np.abs(c.astype(np.int64) - ref["c"]) != 1) | ~in_band)
     st["norm_mismatch"] = int(nm.sum())
-    bad = nm & ((np.abs(c - ref["c"]) != 1) | (dist_mid > beta))
     st["norm_mismatch_outside_band"] = int(bad.sum())
-    st["norm_band_population"] = int((dist_mid <= beta).sum())
+    st["norm_band_population"] = int(in_band.sum())
     assert st["norm_mismatch_outside_band"] == 0, (label, st, np.argwhere(bad)[:5])
-    if not structured:
-        assert st["norm_mismatch"] <= max(2, 1e-4 * st["codes"]), (label, st)
+    assert st["norm_mismatch"] <= _allowed(st["codes"]), (label, st)
     return st
 
 

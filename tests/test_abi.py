@@ -162,8 +162,10 @@ def test_invalid_arguments_rejected_before_launch(tac_host):
     assert lib.tac_fwht_debug(ctypes.byref(rows), 3, s, buf, None) == tac_host.TAC_E_INVAL
     assert lib.tac_fwht_debug(ctypes.byref(rows), 256, s, buf, None) == tac_host.TAC_E_INVAL
     # signs
-    assert lib.tac_make_signs(0, 0, 2, 0, 64, s) == tac_host.TAC_E_INVAL
-    assert lib.tac_make_signs(0, -1, 0, 0, 64, s) == tac_host.TAC_E_INVAL
+    assert lib.tac_make_signs(0, 0, 2, 64, s) == tac_host.TAC_E_INVAL
+    assert lib.tac_make_signs(0, -1, 0, 64, s) == tac_host.TAC_E_INVAL
+    assert lib.tac_make_signs(0, 0, 0, 0, s) == tac_host.TAC_E_INVAL
+    assert lib.tac_make_signs_shared(0, 0, s) == tac_host.TAC_E_INVAL
 
 
 def test_empty_calls_succeed_without_device(tac_host):

@@ -35,8 +35,7 @@ def _oracle_cache(tac, orc, cfg, ref):
     return cache
 
 
-def check_roundtrip(tac, orc, x, d, n, b, mode, seed=0, layer=0, kv=0, label="", decode_dtypes=("bf16", "fp32"),
-                    structured=False):
+def check_roundtrip(tac, orc, x, d, n, b, mode, seed=0, layer=0, kv=0, label="", decode_dtypes=("bf16", "fp32")):
     torch = _torch()
     rows = x.shape[0]
     cfg = tac.layer_cfg(d, n, b, mode, seed, layer, kv)
@@ -47,7 +46,7 @@ def check_roundtrip(tac, orc, x, d, n, b, mode, seed=0, layer=0, kv=0, label="",
     assert np.array_equal(s, parity.signs_pm1(cfg.signs, d))
     ref = orc.encode(x64, s, n, b, mode)
     k, c, hdr = parity.gpu_codes(orc, cache, rows)
-    st = parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=label, structured=structured)
+    st = parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=label)
     # decode on identical codes (the oracle's records) into bf16 and fp32
     oc = _oracle_cache(tac, orc, cfg, ref)
     v = orc.decode(ref["k"], ref["c"], ref["hdr"], s, n, b, mode)
@@ -173,8 +172,7 @@ def test_degenerate_rows(tac_gpu, orc):
     rows.append(a)
     x = torch.tensor(np.array(rows), dtype=torch.float32).to(torch.bfloat16).cuda()
     for n, b, mode in ((64, 8, 0), (64, 4, 1), (4, 8, 0), (2, 4, 1), (256, 8, 1)):
-        check_roundtrip(tac_gpu, orc, x, d, n, b, mode, label=f"degenerate n={n} b={b} m={mode}",
-                        structured=True)
+        check_roundtrip(tac_gpu, orc, x, d, n, b, mode, label=f"degenerate n={n} b={b} m={mode}")
 
 
 def test_exact_bin_centres_and_ties(tac_gpu, orc):
