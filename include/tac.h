@@ -44,8 +44,13 @@
  *   - Inputs must be finite with |x_j| <= 2^56, and each nonzero |x_j| >= 2^-53
  *     for bf16 rows (>= 2^-37 for fp32 rows): then every nonzero pair energy
  *     E^2 + O^2 of the butterfly is a normal fp32 number and the codes and header
- *     match the definitions within the stated tolerances.  Other values give
- *     unspecified codes but never out-of-bounds accesses.
+ *     match the definitions within the stated tolerances.  A row holding a NaN
+ *     or an infinity gets a defined record instead: every angle and norm code 0
+ *     and the header (NaN, NaN) (with fp32 norms: every norm NaN), which decodes
+ *     to a NaN row; an encode given a status word (tac_encode_checked, or the
+ *     status field of a tac_encode_job) stores TAC_E_NONFINITE in it.  Finite
+ *     values outside the range give unspecified codes but never out-of-bounds
+ *     accesses.
  */
 #ifndef TAC_H_
 #define TAC_H_
@@ -63,7 +68,8 @@ typedef enum {
   TAC_OK = 0,
   TAC_E_INVAL = 1,
   TAC_E_UNSUPPORTED = 2,
-  TAC_E_CUDA = 3
+  TAC_E_CUDA = 3,
+  TAC_E_NONFINITE = 4   /* written (asynchronously) to an encode's status word: a row held a NaN or an inf */
 } tac_status;
 
 /* Norm storage: Eq. 2 linear, Eq. 2 on log2 r (Sec. 3.3), or the pair norms as fp32
@@ -106,6 +112,9 @@ typedef struct {
   const int64_t* slot;   /* device, x.rows entries: destination slot of row i, each in
                             [0, capacity); NULL means slot i (then x.rows <= capacity).
                             Duplicate slots race (one of the writers wins). */
+  uint32_t* status;      /* device, 4-byte aligned, or NULL: TAC_E_NONFINITE is stored in
+                            it when a row of x holds a NaN or an infinity; otherwise it is
+                            left as it is (the caller zeroes it; jobs may share one) */
 } tac_encode_job;
 
 /* One decode job of a batched launch: record slots -> rows of y (gather). */
@@ -175,6 +184,16 @@ int tac_rates(int num_layers, const int* n_k, const int* n_v, int b_k, int b_v, 
  */
 int tac_encode(const tac_rows* x, const tac_layer_cfg* cfg, void* out_codes, void* out_norms,
                tac_stream_t stream);
+
+/*
+ * tac_encode with a status word (device, 4-byte aligned, zeroed by the caller):
+ * TAC_E_NONFINITE is stored in *status, in stream order, when a row of x holds a
+ * NaN or an infinity (the paper fixes no behaviour for them; this library's
+ * records for such rows are described under the conventions above).  The
+ * return value reports argument and launch errors only, as for tac_encode.
+ */
+int tac_encode_checked(const tac_rows* x, const tac_layer_cfg* cfg, void* out_codes, void* out_norms,
+                       uint32_t* status, tac_stream_t stream);
 
 /*
  * Decode y->rows records (slots 0..y->rows-1 of a cache of capacity y->rows) into y
@@ -262,9 +281,12 @@ int tac_attend_multi(const tac_attend_job* jobs, int njobs, void* workspace, int
  *   - Nothing in the array needs to start at zero: every partial record is
  *     written by the first kernel before the second reads it.
  *   - First call on each device: resolves the array's address with
- *     cudaGetSymbolAddress, which may load the library's attention module.
- *     Make that first call outside stream capture; a call with njobs = 0 does
- *     only this setup and returns TAC_E_CUDA if it fails.  The first launch
+ *     cudaGetSymbolAddress, which may load the library's attention module,
+ *     and reads the device's SM count.  Make that first call outside stream
+ *     capture; a call with njobs = 0 does only this setup and returns
+ *     TAC_E_CUDA if it fails.  The address is cached per process and device;
+ *     after cudaDeviceReset it is stale (the module is loaded anew), so such a
+ *     process must not call this entry point again.  The first launch
  *     of each kernel shape (d, q dtype, query count) on a device also sets its
  *     shared-memory limit, as in tac_attend_multi.  After both, a call makes
  *     no CUDA runtime call but cudaGetDevice, the launches and

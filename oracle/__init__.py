@@ -238,10 +238,12 @@ def attend(q: np.ndarray, khat: np.ndarray, vhat: np.ndarray, scale: float) -> n
 
 
 def encode_threads(x: np.ndarray, s: np.ndarray, n: int, b: int, mode: int,
-                   threads: int) -> dict:
+                   threads: int, diagnostics: bool = False) -> dict:
     """encode() over row blocks on ``threads`` host threads (ctypes drops the GIL).
 
-    The per-row arithmetic is exactly encode()'s; only rows are split.
+    The per-row arithmetic is exactly encode()'s; only rows are split.  With
+    diagnostics the edge distances, pre-round Eq. 2 values and exact norms come
+    back too, as from encode().
     """
     x = np.ascontiguousarray(x, dtype=np.float64)
     rows = x.shape[0]
@@ -250,7 +252,7 @@ def encode_threads(x: np.ndarray, s: np.ndarray, n: int, b: int, mode: int,
 
     def work(i, idx):
         if len(idx):
-            res[i] = encode(x[idx[0]:idx[-1] + 1], s, n, b, mode, diagnostics=False)
+            res[i] = encode(x[idx[0]:idx[-1] + 1], s, n, b, mode, diagnostics=diagnostics)
 
     ts = [threading.Thread(target=work, args=(i, p)) for i, p in enumerate(parts)]
     for t in ts:
@@ -258,7 +260,7 @@ def encode_threads(x: np.ndarray, s: np.ndarray, n: int, b: int, mode: int,
     for t in ts:
         t.join()
     res = [r for r in res if r is not None]
-    return {key: np.concatenate([r[key] for r in res]) for key in ("k", "c", "hdr")}
+    return {key: np.concatenate([r[key] for r in res]) for key in res[0]}
 
 
 def decode_threads(k, c, hdr, s, n, b, mode, threads: int) -> np.ndarray:

@@ -19,7 +19,7 @@ from dataclasses import dataclass, field
 import numpy as np
 
 __all__ = [
-    "TAC_OK", "TAC_E_INVAL", "TAC_E_UNSUPPORTED", "TAC_E_CUDA", "NORM_LINEAR", "NORM_LOG", "NORM_FP32",
+    "TAC_OK", "TAC_E_INVAL", "TAC_E_UNSUPPORTED", "TAC_E_CUDA", "TAC_E_NONFINITE", "NORM_LINEAR", "NORM_LOG", "NORM_FP32",
     "BF16", "FP32", "TacError", "LayerCfg", "EncodeJob", "DecodeJob", "library_path", "load",
     "make_signs", "layer_cfg", "angle_row_bytes", "norm_row_bytes", "header_offset",
     "codes_bytes", "norms_bytes", "avg_angle_bits", "total_bits", "encode", "decode",
@@ -27,7 +27,7 @@ __all__ = [
     "AttendJob", "attend_multi", "attend_workspace_bytes",
 ]
 
-TAC_OK, TAC_E_INVAL, TAC_E_UNSUPPORTED, TAC_E_CUDA = 0, 1, 2, 3
+TAC_OK, TAC_E_INVAL, TAC_E_UNSUPPORTED, TAC_E_CUDA, TAC_E_NONFINITE = 0, 1, 2, 3, 4
 NORM_LINEAR, NORM_LOG, NORM_FP32 = 0, 1, 2
 BF16, FP32 = 0, 1
 MAX_D = 128
@@ -59,7 +59,7 @@ class _Rows(ctypes.Structure):
 
 class _EncJob(ctypes.Structure):
     _fields_ = [("cfg", _Cfg), ("x", _Rows), ("codes", ctypes.c_void_p), ("norms", ctypes.c_void_p),
-                ("capacity", ctypes.c_int64), ("slot", ctypes.c_void_p)]
+                ("capacity", ctypes.c_int64), ("slot", ctypes.c_void_p), ("status", ctypes.c_void_p)]
 
 
 class _DecJob(ctypes.Structure):
@@ -107,6 +107,8 @@ def load():
         lib.tac_total_bits.argtypes = [ctypes.c_double, ctypes.c_double, i32]
         lib.tac_encode.restype = i32
         lib.tac_encode.argtypes = [P(_Rows), P(_Cfg), vp, vp, vp]
+        lib.tac_encode_checked.restype = i32
+        lib.tac_encode_checked.argtypes = [P(_Rows), P(_Cfg), vp, vp, vp, vp]
         lib.tac_decode.restype = i32
         lib.tac_decode.argtypes = [vp, vp, P(_Cfg), P(_Rows), vp]
         lib.tac_encode_multi.restype = i32
@@ -295,6 +297,7 @@ class EncodeJob:
     x: object            # [rows, d] bf16/fp32 device tensor
     cache: Cache
     slot: object = None  # optional int64 device tensor [rows]
+    status: object = None  # optional int32 device tensor [1], zeroed: gets TAC_E_NONFINITE
 
 
 @dataclass
@@ -305,16 +308,22 @@ class DecodeJob:
     slot: object = None  # optional int64 device tensor [rows]
 
 
-def encode(x, cfg: LayerCfg, cache: Cache | None = None, stream=None) -> Cache:
-    """tac_encode: rows of x -> record slots 0..rows-1 of a cache of capacity rows."""
+def encode(x, cfg: LayerCfg, cache: Cache | None = None, stream=None, status=None) -> Cache:
+    """tac_encode: rows of x -> record slots 0..rows-1 of a cache of capacity rows.
+    With `status` (an int32 device tensor of one element, zeroed by the caller)
+    tac_encode_checked stores TAC_E_NONFINITE in it if a row holds a NaN or an inf."""
     if cache is None:
         cache = Cache.empty(cfg, x.shape[0], device=x.device)
     if cache.capacity != x.shape[0]:
         raise ValueError("tac_encode writes a cache of capacity rows; use encode_multi for slots")
     r = _rows(x, cfg.d)
     c = cfg.to_c()
-    _check(load().tac_encode(ctypes.byref(r), ctypes.byref(c), cache.codes.data_ptr(),
-                             cache.norms.data_ptr(), _stream_ptr(stream)))
+    if status is None:
+        _check(load().tac_encode(ctypes.byref(r), ctypes.byref(c), cache.codes.data_ptr(),
+                                 cache.norms.data_ptr(), _stream_ptr(stream)))
+    else:
+        _check(load().tac_encode_checked(ctypes.byref(r), ctypes.byref(c), cache.codes.data_ptr(),
+                                         cache.norms.data_ptr(), status.data_ptr(), _stream_ptr(stream)))
     return cache
 
 
@@ -355,6 +364,7 @@ def _enc_array(jobs):
         e.norms = j.cache.norms.data_ptr()
         e.capacity = j.cache.capacity
         e.slot = j.slot.data_ptr() if j.slot is not None else None
+        e.status = j.status.data_ptr() if j.status is not None else None
     return arr
 
 

@@ -2,6 +2,7 @@
 // generator and the batched launch planner.  Kernels live in tac_encode.cu,
 // tac_decode.cu and tac_fwht_debug.cu.
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <mutex>
 #include <cstdarg>
@@ -187,16 +188,16 @@ void sm_shares(const int64_t* tiles, int ngroups, int sms, int* caps) {
 }
 
 int num_sms() {
-  static int cache[64] = {0};
+  static std::atomic<int> cache[64];   // per device; concurrent first calls store the same value
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   if (dev < 0 || dev >= 64) return 0;
-  if (!cache[dev]) {
-    int v = 0;
+  int v = cache[dev].load(std::memory_order_relaxed);
+  if (!v) {
     if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    cache[dev] = v;
+    cache[dev].store(v, std::memory_order_relaxed);
   }
-  return cache[dev];
+  return v;
 }
 
 void copy_signs(uint32_t* dst, const tac_layer_cfg* c) {
@@ -408,6 +409,7 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
       return fail(TAC_E_INVAL, "%s: job %d rows %lld > capacity %lld", who, j, (long long)J.x.rows,
                   (long long)J.capacity);
     if (J.slot && ((uintptr_t)J.slot & 7u)) return fail(TAC_E_INVAL, "%s: job %d slot misaligned", who, j);
+    if (J.status && ((uintptr_t)J.status & 3u)) return fail(TAC_E_INVAL, "%s: job %d status misaligned", who, j);
     live.push_back(j);
   }
   const int sms = num_sms();
@@ -445,6 +447,7 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
       E.norms = static_cast<uint8_t*>(J.norms);
       E.hdr = static_cast<uint8_t*>(J.norms) + header_offset(&J.cfg, J.capacity);
       E.slot = J.slot;
+      E.status = J.status;
       E.capacity = J.capacity;
       E.rows = J.x.rows;
       E.stride = J.x.row_stride;
@@ -591,6 +594,23 @@ int tac_encode(const tac_rows* x, const tac_layer_cfg* cfg, void* out_codes, voi
   j.norms = out_norms;
   j.capacity = x->rows;
   j.slot = nullptr;
+  return tac_encode_multi(&j, 1, stream);
+}
+
+int tac_encode_checked(const tac_rows* x, const tac_layer_cfg* cfg, void* out_codes, void* out_norms,
+                       uint32_t* status, tac_stream_t stream) {
+  if (!x) return fail(TAC_E_INVAL, "tac_encode_checked: x is NULL");
+  if (!cfg) return fail(TAC_E_INVAL, "tac_encode_checked: cfg is NULL");
+  if (!status) return fail(TAC_E_INVAL, "tac_encode_checked: status is NULL");
+  tac_encode_job j;
+  std::memset(&j, 0, sizeof(j));
+  j.cfg = *cfg;
+  j.x = *x;
+  j.codes = out_codes;
+  j.norms = out_norms;
+  j.capacity = x->rows;
+  j.slot = nullptr;
+  j.status = status;
   return tac_encode_multi(&j, 1, stream);
 }
 
@@ -794,8 +814,8 @@ int tac_attend_multi_static(const tac_attend_job* jobs, int njobs, tac_stream_t 
   float* ws = nullptr;
   const cudaError_t e = tac::attend_static_workspace(&ws);
   if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: static workspace: %s", who, cudaGetErrorString(e));
+  if (num_sms() <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);   // cached for later calls
   if (njobs == 0) return ok();
-  if (num_sms() <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
   return run_attend(jobs, njobs, ws, reinterpret_cast<cudaStream_t>(stream), false, who);
 }
 

@@ -549,19 +549,19 @@ template <int D, typename TQ, int NQ>
 static cudaError_t launch_attend_t(const AttParams& p_in, int nrows_total, float* ws, cudaStream_t st) {
   using C = Att<D, NQ>;
   auto kp = attend_partial<D, NQ>;
-  static int configured[64] = {0};
-  static int regs[64] = {0};
+  // per device, set on the first launch; atomic so that host threads making
+  // first calls at once do not race (each sets the same values)
+  static std::atomic<int> regs[64];
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!configured[dev]) {
+  if (regs[dev].load(std::memory_order_acquire) == 0) {
     cudaError_t e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     if (e != cudaSuccess) return e;
     cudaFuncAttributes fa;
     e = cudaFuncGetAttributes(&fa, kp);
     if (e != cudaSuccess) return e;
-    regs[dev] = fa.numRegs;
-    configured[dev] = 1;
+    regs[dev].store(fa.numRegs > 0 ? fa.numRegs : 1, std::memory_order_release);
   }
   AttParams p = p_in;
   int stage = 0;
@@ -569,7 +569,7 @@ static cudaError_t launch_attend_t(const AttParams& p_in, int nrows_total, float
     const AttJob& J = p.job[j];
     stage = std::max(stage, att_stage_bytes(D, J.wk, J.bk, J.mk, J.wv, J.bv, J.mv));
   }
-  const int wpc = att_warps_per_cta(C::smem(stage, 0), C::smem(stage, 1) - C::smem(stage, 0), regs[dev]);
+  const int wpc = att_warps_per_cta(C::smem(stage, 0), C::smem(stage, 1) - C::smem(stage, 0), regs[dev].load(std::memory_order_relaxed));
   int64_t ctas = 0;
   for (int j = 0; j < p.njobs; ++j) {
     AttJob& J = p.job[j];

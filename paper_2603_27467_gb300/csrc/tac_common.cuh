@@ -128,6 +128,7 @@ struct EncJob {
   uint8_t* norms;      // norm plane base
   uint8_t* hdr;        // header plane base (float2 per slot)
   const int64_t* slot; // destination slots or nullptr
+  uint32_t* status;    // gets TAC_E_NONFINITE when a row holds a NaN or an inf (or nullptr)
   int64_t capacity;    // record slots of the destination planes
   int64_t rows;
   int64_t stride;      // elements

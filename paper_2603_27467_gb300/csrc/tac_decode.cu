@@ -18,6 +18,8 @@
 //   3. D is a sign XOR on the output bits (after bf16 round-to-nearest-even, or
 //      on fp32); each lane stores its pairs straight from registers: the L
 //      lanes of a row write L consecutive pairs, whole 32-byte sectors.
+#include <atomic>
+
 #include "tac_common.cuh"
 
 namespace tac {
@@ -426,13 +428,13 @@ template <int D, typename TOut, int N, int B, int MODE>
 static cudaError_t launch_decode_v(const DecParams& p, int grid_cap, cudaStream_t st) {
   using C = Dec<D, TOut, N, B, MODE>;
   auto kern = decode_kernel<D, TOut, N, B, MODE>;
-  static int configured[64] = {0};
+  static std::atomic<int> configured[64];   // per device; concurrent first calls set the same
   int dev = 0;
   cudaGetDevice(&dev);
-  if (dev >= 0 && dev < 64 && !configured[dev]) {
+  if (dev >= 0 && dev < 64 && configured[dev].load(std::memory_order_acquire) == 0) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
-    configured[dev] = 1;
+    configured[dev].store(1, std::memory_order_release);
   }
   int per_sm = 0;
   cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, C::THREADS, C::SMEM);

@@ -32,6 +32,8 @@
 //   5. each lane packs its 8 codes LSB-first; the warp stages its records in
 //      shared memory and writes them with one 16-byte store per lane (contiguous
 //      slots) or per row (scatter-append slots).
+#include <atomic>
+
 #include "tac_common.cuh"
 
 namespace tac {
@@ -518,12 +520,17 @@ __device__ __forceinline__ void load_row_words(const uint8_t* src, RowWords<D, T
   }
 }
 
-// Exact butterfly halves of every pair of one row, in 64-bit fixed point in
-// the warp's scratch (E at x[0 .. P), O at x[P .. 2P)): the row's elements
-// (this lane's words) are put on one fixed-point scale with D applied and
-// transformed by the unnormalized Sylvester butterfly (integer adds, exact).
+// A lane's elements of one row (pair indices jj = lane + 32 q), D and their
+// signs applied, in 64-bit fixed point on the row's largest exponent.
 template <int D, typename TIn>
-__device__ __forceinline__ void exact_row(const EncJob& J, const RowWords<D, TIn>& r, long long* x, int lane) {
+struct FixWords {
+  static constexpr int Q = RowWords<D, TIn>::Q;
+  long long xe[Q], xo[Q];
+};
+
+template <int D, typename TIn>
+__device__ __forceinline__ void fix_words(const EncJob& J, const RowWords<D, TIn>& r, FixWords<D, TIn>& f,
+                                          int lane) {
   constexpr bool BF = sizeof(TIn) == 2;
   constexpr int P = Geo<D>::P, Q = RowWords<D, TIn>::Q, MB = BF ? 7 : 23, SB = BF ? 15 : 31;
   uint32_t w0[Q], w1[Q];
@@ -543,10 +550,48 @@ __device__ __forceinline__ void exact_row(const EncJob& J, const RowWords<D, TIn
 #pragma unroll
   for (int q = 0; q < Q; ++q) {
     const int jj = lane + 32 * q, e0 = 2 * jj, e1 = 2 * jj + 1;
+    f.xe[q] = f.xo[q] = 0;
     if (jj < P) {
       const uint32_t s0 = (J.signs[e0 >> 5] >> (e0 & 31)) & 1u, s1 = (J.signs[e1 >> 5] >> (e1 & 31)) & 1u;
-      x[jj] = fix_elem<TIn>(w0[q], emax, ((w0[q] >> SB) & 1u) ^ s0);
-      x[P + jj] = fix_elem<TIn>(w1[q], emax, ((w1[q] >> SB) & 1u) ^ s1);
+      f.xe[q] = fix_elem<TIn>(w0[q], emax, ((w0[q] >> SB) & 1u) ^ s0);
+      f.xo[q] = fix_elem<TIn>(w1[q], emax, ((w1[q] >> SB) & 1u) ^ s1);
+    }
+  }
+}
+
+// E and O of the pair in slot v alone, exact (a warp-wide integer sum).
+template <int D, typename TIn>
+__device__ __forceinline__ longlong2 fix_pair(const FixWords<D, TIn>& f, int v, int lane) {
+  constexpr int Q = FixWords<D, TIn>::Q;
+  const int ip = slot_pair<D>(v);
+  long long e = 0, o = 0;
+#pragma unroll
+  for (int q = 0; q < Q; ++q) {
+    const int jj = lane + 32 * q;
+    const bool neg = __popc((unsigned)(ip & jj)) & 1;
+    e += neg ? -f.xe[q] : f.xe[q];
+    o += neg ? -f.xo[q] : f.xo[q];
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    e += __shfl_xor_sync(0xffffffffu, e, off);
+    o += __shfl_xor_sync(0xffffffffu, o, off);
+  }
+  return make_longlong2(e, o);
+}
+
+// Exact butterfly halves of every pair of one row, in 64-bit fixed point in
+// the warp's scratch (E at x[0 .. P), O at x[P .. 2P)): the unnormalized
+// Sylvester butterfly on the lane's fixed-point elements (integer adds, exact).
+template <int D, typename TIn>
+__device__ __forceinline__ void exact_row(const FixWords<D, TIn>& f, long long* x, int lane) {
+  constexpr int P = Geo<D>::P, Q = FixWords<D, TIn>::Q;
+#pragma unroll
+  for (int q = 0; q < Q; ++q) {
+    const int jj = lane + 32 * q;
+    if (jj < P) {
+      x[jj] = f.xe[q];
+      x[P + jj] = f.xo[q];
     }
   }
   __syncwarp();
@@ -653,7 +698,9 @@ __device__ __noinline__ void flush_queue(const EncParams* p, uint4* q, int qn, l
       const EncJob& J = p->job[a0.x & 0xFFu];
       uint8_t *codes, *norms;
       if (!record(J, (long long)a0.y, codes, norms)) continue;
-      exact_row<D, TIn>(J, rw[b], scratch, lane);
+      FixWords<D, TIn> fw;
+      fix_words<D, TIn>(J, rw[b], fw, lane);
+      exact_row<D, TIn>(fw, scratch, lane);
       bool have_ext = false;
       float2 smn = make_float2(0.f, 0.f), smx = make_float2(0.f, 0.f);
       for (int f = bs[b]; f < be[b]; ++f) {
@@ -824,7 +871,7 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
     smax = fmaxf(smax, __shfl_xor_sync(0xffffffffu, smax, off));
     ssum += __shfl_xor_sync(0xffffffffu, ssum, off);
   }
-  const bool zero_row = !(smax > 0.f);
+  const bool zero_row = smax == 0.f;               // (a NaN row goes on, to the non-finite check)
 
   // ---- row constants: stored header (Sec. 3.3), Eq. 2 as code = floor(f(s) qs + qo) ----
   constexpr float k2 = 2.0f / (float)D;
@@ -972,8 +1019,27 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
   const bool nflag = !FP32N && (nall || nfr < thb2);
   // fl: bits 0-7 name the angle codes to re-decide, bits 8-15 the norm codes
   uint32_t fl = 0;
+  // a row whose energy sum is not finite may hold a NaN or an inf: its lanes
+  // look at their 16 staged elements
+  const bool odd = !(ssum <= 3.4028234663852886e38f);
+  bool nf = false;
   if (zero_row) { alo = ahi = nlo = nhi = 0; hmin = hmax = 0.f; }
-  else if (mmin < tau || lmin_s < sthr || nflag) {  // rare: name the uncertified pairs
+  else if (mmin < tau || lmin_s < sthr || nflag || odd) {  // rare: name the uncertified pairs
+    if (odd) {
+      const uint4* e16 = reinterpret_cast<const uint4*>(in + r * IT::STRIDE + l * 16 * C::ESZ);
+#pragma unroll
+      for (int c = 0; c < C::ESZ; ++c) {
+        const uint4 w = e16[c];
+        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          if constexpr (C::ESZ == 2)
+            nf |= (ww[k] & 0x7F80u) == 0x7F80u || (ww[k] & 0x7F800000u) == 0x7F800000u;
+          else
+            nf |= (ww[k] & 0x7F800000u) == 0x7F800000u;
+        }
+      }
+    }
 #pragma unroll
     for (int j = 0; j < 8; ++j)
       if (am[j] < tau || s[j] < sthr) fl |= 1u << j;
@@ -989,11 +1055,31 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
       }
     }
   }
-  if (!live) fl = 0;
+  if (!live) { fl = 0; nf = false; }
 
-  // ---- queue the codes to re-decide (kQ - qn >= kMaxPerTile on entry) ----
-  if (__ballot_sync(0xffffffffu, fl != 0u) != 0u) {
+  // ---- rows holding a NaN or an inf: all codes 0, header (NaN, NaN), the
+  // job's status word set; then queue the codes to re-decide (kQ - qn >=
+  // kMaxPerTile on entry) ----
+  if (__ballot_sync(0xffffffffu, fl != 0u || nf) != 0u) {
     using QG = QGeo<D>;
+    const unsigned nfb = __ballot_sync(0xffffffffu, nf);
+    if (nfb != 0u) {
+      constexpr uint32_t kRL = (L >= 32) ? 0xFFFFFFFFu : ((1u << L) - 1u);
+      if ((nfb >> (r * L)) & kRL) {
+        const float qnan = __int_as_float(0x7FC00000);
+        fl = 0;
+        alo = ahi = nlo = nhi = 0;
+        hmin = hmax = qnan;
+        if constexpr (FP32N) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) rn[j] = qnan;
+        }
+        if (l == 0) {
+          uint32_t* st = p.job[reinterpret_cast<const WarpJob*>(wsm + C::W_JOB)->job].status;
+          if (st) atomicOr(st, (uint32_t)TAC_E_NONFINITE);
+        }
+      }
+    }
     const int cnt = __popc(fl & 0xFFFFu);
     int rowcnt = cnt;
 #pragma unroll
@@ -1319,13 +1405,13 @@ template <int D, typename TIn, int N, int B, int MODE>
 static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_t st) {
   using C = Enc<D, TIn, N, B, MODE>;
   auto kern = encode_kernel<D, TIn, N, B, MODE>;
-  static int configured[64] = {0};
+  static std::atomic<int> configured[64];   // per device; concurrent first calls set the same
   int dev = 0;
   cudaGetDevice(&dev);
-  if (dev >= 0 && dev < 64 && !configured[dev]) {
+  if (dev >= 0 && dev < 64 && configured[dev].load(std::memory_order_acquire) == 0) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
-    configured[dev] = 1;
+    configured[dev].store(1, std::memory_order_release);
   }
   int per_sm = 0;
   cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kEncThreads, C::SMEM);

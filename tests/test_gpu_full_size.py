@@ -2,6 +2,7 @@
 launch over every (layer, K/V) block), checked on sampled rows against the oracle
 and on properties that hold at any size."""
 import math
+import os
 
 import numpy as np
 import pytest
@@ -46,7 +47,9 @@ def test_full_cache_encode_decode_sampled(tac_gpu, orc, name):
     tac.decode_multi([tac.DecodeJob(cfgs[key], caches[key], ys[key]) for key in xs])
     torch.cuda.synchronize()
     rng = np.random.default_rng(1)
-    per_block = 48 if name == "mistral7b" else 96
+    # at least 10^6 codes per workload: 64 blocks x 256 rows x 64 pairs, 32 x 1000 x 32
+    per_block = 256 if name == "mistral7b" else 1000
+    threads = os.cpu_count() or 1
     tot = {"codes": 0, "angle_mismatch": 0, "norm_mismatch": 0}
     for key in xs:
         d, n, b, mode = w.codebook(*key)
@@ -55,14 +58,15 @@ def test_full_cache_encode_decode_sampled(tac_gpu, orc, name):
         it = torch.from_numpy(idx).cuda()
         x64 = parity.to_f64(xs[key][it])
         s = orc.signs(0, key[0], key[1], d)
-        ref = orc.encode(x64, s, n, b, mode)
+        ref = orc.encode_threads(x64, s, n, b, mode, threads, diagnostics=True)
         k, c, hdr = parity.gpu_codes(orc, caches[key], slots=idx)
         st = parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=f"{name} {key}")
         for f in tot:
             tot[f] += st[f]
-        v = orc.decode(k, c, hdr, s, n, b, mode)
+        v = orc.decode_threads(k, c, hdr, s, n, b, mode, threads)
         parity.compare_decode(parity.to_f64(ys[key][it]), v, "bf16", label=f"{name} {key} decode")
-    assert tot["angle_mismatch"] <= 1e-6 * tot["codes"]
+    assert tot["codes"] >= 1_000_000
+    assert tot["angle_mismatch"] <= 1e-6 * tot["codes"] and tot["norm_mismatch"] <= 1e-6 * tot["codes"], tot
 
 
 def test_full_cache_properties(tac_gpu):
@@ -111,38 +115,45 @@ def test_append_step_full(tac_gpu, orc):
     tac.encode_multi(jobs)
     torch.cuda.synchronize()
     sl = slots.cpu().numpy()
-    for j, key in zip(jobs[:: 9], list(xs)[:: 9]):
+    threads = os.cpu_count() or 1
+    for j, key in zip(jobs, list(xs)):   # every block: 64 x 2048 rows, 8.4e6 codes
         d, n, b, mode = w.codebook(*key)
         x64 = parity.to_f64(j.x)
-        ref = orc.encode(x64, orc.signs(0, key[0], key[1], d), n, b, mode)
+        ref = orc.encode_threads(x64, orc.signs(0, key[0], key[1], d), n, b, mode, threads, diagnostics=True)
         k, c, hdr = parity.gpu_codes(orc, j.cache, slots=sl)
         parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=f"append {key}")
 
 
 def test_longctx_decode_sweep_sampled(tac_gpu, orc):
-    """Config 5 shape (4 heads x 131072 tokens per (layer, kv)), codebooks swept."""
+    """Config 5 shape (4 heads x 131072 tokens per (layer, kv)) on layers 0, 13,
+    27: every n of the sweep for K and for V (K and V are coded independently,
+    so this covers all 25 (n_K, n_V) pairs), each whole block encoded and
+    decoded, 400 rows of each compared with the oracle."""
     torch = _torch()
     tac = tac_gpu
     w = workloads.CONFIGS["longctx"]
     rng = np.random.default_rng(3)
-    for (nk, nv) in ((16, 256), (256, 16), (64, 32)):
-        for kv, n in ((0, nk), (1, nv)):
+    threads = os.cpu_count() or 1
+    for layer in (0, 13, 27):
+        for kv in (0, 1):
+            x = workloads.block(w, layer, kv, seed=5, device="cuda")
             b, mode = (8, 0) if kv == 0 else (4, 1)
-            cfg = tac.layer_cfg(128, n, b, mode, 0, 13, kv)
-            x = workloads.block(w, 13, kv, seed=5, device="cuda")
-            cache = tac.encode(x, cfg)
-            y = tac.decode(cache, cfg)
-            torch.cuda.synchronize()
-            idx = _sample(x.shape[0], 200, rng)
-            k, c, hdr = parity.gpu_codes(orc, cache, slots=idx)
-            s = orc.signs(0, 13, kv, 128)
-            v = orc.decode(k, c, hdr, s, n, b, mode)
-            parity.compare_decode(parity.to_f64(y[torch.from_numpy(idx).cuda()]), v, "bf16",
-                                  label=f"longctx n={n}")
-            x64 = parity.to_f64(x[torch.from_numpy(idx).cuda()])
-            ref = orc.encode(x64, s, n, b, mode)
-            parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=f"longctx enc n={n}")
-            del x, y, cache
+            s = orc.signs(0, layer, kv, 128)
+            for n in workloads.SWEEP_N:
+                cfg = tac.layer_cfg(128, n, b, mode, 0, layer, kv)
+                cache = tac.encode(x, cfg)
+                y = tac.decode(cache, cfg)
+                torch.cuda.synchronize()
+                idx = _sample(x.shape[0], 400, rng)
+                it = torch.from_numpy(idx).cuda()
+                k, c, hdr = parity.gpu_codes(orc, cache, slots=idx)
+                v = orc.decode(k, c, hdr, s, n, b, mode)
+                parity.compare_decode(parity.to_f64(y[it]), v, "bf16", label=f"longctx L{layer} kv{kv} n={n}")
+                x64 = parity.to_f64(x[it])
+                ref = orc.encode_threads(x64, s, n, b, mode, threads, diagnostics=True)
+                parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=f"longctx enc L{layer} kv{kv} n={n}")
+                del y, cache
+            del x
 
 
 def test_full_cache_attention_sampled(tac_gpu, orc):

@@ -289,3 +289,48 @@ def _encode_diag_threads(orc, x64, s, n, b, mode, threads):
     for t in ts:
         t.join()
     return {key: np.concatenate([o[key] for o in out if o is not None]) for key in out[0]}
+
+
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+@pytest.mark.parametrize("b,mode", [(8, 0), (4, 1), (32, 2)])
+def test_nonfinite_rows(tac_gpu, orc, dt, b, mode):
+    """Rows holding a NaN or an infinity: every code 0 and the header (NaN, NaN)
+    (fp32 norms: NaN), a NaN row on decode, TAC_E_NONFINITE in the status word;
+    the other rows of the call are unaffected, and an all-finite call leaves the
+    status word alone."""
+    torch = _torch()
+    d, n, layer, kv = 128, 64, 1, mode % 2
+    w = workloads.CONFIGS["mistral7b"]
+    x = _rows(w, 70, seed=11, dtype=torch.float32, layer=layer, kv=kv).clone()
+    bad = np.array([3, 17, 40, 69])
+    x[3, 5] = float("nan")
+    x[17, 100] = float("inf")
+    x[40, 0] = float("-inf")
+    x[69, :] = float("nan")
+    x = (x.to(torch.bfloat16) if dt == "bf16" else x).contiguous()
+    good = np.setdiff1d(np.arange(x.shape[0]), bad)
+    cfg = tac_gpu.layer_cfg(d, n, b, mode, 0, layer, kv)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    cache = tac_gpu.encode(x, cfg, status=status)
+    y = tac_gpu.decode(cache, cfg, dtype=torch.float32)
+    torch.cuda.synchronize()
+    assert int(status.item()) == tac_gpu.TAC_E_NONFINITE
+    k, c, hdr = parity.gpu_codes(orc, cache, x.shape[0])
+    assert np.all(k[bad] == 0)
+    if mode == parity.FP32_MODE:
+        assert np.all(np.isnan(np.ascontiguousarray(c[bad], dtype=np.int32).view(np.float32)))
+    else:
+        assert np.all(c[bad] == 0) and np.all(np.isnan(hdr[bad]))
+    yb = parity.to_f64(y)[bad]
+    assert np.all(np.isnan(yb)), yb[:, :4]
+    # the finite rows of the same call match the oracle
+    x64 = parity.to_f64(x)[good]
+    s = orc.signs(0, layer, kv, d)
+    ref = orc.encode(x64, s, n, b, mode)
+    parity.compare_encode(orc, x64, ref, k[good], c[good], hdr[good] if hdr is not None else None, n, b, mode,
+                          label=f"finite rows beside non-finite ones {dt} b={b} m={mode}")
+    # an all-finite call leaves the status word as it is
+    status.zero_()
+    tac_gpu.encode(x[torch.from_numpy(good).cuda()].contiguous(), cfg, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
