@@ -35,8 +35,12 @@
  *   - All device pointers must be 16-byte aligned; rows are row_stride elements
  *     apart and row_stride * sizeof(element) must be a multiple of 16.
  *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
- *     stream), allocate no device memory, and never synchronize (the batched
- *     calls create their helper streams once, see tac_encode_multi).
+ *     stream) and never synchronize (the batched calls create their helper
+ *     streams once, see tac_encode_multi).  They allocate no device memory,
+ *     except that tac_encode, tac_encode_checked and tac_encode_multi take the
+ *     encode's re-decision workspace from the device's stream-ordered memory
+ *     pool (cudaMallocAsync / cudaFreeAsync on `stream`); tac_encode_multi_ws
+ *     takes it from the caller instead.
  *   - Errors: a nonzero tac_status is returned and tac_last_error() gives a message
  *     (per host thread).  TAC_E_INVAL: a bad argument (nothing launched).
  *     TAC_E_UNSUPPORTED: a valid but unimplemented shape (nothing launched).
@@ -219,6 +223,31 @@ int tac_decode(const void* codes, const void* norms, const tac_layer_cfg* cfg, t
  * slots (streaming append).  Jobs must not write overlapping slots.
  */
 int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream);
+
+/*
+ * The encode's re-decision workspace.  The fast path decides every code in
+ * fp32 and certifies it against a bound on its own error (Alg. 1's edge test,
+ * Eq. 2's rounding); each launch appends the codes it could not certify (a few
+ * in ten thousand) to a queue in this workspace, and a fix-up kernel on the
+ * launch's stream re-decides them (double-float, then exact integer sums).
+ *
+ * tac_encode_workspace_bytes returns the recommended size for the call
+ * tac_encode_multi_ws(jobs, njobs, ...) (queue room for one code in 512 of
+ * every group, far above the rates of the paper's workloads) and stores the
+ * minimum in *min_bytes (if not NULL): a counter block and one bit per row.
+ * With less than the recommended size the queues shrink; a code that finds its
+ * queue full has its whole row re-decided instead, so the results do not depend
+ * on the size, only the time does.  Returns -1 (tac_last_error) for a call
+ * tac_encode_multi would reject.
+ *
+ * tac_encode_multi_ws is tac_encode_multi with the caller's workspace (device
+ * memory, 16-byte aligned, at least the minimum; its contents need no
+ * initialization; it must not be used by other work until the call's work on
+ * `stream` is done).  TAC_E_INVAL if the workspace is too small.
+ */
+int64_t tac_encode_workspace_bytes(const tac_encode_job* jobs, int njobs, int64_t* min_bytes);
+int tac_encode_multi_ws(const tac_encode_job* jobs, int njobs, void* workspace, int64_t workspace_bytes,
+                        tac_stream_t stream);
 
 /* Batched decode, grouped into launches (run concurrently) like tac_encode_multi. */
 int tac_decode_multi(const tac_decode_job* jobs, int njobs, tac_stream_t stream);

@@ -113,6 +113,10 @@ def load():
         lib.tac_decode.argtypes = [vp, vp, P(_Cfg), P(_Rows), vp]
         lib.tac_encode_multi.restype = i32
         lib.tac_encode_multi.argtypes = [P(_EncJob), i32, vp]
+        lib.tac_encode_workspace_bytes.restype = i64
+        lib.tac_encode_workspace_bytes.argtypes = [P(_EncJob), i32, P(ctypes.c_int64)]
+        lib.tac_encode_multi_ws.restype = i32
+        lib.tac_encode_multi_ws.argtypes = [P(_EncJob), i32, vp, i64, vp]
         lib.tac_decode_multi.restype = i32
         lib.tac_decode_multi.argtypes = [P(_DecJob), i32, vp]
         lib.tac_attend_workspace_bytes.restype = i64
@@ -368,14 +372,42 @@ def _enc_array(jobs):
     return arr
 
 
-def encode_multi(jobs, stream=None) -> None:
-    """tac_encode_multi: one launch per kernel group (see launch_count)."""
-    _check(load().tac_encode_multi(_enc_array(jobs), len(jobs), _stream_ptr(stream)))
+def encode_workspace_bytes(jobs) -> tuple[int, int]:
+    """tac_encode_workspace_bytes: (recommended, minimum) workspace bytes."""
+    mn = ctypes.c_int64(0)
+    n = load().tac_encode_workspace_bytes(_enc_array(jobs), len(jobs), ctypes.byref(mn))
+    if n < 0:
+        raise TacError(TAC_E_INVAL, last_error())
+    return int(n), int(mn.value)
 
 
-def encode_multi_prepared(jobs) -> Prepared:
-    """tac_encode_multi over `jobs`, marshalled once (see Prepared)."""
-    return Prepared(load().tac_encode_multi, _enc_array(jobs), len(jobs), (), list(jobs))
+def _enc_workspace(jobs, workspace):
+    if workspace is None:
+        need = encode_workspace_bytes(jobs)[0] if jobs else 0
+        dev = jobs[0].x.device if jobs else "cuda"
+        workspace = _torch().empty(max(need, 16), dtype=_torch().uint8, device=dev)
+    return workspace
+
+
+def encode_multi(jobs, stream=None, workspace=None):
+    """tac_encode_multi_ws: one encode launch and one fix-up launch per kernel
+    group (see launch_count); allocates the re-decision workspace (torch) when
+    none is given.  Returns the workspace."""
+    arr = _enc_array(jobs)
+    workspace = _enc_workspace(jobs, workspace)
+    _check(load().tac_encode_multi_ws(arr, len(jobs), workspace.data_ptr(),
+                                      workspace.numel() * workspace.element_size(), _stream_ptr(stream)))
+    if stream is not None and jobs:
+        workspace.record_stream(stream)   # in use on `stream` until its work is done
+    return workspace
+
+
+def encode_multi_prepared(jobs, workspace=None) -> Prepared:
+    """tac_encode_multi_ws over `jobs`, marshalled once (see Prepared), with
+    a workspace allocated (torch) once when none is given."""
+    workspace = _enc_workspace(jobs, workspace)
+    extra = (workspace.data_ptr(), workspace.numel() * workspace.element_size())
+    return Prepared(load().tac_encode_multi_ws, _enc_array(jobs), len(jobs), extra, (list(jobs), workspace))
 
 
 def _dec_array(jobs):
@@ -476,15 +508,19 @@ def attend_multi_static(jobs, stream=None):
 def launch_count(jobs) -> int:
     """Kernel launches one encode_multi / decode_multi call makes for `jobs`:
     jobs with rows are grouped by kernel (d, dtype, n, norm bits, norm mode),
-    at most MAX_JOBS jobs per launch."""
+    at most MAX_JOBS jobs per group; a decode group is one launch, an encode
+    group two (the encode and its fix-up)."""
     groups: dict = {}
+    per = 1
     for j in jobs:
         t = j.x if isinstance(j, EncodeJob) else j.y
+        if isinstance(j, EncodeJob):
+            per = 2
         if t.shape[0] == 0:
             continue
         key = (j.cfg.d, str(t.dtype), j.cfg.n_angle, j.cfg.norm_bits, j.cfg.norm_mode)
         groups[key] = groups.get(key, 0) + 1
-    return sum(-(-c // MAX_JOBS) for c in groups.values())
+    return per * sum(-(-c // MAX_JOBS) for c in groups.values())
 
 
 def fwht_debug(x, signs: np.ndarray, d: int, stream=None):

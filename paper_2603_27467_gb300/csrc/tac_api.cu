@@ -388,8 +388,13 @@ struct DecGroup {
 
 }  // namespace
 
-int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream) {
-  static const char* who = "tac_encode_multi";
+namespace {
+
+// Validates an encode call and groups its jobs by kernel: (d, dtype, n, norm
+// bits, norm mode), one launch per group and up to TAC_MAX_JOBS jobs each,
+// largest groups first.  Returns 0 or the call's tac status.
+int plan_encode(const tac_encode_job* jobs, int njobs, const char* who, std::vector<EncGroup>& groups) {
+  groups.clear();
   if (njobs < 0) return fail(TAC_E_INVAL, "%s: njobs = %d", who, njobs);
   if (njobs > 0 && !jobs) return fail(TAC_E_INVAL, "%s: jobs is NULL", who);
   // Validate everything before launching anything.
@@ -412,27 +417,19 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
     if (J.status && ((uintptr_t)J.status & 3u)) return fail(TAC_E_INVAL, "%s: job %d status misaligned", who, j);
     live.push_back(j);
   }
-  const int sms = num_sms();
-  if (live.empty()) return ok();
-  if (sms <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
-  // Group by kernel: (d, dtype, n, norm bits, norm mode); one launch per group
-  // and up to TAC_MAX_JOBS jobs per launch.
   auto kernel_key = [&](int j) {
     const tac_encode_job& J = jobs[j];
     return (((J.cfg.d * 4 + J.x.dtype) * 512 + J.cfg.n_angle) * 64 + J.cfg.norm_bits) * 4 + J.cfg.norm_mode;
   };
   std::stable_sort(live.begin(), live.end(), [&](int a, int b) { return kernel_key(a) < kernel_key(b); });
-  static thread_local std::vector<EncGroup> groups;
-  groups.clear();
   size_t i = 0;
   while (i < live.size()) {
     const int key = kernel_key(live[i]);
     const tac_layer_cfg& c0 = jobs[live[i]].cfg;
     const int d = c0.d, dt = jobs[live[i]].x.dtype;
-    const int na = c0.n_angle, nb = c0.norm_bits, mode = c0.norm_mode;
     groups.emplace_back();
     EncGroup& G = groups.back();
-    G.d = d; G.dt = dt; G.na = na; G.nb = nb; G.mode = mode;
+    G.d = d; G.dt = dt; G.na = c0.n_angle; G.nb = c0.norm_bits; G.mode = c0.norm_mode;
     tac::EncParams& P = G.p;
     std::memset(&P, 0, sizeof(P));
     int64_t tiles = 0;
@@ -440,7 +437,7 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
       const tac_encode_job& J = jobs[live[i]];
       const int64_t tr = tile_rows(d);
       const int64_t jt = (J.x.rows + tr - 1) / tr;
-      if (tiles + jt > 0x7fffffff) break;
+      if (tiles + jt > 0x7fffffff / tr) break;          // warp-tile rows must index in 31 bits
       tac::EncJob& E = P.job[P.njobs];
       E.x = J.x.data;
       E.codes = static_cast<uint8_t*>(J.codes);
@@ -466,23 +463,124 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
   // largest groups first: the small ones fill the tail of the large ones
   std::stable_sort(groups.begin(), groups.end(),
                    [](const EncGroup& a, const EncGroup& b) { return a.p.ntiles > b.p.ntiles; });
+  return 0;
+}
+
+// Workspace of an encode call: per launch group a 64-byte counter block and a
+// bitmap of its warp-tile rows (together the part zeroed at the call), then
+// per group its re-decision queue, 32-byte entries.  The queue's recommended
+// capacity is one entry per 512 angle pairs plus 1024 (the synthetic caches
+// of every workload queue about one per 2400 pairs); with less room the
+// capacities shrink in proportion, down to none (then every row with a code to
+// re-decide is re-decided whole through the bitmap).
+constexpr int64_t kEncCtrBytes = 64, kEncEntryBytes = 32;
+int64_t enc_ovf_bytes(const EncGroup& G) {
+  const int64_t bits = (int64_t)G.p.ntiles * tile_rows(G.d);
+  return ((bits + 127) / 128) * 16;
+}
+int64_t enc_rec_cap(const EncGroup& G) {
+  int64_t pairs = 0;
+  for (int j = 0; j < G.p.njobs; ++j) pairs += G.p.job[j].rows * (G.d / 2);
+  return pairs / 512 + 1024;
+}
+struct EncWs {
+  int64_t zero = 0, min = 0, rec = 0, rec_entries = 0;
+};
+EncWs enc_ws(const std::vector<EncGroup>& groups) {
+  EncWs w;
+  w.zero = kEncCtrBytes * (int64_t)groups.size();
+  for (const EncGroup& G : groups) {
+    w.zero += enc_ovf_bytes(G);
+    w.rec_entries += enc_rec_cap(G);
+  }
+  w.min = w.zero;
+  w.rec = w.zero + kEncEntryBytes * w.rec_entries;
+  return w;
+}
+
+// Launches a planned encode call with its workspace (ws_bytes >= the minimum).
+int run_encode(std::vector<EncGroup>& groups, uint8_t* ws, int64_t ws_bytes, cudaStream_t st, const char* who) {
+  const int sms = num_sms();
+  if (sms <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
+  const EncWs w = enc_ws(groups);
+  const int64_t avail = (ws_bytes - w.zero) / kEncEntryBytes;
+  int64_t ovf_off = kEncCtrBytes * (int64_t)groups.size(), q_off = w.zero;
+  for (size_t g = 0; g < groups.size(); ++g) {
+    tac::EncParams& P = groups[g].p;
+    const int64_t rc = enc_rec_cap(groups[g]);
+    const int64_t cap = avail >= w.rec_entries ? rc : (int64_t)((double)rc * (double)avail / (double)w.rec_entries);
+    P.gq_n = reinterpret_cast<unsigned long long*>(ws + kEncCtrBytes * (int64_t)g);
+    P.ovf = reinterpret_cast<uint32_t*>(ws + ovf_off);
+    P.gq = reinterpret_cast<uint4*>(ws + q_off);
+    P.gq_cap = cap;
+    ovf_off += enc_ovf_bytes(groups[g]);
+    q_off += kEncEntryBytes * cap;
+  }
+  cudaError_t e = cudaMemsetAsync(ws, 0, (size_t)w.zero, st);
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(e));
   static thread_local std::vector<int64_t> gtiles;
   static thread_local std::vector<int> caps;
   gtiles.resize(groups.size());
   caps.resize(groups.size());
   for (size_t g = 0; g < groups.size(); ++g) gtiles[g] = groups[g].p.ntiles;
   sm_shares(gtiles.data(), (int)groups.size(), sms, caps.data());
-  GroupFork fork(reinterpret_cast<cudaStream_t>(stream), (int)groups.size());
+  GroupFork fork(st, (int)groups.size());
   if (fork.error() != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(fork.error()));
   for (size_t g = 0; g < groups.size(); ++g) {
     const EncGroup& G = groups[g];
-    cudaError_t e = tac::launch_encode(G.d, G.dt, G.na, G.nb, G.mode, G.p, caps[g], fork.stream((int)g));
+    e = tac::launch_encode(G.d, G.dt, G.na, G.nb, G.mode, G.p, caps[g], fork.stream((int)g));
     if (e != cudaSuccess) {
       fork.join();
       return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
     }
   }
-  const cudaError_t e = fork.join();
+  e = fork.join();
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(e));
+  return 0;
+}
+
+}  // namespace
+
+int64_t tac_encode_workspace_bytes(const tac_encode_job* jobs, int njobs, int64_t* min_bytes) {
+  static thread_local std::vector<EncGroup> groups;
+  if (plan_encode(jobs, njobs, "tac_encode_workspace_bytes", groups)) return -1;
+  const EncWs w = enc_ws(groups);
+  if (min_bytes) *min_bytes = w.min;
+  ok();
+  return w.rec;
+}
+
+int tac_encode_multi_ws(const tac_encode_job* jobs, int njobs, void* workspace, int64_t workspace_bytes,
+                        tac_stream_t stream) {
+  static const char* who = "tac_encode_multi_ws";
+  static thread_local std::vector<EncGroup> groups;
+  int rc = plan_encode(jobs, njobs, who, groups);
+  if (rc) return rc;
+  if (groups.empty()) return ok();
+  const EncWs w = enc_ws(groups);
+  if (!workspace || !aligned16(workspace)) return fail(TAC_E_INVAL, "%s: workspace NULL or not 16-byte aligned", who);
+  if (workspace_bytes < w.min)
+    return fail(TAC_E_INVAL, "%s: workspace of %lld bytes < the minimum %lld", who, (long long)workspace_bytes,
+                (long long)w.min);
+  rc = run_encode(groups, static_cast<uint8_t*>(workspace), workspace_bytes, reinterpret_cast<cudaStream_t>(stream),
+                  who);
+  return rc ? rc : ok();
+}
+
+int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream) {
+  static const char* who = "tac_encode_multi";
+  static thread_local std::vector<EncGroup> groups;
+  int rc = plan_encode(jobs, njobs, who, groups);
+  if (rc) return rc;
+  if (groups.empty()) return ok();
+  const EncWs w = enc_ws(groups);
+  const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  void* ws = nullptr;
+  cudaError_t e = cudaMallocAsync(&ws, (size_t)w.rec, st);
+  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: workspace allocation: %s", who, cudaGetErrorString(e));
+  rc = run_encode(groups, static_cast<uint8_t*>(ws), w.rec, st, who);
+  e = cudaFreeAsync(ws, st);
+  if (rc) return rc;
   if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(e));
   return ok();
 }

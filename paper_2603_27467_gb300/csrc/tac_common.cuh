@@ -142,6 +142,13 @@ struct EncJob {
 struct EncParams {
   int32_t njobs;
   int32_t ntiles;
+  // Re-decision queue of the launch (workspace, see the encode kernel): the
+  // codes the fast path could not certify, 32-byte entries.
+  uint4* gq;                   // gq_cap entries (two uint4 each)
+  unsigned long long* gq_n;    // entries appended (may pass gq_cap: the rest went to ovf)
+  uint32_t* ovf;               // one bit per warp-tile row (tile * RW + row in tile): rows
+                               // whose entries found the queue full, re-decided whole
+  int64_t gq_cap;
   EncJob job[TAC_MAX_JOBS];
 };
 

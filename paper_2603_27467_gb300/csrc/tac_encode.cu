@@ -32,6 +32,7 @@
 //   5. each lane packs its 8 codes LSB-first; the warp stages its records in
 //      shared memory and writes them with one 16-byte store per lane (contiguous
 //      slots) or per row (scatter-append slots).
+#include <algorithm>
 #include <atomic>
 
 #include "tac_common.cuh"
@@ -96,16 +97,12 @@ struct Enc {
   static constexpr int W_RC = W_JOB + 64;                    // the rows' fp32 (smin, smax, ty) for the queue
   static constexpr int W_Q = W_RC + RW * 16;                 // re-decision queue (kQ entries of 32 bytes)
   static constexpr int WARP_B = W_Q + kQ * 32;
-  // scratch of the queue's exact path (2P longs), free between tiles: the
-  // transpose rows, or for d = 16 (no transpose) the staged records
-  static constexpr int W_SCR = (G::TP_W >= 16 * P) ? W_TP : W_ANG;
   static constexpr int TABR = tab_copies(n, 8192);           // edge table copies
   static constexpr int OFF_TAB = kEncWarps * WARP_B;           // fp32 edge table of this n (TABR copies)
   static constexpr int SMEM = OFF_TAB + n * TABR * 8;
   static_assert((RW * AB) % 16 == 0 && (RW * NB) % 16 == 0 && (RW * HB) % 16 == 0, "record segments");
   static_assert(W_TP % 16 == 0 && W_ANG % 16 == 0 && W_JOB % 16 == 0 && WARP_B % 16 == 0, "alignment");
   static_assert(32 % CPR == 0 && RW % RPQ == 0, "chunk map");
-  static_assert(G::TP_W >= 16 * P || RW * (AB + NB + HB) >= 16 * P, "queue scratch");
 };
 
 // The job a warp is encoding as far as the rare paths need it (exact
@@ -437,10 +434,11 @@ __device__ __forceinline__ void patch_bits(uint8_t* base, int bit, int w, uint32
 // the end.  Doing so outside the tile body keeps the body's registers and
 // instructions free of the rare path; the records, written already, are
 // patched in place.  An entry (32 bytes): job | slot << 8 | kind << 14, the
-// row in the job, and for a norm code its pair energy s and the row's smin,
-// smax and ty of the fast path.  kind: 0 an angle code, 1 a norm code, 2 the
-// whole row (rows with more flagged codes than kRowEntries, or whose norm
-// band is too wide to be useful), 3 settled.
+// row in the job, then for an angle code the pair's fp32 butterfly halves E, O
+// and (in the second half) the row's ty, for a norm code its pair energy s and
+// the row's smin, smax and ty of the fast path.  kind: 0 an angle code, 1 a
+// norm code, 2 the whole row (rows with more flagged codes than kRowEntries,
+// or whose norm band is too wide to be useful).
 // ---------------------------------------------------------------------------
 template <int D>
 struct QGeo {
@@ -492,6 +490,29 @@ __device__ __forceinline__ int norm_second_look(float s, float smin, float smax,
     if (!(fminf(fr, 1.f - fr) > band)) return -1;
     return min(max((int)c, 0), Lq);
   }
+}
+
+// Second look at a flagged angle code from the fast path's fp32 butterfly
+// halves (E, O) and the row's transform bound ty: the edge test in
+// double-float against the double-float edge direction, so that only the
+// transform's error is left.  That error moves m = E cos psi - O sin psi by at
+// most sqrt(dE^2 + dO^2) <= ty (first order); the code is returned when |m|
+// exceeds norm_kappa() of it (the fast band's transform part) plus the
+// double-float arithmetic's own (below 2^-43 sqrt(E^2 + O^2)), else -1.  Pairs
+// under the fast path's small-norm threshold (same expression, same value)
+// always go on to the exact path: their fp32 angle may be off by more than the
+// candidate edge allows for.
+template <int D, int N>
+__device__ __forceinline__ int angle_second_look(float E, float O, float ty) {
+  const float s = __fmaf_rn(E, E, __fmul_rn(O, O));
+  const float rthr = ty * (4.f * (float)N / 3.14159265f);
+  if (s < rthr * rthr || !(s > 0.f)) return -1;
+  const int ec = candidate_edge<N>(E, O);
+  const float4 dir = g_edge_df.v[tab_offset_n(N) + ec];
+  const float2 m = df_add(df_mulf(make_float2(dir.x, dir.y), E), df_neg(df_mulf(make_float2(dir.z, dir.w), O)));
+  const float band = norm_kappa<D>() * ty * 1.001f + 1.0e-12f * sqrt_approx(s);
+  if (!(fabsf(m.x) > band)) return -1;
+  return wrap_bin<N>(ec + (m.x > 0.f ? 1 : 0));
 }
 
 // The words of one input row a lane takes for the exact path: for pair
@@ -613,20 +634,74 @@ __device__ __forceinline__ void exact_row(const FixWords<D, TIn>& f, long long* 
   }
 }
 
-// Works through a warp's queue (all lanes call it): first the second look at
-// every norm entry, one entry a lane; then, warp-wide and a row at a time, the
-// exact path for what is left: the row's transform in fixed point, its exact
-// minimum and maximum pair energy, and the codes from the exact sums.  The
-// records in global memory are patched.  scratch: 2P longs of the warp's
-// shared memory.  Out of line: it runs once per few dozen entries.
+// Exact minimum and maximum pair energy of the row in scratch (E at x[0, P),
+// O at x[P, 2P), 64-bit fixed point) as double-floats, the same on every lane.
+// fp32 estimates from the exact sums (each within 4u of its energy, so two
+// energies in one order have estimates at most 8 ulp the other way) name the
+// candidates: the pairs whose estimate lies within 32 ulp of the smallest
+// (largest) estimate.  Only those get the double-float energy.
+template <int D>
+__device__ __forceinline__ void exact_extremes(const long long* x, int lane, float2& smn, float2& smx) {
+  constexpr int P = Geo<D>::P, Q = (P + 31) / 32;
+  uint32_t eb[Q];
+  uint32_t lo = 0xFFFFFFFFu, hi = 0u;
+#pragma unroll
+  for (int k = 0; k < Q; ++k) {
+    const int ip = lane + 32 * k;
+    eb[k] = 0u;
+    if (ip < P) {
+      const float e = __ll2float_rn(x[ip]), o = __ll2float_rn(x[P + ip]);
+      eb[k] = __float_as_uint(__fmaf_rn(e, e, __fmul_rn(o, o)));
+      lo = min(lo, eb[k]);
+      hi = max(hi, eb[k]);
+    }
+  }
+  const uint32_t tmn = __reduce_min_sync(0xffffffffu, lo) + 32u;   // finite estimates: no overflow
+  const uint32_t mxb = __reduce_max_sync(0xffffffffu, hi);
+  const uint32_t tmx = mxb > 32u ? mxb - 32u : 0u;
+  float2 mn = make_float2(3.4028234663852886e38f, 0.f), mx = make_float2(0.f, 0.f);
+  bool cmn = false, cmx = false;
+#pragma unroll
+  for (int k = 0; k < Q; ++k) {
+    const int ip = lane + 32 * k;
+    if (ip < P && (eb[k] <= tmn || eb[k] >= tmx)) {
+      const float2 se = df_energy(make_longlong2(x[ip], x[P + ip]));
+      if (eb[k] <= tmn) { cmn = true; if (df_less(se, mn)) mn = se; }
+      if (eb[k] >= tmx) { cmx = true; if (df_less(mx, se)) mx = se; }
+    }
+  }
+  const unsigned bmn = __ballot_sync(0xffffffffu, cmn), bmx = __ballot_sync(0xffffffffu, cmx);
+  if (__popc(bmn) > 1 || __popc(bmx) > 1) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const float2 omn = make_float2(__shfl_xor_sync(0xffffffffu, mn.x, off), __shfl_xor_sync(0xffffffffu, mn.y, off));
+      const float2 omx = make_float2(__shfl_xor_sync(0xffffffffu, mx.x, off), __shfl_xor_sync(0xffffffffu, mx.y, off));
+      if (df_less(omn, mn)) mn = omn;
+      if (df_less(mx, omx)) mx = omx;
+    }
+    smn = mn;
+    smx = mx;
+  } else {
+    const int a = __ffs(bmn) - 1, b = __ffs(bmx) - 1;
+    smn = make_float2(__shfl_sync(0xffffffffu, mn.x, a), __shfl_sync(0xffffffffu, mn.y, a));
+    smx = make_float2(__shfl_sync(0xffffffffu, mx.x, b), __shfl_sync(0xffffffffu, mx.y, b));
+  }
+}
+
+// Works through qn entries of the queue (all lanes of a warp call it), 32 at a
+// time, one entry a lane: first the second look at each angle and norm code;
+// then, warp-wide and a row at a time, the exact transform of every row that
+// still has codes left (a row's entries are consecutive in the queue), from
+// which each lane takes its entry's exact sums and the row's exact extreme
+// energies; last, each lane decides its own code.  The records in global
+// memory are patched.  scratch: 2P longs of the warp's shared memory.
 template <int D, typename TIn, int N, int B, int MODE>
-__device__ __noinline__ void flush_queue(const EncParams* p, uint4* q, int qn, long long* scratch, int lane) {
+__device__ __forceinline__ void flush_queue(const EncParams* p, const uint4* q, int qn, long long* scratch, int lane) {
   constexpr int P = Geo<D>::P;
   constexpr int W = code_bits(N);
   constexpr bool FP32N = MODE == TAC_NORM_FP32;
   constexpr int AB = P * W / 8, NB = P * (FP32N ? 32 : B) / 8;
   constexpr int kB = 4;                                 // rows whose loads are in flight together
-  __syncwarp();
   auto record = [&](const EncJob& J, long long row, uint8_t*& codes, uint8_t*& norms) -> bool {
     const long long sl = J.slot ? J.slot[row] : row;
     if (sl < 0 || sl >= J.capacity) return false;   // skipped slots get no record
@@ -634,121 +709,132 @@ __device__ __noinline__ void flush_queue(const EncParams* p, uint4* q, int qn, l
     norms = J.norms + sl * NB;
     return true;
   };
-  auto settled = [&](int e) { return ((q[2 * e].x >> 14) & 3u) == 3u; };
-  // The rows of the entries left after the second look are read again from
-  // global memory; ask for all of them now, so that their latency (long
-  // while the encoder streams) passes during the second look.
-  for (int e = lane; e < qn; e += 32) {
-    const uint4 a = q[2 * e];
-    const EncJob& J = p->job[a.x & 0xFFu];
-    const char* row = reinterpret_cast<const char*>(J.x) + (long long)a.y * J.stride * (long long)sizeof(TIn);
-#pragma unroll
-    for (int c = 0; c < D * (int)sizeof(TIn); c += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(row + c));
-  }
-  if constexpr (!FP32N) {
-    for (int e = lane; e < qn; e += 32) {
-      const uint4 a = q[2 * e];
-      if (((a.x >> 14) & 3u) != 1u) continue;
-      const uint4 b = q[2 * e + 1];
-      const int c = norm_second_look<D, B, MODE>(__uint_as_float(a.z), __uint_as_float(a.w), __uint_as_float(b.x),
-                                                 __uint_as_float(b.y));
-      if (c < 0) continue;
-      const EncJob& J = p->job[a.x & 0xFFu];
-      uint8_t *codes, *norms;
-      if (record(J, (long long)a.y, codes, norms)) patch_bits(norms, (int)((a.x >> 8) & 63u) * B, B, (uint32_t)c);
-      q[2 * e].x = a.x | (3u << 14);
+  auto row_src = [&](const EncJob& J, uint32_t row) {
+    return reinterpret_cast<const uint8_t*>(J.x) + (long long)row * J.stride * (long long)sizeof(TIn);
+  };
+  __syncwarp();
+  for (int base = 0; base < qn; base += 32) {
+    const int e = base + lane;
+    uint4 a = make_uint4(0u, 0u, 0u, 0u), b = a;
+    uint32_t kind = 3u;
+    if (e < qn) {
+      a = q[2 * e];
+      b = q[2 * e + 1];
+      kind = (a.x >> 14) & 3u;
     }
-    __syncwarp();
-  }
-  // The rest, a batch of up to kB rows at a time (a row's entries are
-  // consecutive): the rows' loads are issued together so that their latencies
-  // overlap, then each row is transformed exactly and its codes decided.
-  int e = 0;
-  while (true) {
-    int bs[kB], be[kB], nb = 0;
-#pragma unroll
-    for (int b = 0; b < kB; ++b) {
-      bs[b] = be[b] = qn;
-      while (e < qn && settled(e)) ++e;
-      if (e < qn) {
-        const uint4 a = q[2 * e];
-        int g = e + 1;
-        while (g < qn && (q[2 * g].x & 0xFFu) == (a.x & 0xFFu) && q[2 * g].y == a.y) ++g;
-        bs[b] = e;
-        be[b] = g;
-        nb = b + 1;
-        e = g;
+    const uint32_t ej = a.x & 0xFFu;
+    const int v = (int)((a.x >> 8) & 63u);
+    // ---- second look ----
+    int c = -1;
+    if (kind == 0u) {
+      c = angle_second_look<D, N>(__uint_as_float(a.z), __uint_as_float(a.w), __uint_as_float(b.y));
+    } else if (kind == 1u) {
+      if constexpr (!FP32N)
+        c = norm_second_look<D, B, MODE>(__uint_as_float(a.z), __uint_as_float(a.w), __uint_as_float(b.x),
+                                         __uint_as_float(b.y));
+    }
+    if (c >= 0) {
+      uint8_t *codes, *norms;
+      if (record(p->job[ej], (long long)a.y, codes, norms)) {
+        if (kind == 0u) patch_bits(codes, v * W, W, (uint32_t)c);
+        else patch_bits(norms, v * B, B, (uint32_t)c);
       }
     }
-    if (nb == 0) break;
-    RowWords<D, TIn> rw[kB];
+    const bool need = kind != 3u && c < 0;
+    const unsigned nm = __ballot_sync(0xffffffffu, need);
+    if (nm == 0u) continue;
+    // ---- rows left: runs of needed entries of one (job, row) ----
+    const unsigned below = nm & ((1u << lane) - 1u);
+    const int pl = below ? 31 - __clz(below) : lane;
+    const uint32_t pj = __shfl_sync(0xffffffffu, ej, pl), pr = __shfl_sync(0xffffffffu, a.y, pl);
+    const bool start = need && (below == 0u || pj != ej || pr != a.y);
+    unsigned sm = __ballot_sync(0xffffffffu, start);
+    const unsigned upto = sm & (lane == 31 ? 0xFFFFFFFFu : ((2u << lane) - 1u));
+    const int mys = need ? 31 - __clz(upto) : -1;     // the lane that starts this lane's row
+    longlong2 eo = make_longlong2(0, 0);
+    float2 smn = make_float2(0.f, 0.f), smx = make_float2(0.f, 0.f);
+    while (sm != 0u) {
+      int rs[kB], nb = 0;
 #pragma unroll
-    for (int b = 0; b < kB; ++b) {
-      if (b < nb) {
-        const uint4 a = q[2 * bs[b]];
-        const EncJob& J = p->job[a.x & 0xFFu];
-        load_row_words<D, TIn>(reinterpret_cast<const uint8_t*>(J.x) + (long long)a.y * J.stride * (long long)sizeof(TIn),
-                               rw[b], lane);
+      for (int r = 0; r < kB; ++r) {
+        rs[r] = 0;
+        if (sm != 0u) { rs[r] = __ffs(sm) - 1; sm &= sm - 1u; nb = r + 1; }
       }
-    }
+      RowWords<D, TIn> rw[kB];
+      uint32_t rj[kB], rr[kB];
 #pragma unroll
-    for (int b = 0; b < kB; ++b) {
-      if (b >= nb) continue;
-      const uint4 a0 = q[2 * bs[b]];
-      const EncJob& J = p->job[a0.x & 0xFFu];
-      uint8_t *codes, *norms;
-      if (!record(J, (long long)a0.y, codes, norms)) continue;
-      FixWords<D, TIn> fw;
-      fix_words<D, TIn>(J, rw[b], fw, lane);
-      exact_row<D, TIn>(fw, scratch, lane);
-      bool have_ext = false;
-      float2 smn = make_float2(0.f, 0.f), smx = make_float2(0.f, 0.f);
-      for (int f = bs[b]; f < be[b]; ++f) {
-        const uint4 a = q[2 * f];
-        const uint32_t kind = (a.x >> 14) & 3u;
-        if (kind == 3u) continue;
-        if (kind != 0u && !have_ext) {
-          have_ext = true;
-          if constexpr (!FP32N) {
-            // exact extremes of the pair energies
-            smn = make_float2(3.4028234663852886e38f, 0.f);
-            smx = make_float2(0.f, 0.f);
+      for (int r = 0; r < kB; ++r) {
+        rj[r] = __shfl_sync(0xffffffffu, ej, rs[r]);
+        rr[r] = __shfl_sync(0xffffffffu, a.y, rs[r]);
+        if (r < nb) load_row_words<D, TIn>(row_src(p->job[rj[r]], rr[r]), rw[r], lane);
+      }
+#pragma unroll
+      for (int r = 0; r < kB; ++r) {
+        if (r >= nb) continue;
+        const EncJob& R = p->job[rj[r]];
+        FixWords<D, TIn> fw;
+        fix_words<D, TIn>(R, rw[r], fw, lane);
+        exact_row<D, TIn>(fw, scratch, lane);
+        const bool mine = mys == rs[r];
+        float2 rmn = make_float2(0.f, 0.f), rmx = make_float2(0.f, 0.f);
+        if constexpr (!FP32N) {
+          if (__ballot_sync(0xffffffffu, mine && kind != 0u) != 0u) exact_extremes<D>(scratch, lane, rmn, rmx);
+        }
+        if (mine) {
+          smn = rmn;
+          smx = rmx;
+          if (kind != 2u) {
+            const int ip = slot_pair<D>(v);
+            eo = make_longlong2(scratch[ip], scratch[P + ip]);
+          }
+        }
+        if (__ballot_sync(0xffffffffu, mine && kind == 2u) != 0u) {   // the whole row, a pair a lane
+          uint8_t *codes, *norms;
+          if (record(R, (long long)rr[r], codes, norms)) {
             for (int ip = lane; ip < P; ip += 32) {
-              const float2 se = df_energy(make_longlong2(scratch[ip], scratch[P + ip]));
-              if (df_less(se, smn)) smn = se;
-              if (df_less(smx, se)) smx = se;
-            }
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) {
-              const float2 omn = make_float2(__shfl_xor_sync(0xffffffffu, smn.x, off), __shfl_xor_sync(0xffffffffu, smn.y, off));
-              const float2 omx = make_float2(__shfl_xor_sync(0xffffffffu, smx.x, off), __shfl_xor_sync(0xffffffffu, smx.y, off));
-              if (df_less(omn, smn)) smn = omn;
-              if (df_less(smx, omx)) smx = omx;
+              const longlong2 pe = make_longlong2(scratch[ip], scratch[P + ip]);
+              const int vs = pair_slot<D>(ip);
+              patch_bits(codes, vs * W, W, (uint32_t)fix_angle_code<N>(pe));
+              if constexpr (!FP32N)
+                patch_bits(norms, vs * B, B, (uint32_t)fix_norm_code<B, MODE>(df_energy(pe), rmn, rmx));
             }
           }
         }
-        if (kind == 2u) {   // the whole row, a pair a lane
-          for (int ip = lane; ip < P; ip += 32) {
-            const longlong2 eo = make_longlong2(scratch[ip], scratch[P + ip]);
-            const int v = pair_slot<D>(ip);
-            patch_bits(codes, v * W, W, (uint32_t)fix_angle_code<N>(eo));
-            if constexpr (!FP32N) patch_bits(norms, v * B, B, (uint32_t)fix_norm_code<B, MODE>(df_energy(eo), smn, smx));
-          }
+        __syncwarp();
+      }
+    }
+    // ---- exact decisions, one entry a lane ----
+    if (need && kind != 2u) {
+      uint8_t *codes, *norms;
+      if (record(p->job[ej], (long long)a.y, codes, norms)) {
+        if (kind == 0u) {
+          patch_bits(codes, v * W, W, (uint32_t)fix_angle_code<N>(eo));
         } else {
-          const int v = (int)((a.x >> 8) & 63u);
-          const int ip = slot_pair<D>(v);
-          const longlong2 eo = make_longlong2(scratch[ip], scratch[P + ip]);
-          if (kind == 0u) {
-            const int k = fix_angle_code<N>(eo);
-            if (lane == 0) patch_bits(codes, v * W, W, (uint32_t)k);
-          } else if constexpr (!FP32N) {
-            const int c = fix_norm_code<B, MODE>(df_energy(eo), smn, smx);
-            if (lane == 0) patch_bits(norms, v * B, B, (uint32_t)c);
-          }
+          if constexpr (!FP32N) patch_bits(norms, v * B, B, (uint32_t)fix_norm_code<B, MODE>(df_energy(eo), smn, smx));
         }
       }
-      __syncwarp();
     }
+  }
+  __syncwarp();
+}
+
+// Moves a warp's qn queued entries to the launch's queue in global memory
+// (one atomic add reserves their places).  Entries beyond its capacity set
+// their row's bit in ovf instead: the fix-up kernel then re-decides that row
+// whole.
+template <int D>
+__device__ __forceinline__ void spill_queue(const EncParams& p, const uint4* q, int qn, int lane) {
+  __syncwarp();
+  unsigned long long base = 0;
+  if (lane == 0) base = atomicAdd(p.gq_n, (unsigned long long)qn);
+  base = __shfl_sync(0xffffffffu, base, 0);
+  const unsigned long long cap = (unsigned long long)p.gq_cap;
+  const int fit = base >= cap ? 0 : (int)min((unsigned long long)qn, cap - base);
+  for (int i = lane; i < 2 * fit; i += 32) p.gq[2 * base + i] = q[i];
+  for (int e = fit + lane; e < qn; e += 32) {
+    const uint4 a = q[2 * e];
+    const long long bit = (long long)p.job[a.x & 0xFFu].tile0 * Geo<D>::RW + a.y;
+    atomicOr(p.ovf + (bit >> 5), 1u << (bit & 31));
   }
   __syncwarp();
 }
@@ -1106,8 +1192,9 @@ __device__ __forceinline__ void tile_body(const uint8_t* in, uint8_t* wsm, const
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           if ((fl >> j) & 1u) {
-            e[0] = make_uint4(hd | ((uint32_t)(8 * l + j) << 8), row, 0u, 0u);
-            e[1] = make_uint4(0u, 0u, 0u, 0u);
+            e[0] = make_uint4(hd | ((uint32_t)(8 * l + j) << 8), row, __float_as_uint(v[j].x),
+                              __float_as_uint(v[j].y));
+            e[1] = make_uint4(0u, __float_as_uint(ty), 0u, 0u);
             e += 2;
           }
         }
@@ -1271,16 +1358,13 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
   uint2 msk[8];
 #pragma unroll
   for (int m = 0; m < 8; ++m) msk[m] = make_uint2(0u, 0u);
-  // re-decision queue: qn entries (warp-uniform), drained when fewer than
-  // one tile's worst case of free entries is left, and at the end
+  // re-decision queue: qn entries (warp-uniform), moved to the launch's queue
+  // in global memory when fewer than one tile's worst case of free entries is
+  // left, and at the end
   using QG = QGeo<D>;
   uint4* const qb = reinterpret_cast<uint4*>(wsm + C::W_Q);
-  long long* const scr = reinterpret_cast<long long*>(wsm + C::W_SCR);
   int qn = 0;
-  // Drain threshold, staggered over the warps (up to 28 entries apart) so that
-  // the warps of an SM, whose queues fill at about the same rate, do not all
-  // drain at the same time.
-  const int q_hi = kQ - QG::kMaxPerTile - 4 * (gw & 7);
+  constexpr int q_hi = kQ - QG::kMaxPerTile;
 
   static_assert((kNS & (kNS - 1)) == 0, "stage ring size");
   int stage = 0;
@@ -1296,7 +1380,7 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
       // cursors are settled once after it.
       const int t_start = t, t_stop = t + fast;
       for (; t < t_stop; ++t) {
-        if (qn > q_hi) break;   // the general iteration drains the queue first
+        if (qn > q_hi) break;   // the general iteration moves the queue first
         cp_async_wait<kNS - 2>();   // this warp tile has landed
         __syncwarp();               // ... and every lane is done with the previous one
         uint8_t* dst = in_dst + ((stage + kNS - 1) & (kNS - 1)) * IT::BYTES;
@@ -1326,10 +1410,9 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
     }
 
     // ---- general tile: a job's first tile, tails, scattered slots, range ends,
-    // and the queue's drains (here only, so that the stretches stay free of calls) ----
+    // and the queue's moves to global memory ----
     if (qn > q_hi) {
-      __syncwarp();
-      flush_queue<D, TIn, N, B, MODE>(&p, qb, qn, scr, lane);
+      spill_queue<D>(p, qb, qn, lane);
       qn = 0;
     }
     cp_async_wait<kNS - 2>();
@@ -1391,11 +1474,56 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
     const int64_t f = min(cf, pf);
     fast = f > 0 ? (int)f : 0;
   }
-  if (qn > 0) {
-    __syncwarp();
-    flush_queue<D, TIn, N, B, MODE>(&p, qb, qn, scr, lane);
-  }
+  if (qn > 0) spill_queue<D>(p, qb, qn, lane);
   cp_async_wait<0>();
+}
+
+// ---------------------------------------------------------------------------
+// Fix-up of one encode launch (same stream, after it): the queue's entries, 32
+// to a warp (the second look, then the exact path for the codes it leaves),
+// then the rows whose entries found the queue full, each re-decided whole.
+// Grid-stride over both, so any grid size covers them.
+// ---------------------------------------------------------------------------
+constexpr int kFixWarps = 4;
+
+template <int D, typename TIn, int N, int B, int MODE>
+__global__ void __launch_bounds__(32 * kFixWarps) encode_fixup_kernel(const __grid_constant__ EncParams p) {
+  constexpr int P = Geo<D>::P, RW = Geo<D>::RW;
+  __shared__ long long scratch[kFixWarps][2 * P];
+  __shared__ uint4 whole[kFixWarps][2];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long GW = (long long)gridDim.x * kFixWarps, gw = (long long)blockIdx.x * kFixWarps + warp;
+  const unsigned long long appended = *p.gq_n;
+  const long long n = (long long)min(appended, (unsigned long long)p.gq_cap);
+  for (long long c = gw; 32 * c < n; c += GW)
+    flush_queue<D, TIn, N, B, MODE>(&p, p.gq + 64 * c, (int)min(32LL, n - 32 * c), scratch[warp], lane);
+  if (appended <= (unsigned long long)p.gq_cap) return;
+  const long long nwords = ((long long)p.ntiles * RW + 31) / 32;
+  for (long long w0 = gw * 32; w0 < nwords; w0 += GW * 32) {
+    const long long wi = w0 + lane;
+    const uint32_t word = wi < nwords ? p.ovf[wi] : 0u;
+    unsigned live = __ballot_sync(0xffffffffu, word != 0u);
+    while (live != 0u) {
+      const int src = __ffs(live) - 1;
+      live &= live - 1u;
+      uint32_t bits = __shfl_sync(0xffffffffu, word, src);
+      while (bits != 0u) {
+        const int b = __ffs(bits) - 1;
+        bits &= bits - 1u;
+        const long long bit = (w0 + src) * 32 + b;
+        const int j = find_job(p, (int)(bit / RW));
+        const long long row = bit - (long long)p.job[j].tile0 * RW;
+        if (row >= p.job[j].rows) continue;
+        __syncwarp();
+        if (lane == 0) {
+          whole[warp][0] = make_uint4((uint32_t)j | (2u << 14), (uint32_t)row, 0u, 0u);
+          whole[warp][1] = make_uint4(0u, 0u, 0u, 0u);
+        }
+        __syncwarp();
+        flush_queue<D, TIn, N, B, MODE>(&p, whole[warp], 1, scratch[warp], lane);
+      }
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1422,6 +1550,18 @@ static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_
   if (grid > need) grid = need;
   if (grid < 1) return cudaSuccess;
   kern<<<grid, kEncThreads, C::SMEM, st>>>(p);
+  cudaError_t le = cudaGetLastError();
+  if (le != cudaSuccess) return le;
+  // the fix-up: enough warps for the queue's capacity, up to a full GPU
+  auto fix = encode_fixup_kernel<D, TIn, N, B, MODE>;
+  int fix_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&fix_sm, fix, 32 * kFixWarps, 0);
+  if (e != cudaSuccess) return e;
+  const int64_t chunks = (p.gq_cap + 31) / 32;
+  int64_t fgrid = (int64_t)grid_cap * (fix_sm < 1 ? 1 : fix_sm);
+  fgrid = std::min<int64_t>(fgrid, (chunks + kFixWarps - 1) / kFixWarps);
+  if (fgrid < 1) fgrid = 1;
+  fix<<<(int)fgrid, 32 * kFixWarps, 0, st>>>(p);
   return cudaGetLastError();
 }
 

@@ -168,6 +168,35 @@ def test_invalid_arguments_rejected_before_launch(tac_host):
     assert lib.tac_make_signs_shared(0, 0, s) == tac_host.TAC_E_INVAL
 
 
+def test_encode_workspace_size_and_checks(tac_host):
+    """tac_encode_workspace_bytes: per launch group a 64-byte counter block and
+    one bit per warp-tile row (rounded up to 16 bytes) are the minimum; the
+    recommended size adds a queue of one 32-byte entry per 512 angle pairs plus
+    1024.  tac_encode_multi_ws rejects a NULL, misaligned or too small
+    workspace before any device work."""
+    lib = tac_host.load()
+    rows = tac_host._Rows()
+    rows.data, rows.dtype, rows.rows, rows.row_stride = 16, 0, 1000, 128
+    buf = 4096
+    jobs = (tac_host._EncJob * 2)()
+    for i, (n, b) in enumerate(((64, 8), (256, 4))):   # two kernel shapes: two groups
+        jobs[i].cfg = _cfg(tac_host, n=n, b=b, mode=i)
+        jobs[i].x = rows
+        jobs[i].codes, jobs[i].norms, jobs[i].capacity, jobs[i].slot = buf, buf, 1000, None
+    mn = ctypes.c_int64(0)
+    rec = lib.tac_encode_workspace_bytes(jobs, 2, ctypes.byref(mn))
+    per_min = 64 + ((250 * 4 + 127) // 128) * 16          # d = 128: 4-row warp tiles
+    assert mn.value == 2 * per_min
+    assert rec == 2 * (per_min + 32 * (1000 * 64 // 512 + 1024))
+    assert lib.tac_encode_workspace_bytes(jobs, 2, None) == rec
+    assert lib.tac_encode_workspace_bytes(None, 2, None) == -1
+    assert lib.tac_encode_multi_ws(jobs, 2, None, rec, None) == tac_host.TAC_E_INVAL
+    assert lib.tac_encode_multi_ws(jobs, 2, buf + 8, rec, None) == tac_host.TAC_E_INVAL
+    assert lib.tac_encode_multi_ws(jobs, 2, buf, mn.value - 16, None) == tac_host.TAC_E_INVAL
+    assert lib.tac_encode_multi_ws(None, 0, None, 0, None) == tac_host.TAC_OK
+    assert lib.tac_encode_workspace_bytes(None, 0, ctypes.byref(mn)) == 0 and mn.value == 0
+
+
 def test_empty_calls_succeed_without_device(tac_host):
     lib = tac_host.load()
     rows = tac_host._Rows()

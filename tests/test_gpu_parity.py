@@ -334,3 +334,32 @@ def test_nonfinite_rows(tac_gpu, orc, dt, b, mode):
     tac_gpu.encode(x[torch.from_numpy(good).cuda()].contiguous(), cfg, status=status)
     torch.cuda.synchronize()
     assert int(status.item()) == 0
+
+
+@pytest.mark.parametrize("room", ["min", "partial"])
+def test_small_workspace_rows_redecided_whole(tac_gpu, orc, room):
+    """With the minimum workspace (no queue room) every queued code's row is
+    re-decided whole through the bitmap; with a queue of a few dozen entries
+    some codes go through the queue and the rest of the rows whole.  The
+    records satisfy the same parity rule as with the recommended workspace."""
+    torch = _torch()
+    w = workloads.CONFIGS["mistral7b"]
+    for kv in (workloads.K, workloads.V):
+        d, n, b, mode = w.codebook(0, kv)
+        x = _rows(w, 6000, seed=5, layer=0, kv=kv)
+        cfg = tac_gpu.layer_cfg(d, n, b, mode, 0, 0, kv)
+        cache = tac_gpu.Cache.empty(cfg, x.shape[0])
+        jobs = [tac_gpu.EncodeJob(cfg, x, cache)]
+        rec, mn = tac_gpu.encode_workspace_bytes(jobs)
+        size = mn if room == "min" else mn + 32 * 40
+        wsb = torch.empty(size, dtype=torch.uint8, device="cuda")
+        tac_gpu.encode_multi(jobs, workspace=wsb)
+        torch.cuda.synchronize()
+        x64 = parity.to_f64(x)
+        s = orc.signs(0, 0, kv, d)
+        ref = orc.encode(x64, s, n, b, mode)
+        k, c, hdr = parity.gpu_codes(orc, cache, x.shape[0])
+        parity.compare_encode(orc, x64, ref, k, c, hdr, n, b, mode, label=f"workspace {room} kv={kv}")
+        # the queue overflowed: the counter passed the queue's capacity
+        appended = int(wsb[:8].cpu().numpy().view(np.uint64)[0])
+        assert appended > (0 if room == "min" else 40), appended
