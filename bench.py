@@ -36,16 +36,17 @@ METRIC = "KV encode / decode GB/s (bf16 in/out) on 1 GB300 and % of HBM peak"
 UNIT = "GB/s"
 FALLBACK_HBM_GBS = 6800.0
 
-# DRAM bytes per encoded/decoded row that ncu counted (dram__bytes_read.sum +
-# dram__bytes_write.sum of one launch of the 4096-token Mistral-7B-shaped case,
-# divided by its 2,097,152 rows; the full-size launch has the same codebook mix,
-# so its traffic is this figure times its rows).  Each figure holds only for the
+# DRAM bytes per encoded/decoded row that ncu counted: dram__bytes_read.sum +
+# dram__bytes_write.sum over every launch of one call (encode: the encode and
+# fix-up kernels of each shape) of the 8192-token Mistral-7B-shaped case,
+# divided by its 4,194,304 rows; the full-size call has the same codebook mix,
+# so its traffic is this figure times its rows.  Each figure holds only for the
 # kernel sources it was measured on; after any change to them it reads null.
 MEASURED_TRAFFIC = {
-    "encode": {"sources": ("tac_common.cuh", "tac_encode.cu"), "sha256_16": "4987b67da26c92a9",
-               "bytes_per_row": 319.101},
-    "decode": {"sources": ("tac_common.cuh", "tac_decode.cu"), "sha256_16": "67d77e3f7ce52de4",
-               "bytes_per_row": 272.694},
+    "encode": {"sources": ("tac_common.cuh", "tac_encode.cu"), "sha256_16": "b5e9e4daa232deed",
+               "bytes_per_row": 338.717},
+    "decode": {"sources": ("tac_common.cuh", "tac_decode.cu"), "sha256_16": "2311f3a110360433",
+               "bytes_per_row": 305.526},
     "attend": {"sources": ("tac_common.cuh", "tac_attend.cuh", "tac_attend.cu"), "sha256_16": "2ca20d9ce47a635b",
                "bytes_per_row": 216.889},
 }
