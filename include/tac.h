@@ -234,7 +234,8 @@ int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream)
  * tac_encode_workspace_bytes returns the recommended size for the call
  * tac_encode_multi_ws(jobs, njobs, ...) (queue room for one code in 512 of
  * every group, far above the rates of the paper's workloads) and stores the
- * minimum in *min_bytes (if not NULL): a counter block and one bit per row.
+ * minimum in *min_bytes (if not NULL): per launch a counter block, one bit per
+ * row and a copy of the launch's job table.
  * With less than the recommended size the queues shrink; a code that finds its
  * queue full has its whole row re-decided instead, so the results do not depend
  * on the size, only the time does.  Returns -1 (tac_last_error) for a call

@@ -467,8 +467,9 @@ int plan_encode(const tac_encode_job* jobs, int njobs, const char* who, std::vec
 }
 
 // Workspace of an encode call: per launch group a 64-byte counter block and a
-// bitmap of its warp-tile rows (together the part zeroed at the call), then
-// per group its re-decision queue, 32-byte entries.  The queue's recommended
+// bitmap of its warp-tile rows (together the part zeroed at the call), per
+// group a copy of its job table (written by the encode kernel, read by the
+// fix-up kernel), then per group its re-decision queue, 32-byte entries.  The queue's recommended
 // capacity is one entry per 512 angle pairs plus 1024 (the synthetic caches
 // of every workload queue about one per 2400 pairs); with less room the
 // capacities shrink in proportion, down to none (then every row with a code to
@@ -478,23 +479,27 @@ int64_t enc_ovf_bytes(const EncGroup& G) {
   const int64_t bits = (int64_t)G.p.ntiles * tile_rows(G.d);
   return ((bits + 127) / 128) * 16;
 }
+int64_t enc_job_bytes(const EncGroup& G) {
+  return (((int64_t)G.p.njobs * (int64_t)sizeof(tac::EncJob) + 15) / 16) * 16;
+}
 int64_t enc_rec_cap(const EncGroup& G) {
   int64_t pairs = 0;
   for (int j = 0; j < G.p.njobs; ++j) pairs += G.p.job[j].rows * (G.d / 2);
   return pairs / 512 + 1024;
 }
 struct EncWs {
-  int64_t zero = 0, min = 0, rec = 0, rec_entries = 0;
+  int64_t zero = 0, jobs = 0, min = 0, rec = 0, rec_entries = 0;
 };
 EncWs enc_ws(const std::vector<EncGroup>& groups) {
   EncWs w;
   w.zero = kEncCtrBytes * (int64_t)groups.size();
   for (const EncGroup& G : groups) {
     w.zero += enc_ovf_bytes(G);
+    w.jobs += enc_job_bytes(G);
     w.rec_entries += enc_rec_cap(G);
   }
-  w.min = w.zero;
-  w.rec = w.zero + kEncEntryBytes * w.rec_entries;
+  w.min = w.zero + w.jobs;
+  w.rec = w.min + kEncEntryBytes * w.rec_entries;
   return w;
 }
 
@@ -503,8 +508,8 @@ int run_encode(std::vector<EncGroup>& groups, uint8_t* ws, int64_t ws_bytes, cud
   const int sms = num_sms();
   if (sms <= 0) return fail(TAC_E_CUDA, "%s: no CUDA device", who);
   const EncWs w = enc_ws(groups);
-  const int64_t avail = (ws_bytes - w.zero) / kEncEntryBytes;
-  int64_t ovf_off = kEncCtrBytes * (int64_t)groups.size(), q_off = w.zero;
+  const int64_t avail = (ws_bytes - w.min) / kEncEntryBytes;
+  int64_t ovf_off = kEncCtrBytes * (int64_t)groups.size(), job_off = w.zero, q_off = w.min;
   for (size_t g = 0; g < groups.size(); ++g) {
     tac::EncParams& P = groups[g].p;
     const int64_t rc = enc_rec_cap(groups[g]);
@@ -513,7 +518,9 @@ int run_encode(std::vector<EncGroup>& groups, uint8_t* ws, int64_t ws_bytes, cud
     P.ovf = reinterpret_cast<uint32_t*>(ws + ovf_off);
     P.gq = reinterpret_cast<uint4*>(ws + q_off);
     P.gq_cap = cap;
+    P.gjobs = reinterpret_cast<tac::EncJob*>(ws + job_off);
     ovf_off += enc_ovf_bytes(groups[g]);
+    job_off += enc_job_bytes(groups[g]);
     q_off += kEncEntryBytes * cap;
   }
   cudaError_t e = cudaMemsetAsync(ws, 0, (size_t)w.zero, st);

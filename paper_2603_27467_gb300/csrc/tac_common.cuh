@@ -139,6 +139,8 @@ struct EncJob {
   int32_t tile0;       // first global tile of this job
 };
 
+static_assert(sizeof(EncJob) == 104 && sizeof(EncJob) % 8 == 0, "EncJob: the workspace copy is sized by it");
+
 struct EncParams {
   int32_t njobs;
   int32_t ntiles;
@@ -149,7 +151,20 @@ struct EncParams {
   uint32_t* ovf;               // one bit per warp-tile row (tile * RW + row in tile): rows
                                // whose entries found the queue full, re-decided whole
   int64_t gq_cap;
+  EncJob* gjobs;               // workspace copy of job[0, njobs), written by the encode kernel
   EncJob job[TAC_MAX_JOBS];
+};
+
+// Parameters of the encode's fix-up kernel (small: the job table is read from
+// the copy the encode kernel leaves in the workspace).
+struct FixParams {
+  const EncJob* job;
+  uint4* gq;
+  unsigned long long* gq_n;
+  uint32_t* ovf;
+  int64_t gq_cap;
+  int32_t njobs;
+  int32_t ntiles;
 };
 
 struct DecJob {

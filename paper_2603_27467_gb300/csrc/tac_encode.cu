@@ -302,7 +302,7 @@ __device__ __forceinline__ float2 df_energy(longlong2 eo) {
 // m = E cos psi - O sin psi in double-float against the double-float edge
 // direction (the code is the next bin when m >= 0).
 template <int N>
-__device__ __forceinline__ int fix_angle_code(longlong2 eo) {
+__device__ __noinline__ int fix_angle_code(longlong2 eo) {
   if (eo.x == 0 && eo.y == 0) return 0;  // pair (0, 0) -> bin 0
   const float2 e = ll_to_df(eo.x), o = ll_to_df(eo.y);
   const int ec = candidate_edge<N>(e.x, o.x);
@@ -350,7 +350,7 @@ __device__ __forceinline__ void df_pow(float2 a, int n, float2& m, int& e) {
 }
 
 // rho1^n1 >= rho2^n2 for double-floats rho >= 1 and n >= 0.
-__device__ __forceinline__ bool df_pow_ge(float2 r1, int n1, float2 r2, int n2) {
+static __device__ __noinline__ bool df_pow_ge(float2 r1, int n1, float2 r2, int n2) {
   float2 m1, m2;
   int e1, e2;
   df_pow(r1, n1, m1, e1);
@@ -372,7 +372,7 @@ __device__ __forceinline__ bool df_pow_ge(float2 r1, int n1, float2 r2, int n2) 
 // double-float; log-space by (s/s_lo)^(2 Lq) >= (s_max/s_lo)^(2c - 1), the
 // same inequality raised to integer powers.
 template <int B, int MODE>
-__device__ __forceinline__ int fix_norm_code(float2 sa, float2 smn, float2 smx) {
+__device__ __noinline__ int fix_norm_code(float2 sa, float2 smn, float2 smx) {
   constexpr int Lq = (1 << B) - 1;
   int c;
   if constexpr (MODE == TAC_NORM_LINEAR) {
@@ -458,7 +458,7 @@ __device__ __forceinline__ constexpr float norm_kappa() { return D >= 64 ? 0.015
 // value lies farther than norm_kappa() times that bound from a rounding
 // midpoint, else -1.
 template <int D, int B, int MODE>
-__device__ __forceinline__ int norm_second_look(float s, float smin, float smax, float ty) {
+__device__ __noinline__ int norm_second_look(float s, float smin, float smax, float ty) {
   constexpr int Lq = (1 << B) - 1;
   constexpr float kappa = norm_kappa<D>();
   if constexpr (MODE == TAC_NORM_LINEAR) {
@@ -503,7 +503,7 @@ __device__ __forceinline__ int norm_second_look(float s, float smin, float smax,
 // always go on to the exact path: their fp32 angle may be off by more than the
 // candidate edge allows for.
 template <int D, int N>
-__device__ __forceinline__ int angle_second_look(float E, float O, float ty) {
+__device__ __noinline__ int angle_second_look(float E, float O, float ty) {
   const float s = __fmaf_rn(E, E, __fmul_rn(O, O));
   const float rthr = ty * (4.f * (float)N / 3.14159265f);
   if (s < rthr * rthr || !(s > 0.f)) return -1;
@@ -641,7 +641,7 @@ __device__ __forceinline__ void exact_row(const FixWords<D, TIn>& f, long long* 
 // candidates: the pairs whose estimate lies within 32 ulp of the smallest
 // (largest) estimate.  Only those get the double-float energy.
 template <int D>
-__device__ __forceinline__ void exact_extremes(const long long* x, int lane, float2& smn, float2& smx) {
+__device__ __noinline__ void exact_extremes(const long long* x, int lane, float2& smn, float2& smx) {
   constexpr int P = Geo<D>::P, Q = (P + 31) / 32;
   uint32_t eb[Q];
   uint32_t lo = 0xFFFFFFFFu, hi = 0u;
@@ -696,12 +696,11 @@ __device__ __forceinline__ void exact_extremes(const long long* x, int lane, flo
 // energies; last, each lane decides its own code.  The records in global
 // memory are patched.  scratch: 2P longs of the warp's shared memory.
 template <int D, typename TIn, int N, int B, int MODE>
-__device__ __forceinline__ void flush_queue(const EncParams* p, const uint4* q, int qn, long long* scratch, int lane) {
+__device__ __forceinline__ void flush_queue(const EncJob* jobs, const uint4* q, int qn, long long* scratch, int lane) {
   constexpr int P = Geo<D>::P;
   constexpr int W = code_bits(N);
   constexpr bool FP32N = MODE == TAC_NORM_FP32;
   constexpr int AB = P * W / 8, NB = P * (FP32N ? 32 : B) / 8;
-  constexpr int kB = 4;                                 // rows whose loads are in flight together
   auto record = [&](const EncJob& J, long long row, uint8_t*& codes, uint8_t*& norms) -> bool {
     const long long sl = J.slot ? J.slot[row] : row;
     if (sl < 0 || sl >= J.capacity) return false;   // skipped slots get no record
@@ -735,7 +734,7 @@ __device__ __forceinline__ void flush_queue(const EncParams* p, const uint4* q, 
     }
     if (c >= 0) {
       uint8_t *codes, *norms;
-      if (record(p->job[ej], (long long)a.y, codes, norms)) {
+      if (record(jobs[ej], (long long)a.y, codes, norms)) {
         if (kind == 0u) patch_bits(codes, v * W, W, (uint32_t)c);
         else patch_bits(norms, v * B, B, (uint32_t)c);
       }
@@ -754,59 +753,46 @@ __device__ __forceinline__ void flush_queue(const EncParams* p, const uint4* q, 
     longlong2 eo = make_longlong2(0, 0);
     float2 smn = make_float2(0.f, 0.f), smx = make_float2(0.f, 0.f);
     while (sm != 0u) {
-      int rs[kB], nb = 0;
-#pragma unroll
-      for (int r = 0; r < kB; ++r) {
-        rs[r] = 0;
-        if (sm != 0u) { rs[r] = __ffs(sm) - 1; sm &= sm - 1u; nb = r + 1; }
+      const int rs = __ffs(sm) - 1;
+      sm &= sm - 1u;
+      const uint32_t rj = __shfl_sync(0xffffffffu, ej, rs), rr = __shfl_sync(0xffffffffu, a.y, rs);
+      const EncJob& R = jobs[rj];
+      RowWords<D, TIn> rw;
+      load_row_words<D, TIn>(row_src(R, rr), rw, lane);
+      FixWords<D, TIn> fw;
+      fix_words<D, TIn>(R, rw, fw, lane);
+      exact_row<D, TIn>(fw, scratch, lane);
+      const bool mine = mys == rs;
+      float2 rmn = make_float2(0.f, 0.f), rmx = make_float2(0.f, 0.f);
+      if constexpr (!FP32N) {
+        if (__ballot_sync(0xffffffffu, mine && kind != 0u) != 0u) exact_extremes<D>(scratch, lane, rmn, rmx);
       }
-      RowWords<D, TIn> rw[kB];
-      uint32_t rj[kB], rr[kB];
-#pragma unroll
-      for (int r = 0; r < kB; ++r) {
-        rj[r] = __shfl_sync(0xffffffffu, ej, rs[r]);
-        rr[r] = __shfl_sync(0xffffffffu, a.y, rs[r]);
-        if (r < nb) load_row_words<D, TIn>(row_src(p->job[rj[r]], rr[r]), rw[r], lane);
-      }
-#pragma unroll
-      for (int r = 0; r < kB; ++r) {
-        if (r >= nb) continue;
-        const EncJob& R = p->job[rj[r]];
-        FixWords<D, TIn> fw;
-        fix_words<D, TIn>(R, rw[r], fw, lane);
-        exact_row<D, TIn>(fw, scratch, lane);
-        const bool mine = mys == rs[r];
-        float2 rmn = make_float2(0.f, 0.f), rmx = make_float2(0.f, 0.f);
-        if constexpr (!FP32N) {
-          if (__ballot_sync(0xffffffffu, mine && kind != 0u) != 0u) exact_extremes<D>(scratch, lane, rmn, rmx);
+      if (mine) {
+        smn = rmn;
+        smx = rmx;
+        if (kind != 2u) {
+          const int ip = slot_pair<D>(v);
+          eo = make_longlong2(scratch[ip], scratch[P + ip]);
         }
-        if (mine) {
-          smn = rmn;
-          smx = rmx;
-          if (kind != 2u) {
-            const int ip = slot_pair<D>(v);
-            eo = make_longlong2(scratch[ip], scratch[P + ip]);
+      }
+      if (__ballot_sync(0xffffffffu, mine && kind == 2u) != 0u) {   // the whole row, a pair a lane
+        uint8_t *codes, *norms;
+        if (record(R, (long long)rr, codes, norms)) {
+          for (int ip = lane; ip < P; ip += 32) {
+            const longlong2 pe = make_longlong2(scratch[ip], scratch[P + ip]);
+            const int vs = pair_slot<D>(ip);
+            patch_bits(codes, vs * W, W, (uint32_t)fix_angle_code<N>(pe));
+            if constexpr (!FP32N)
+              patch_bits(norms, vs * B, B, (uint32_t)fix_norm_code<B, MODE>(df_energy(pe), rmn, rmx));
           }
         }
-        if (__ballot_sync(0xffffffffu, mine && kind == 2u) != 0u) {   // the whole row, a pair a lane
-          uint8_t *codes, *norms;
-          if (record(R, (long long)rr[r], codes, norms)) {
-            for (int ip = lane; ip < P; ip += 32) {
-              const longlong2 pe = make_longlong2(scratch[ip], scratch[P + ip]);
-              const int vs = pair_slot<D>(ip);
-              patch_bits(codes, vs * W, W, (uint32_t)fix_angle_code<N>(pe));
-              if constexpr (!FP32N)
-                patch_bits(norms, vs * B, B, (uint32_t)fix_norm_code<B, MODE>(df_energy(pe), rmn, rmx));
-            }
-          }
-        }
-        __syncwarp();
       }
+      __syncwarp();
     }
     // ---- exact decisions, one entry a lane ----
     if (need && kind != 2u) {
       uint8_t *codes, *norms;
-      if (record(p->job[ej], (long long)a.y, codes, norms)) {
+      if (record(jobs[ej], (long long)a.y, codes, norms)) {
         if (kind == 0u) {
           patch_bits(codes, v * W, W, (uint32_t)fix_angle_code<N>(eo));
         } else {
@@ -1282,6 +1268,13 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
 #pragma unroll
     for (int c = 0; c < C::TABR; ++c) etab[e * C::TABR + c] = cs;
   }
+  // the job table, for the fix-up kernel
+  if (blockIdx.x == 0) {
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(p.job);
+    uint32_t* dst = reinterpret_cast<uint32_t*>(p.gjobs);
+    const int words = p.njobs * (int)(sizeof(EncJob) / 4);
+    for (int i = tid; i < words; i += kEncThreads) dst[i] = src[i];
+  }
   __syncthreads();
 
   // Each warp owns a contiguous range of warp tiles (balanced to +-1 tile), so
@@ -1479,15 +1472,18 @@ __global__ void __launch_bounds__(kEncThreads, kMinBlocks) encode_kernel(const _
 }
 
 // ---------------------------------------------------------------------------
-// Fix-up of one encode launch (same stream, after it): the queue's entries, 32
-// to a warp (the second look, then the exact path for the codes it leaves),
-// then the rows whose entries found the queue full, each re-decided whole.
-// Grid-stride over both, so any grid size covers them.
+// Fix-up of one encode launch (same stream, after it): the queue's entries,
+// kFixChunk to a warp (the second look, then the exact path for the codes it
+// leaves), then the rows whose entries found the queue full, each re-decided
+// whole.  Grid-stride over both, so any grid size covers them.  The work is
+// latency-bound (a warp takes its chunk's exact rows one after another), so
+// the chunks are short and the grid wide.
 // ---------------------------------------------------------------------------
 constexpr int kFixWarps = 4;
+constexpr int kFixChunk = 8;
 
 template <int D, typename TIn, int N, int B, int MODE>
-__global__ void __launch_bounds__(32 * kFixWarps) encode_fixup_kernel(const __grid_constant__ EncParams p) {
+__global__ void __launch_bounds__(32 * kFixWarps) encode_fixup_kernel(const __grid_constant__ FixParams p) {
   constexpr int P = Geo<D>::P, RW = Geo<D>::RW;
   __shared__ long long scratch[kFixWarps][2 * P];
   __shared__ uint4 whole[kFixWarps][2];
@@ -1495,8 +1491,9 @@ __global__ void __launch_bounds__(32 * kFixWarps) encode_fixup_kernel(const __gr
   const long long GW = (long long)gridDim.x * kFixWarps, gw = (long long)blockIdx.x * kFixWarps + warp;
   const unsigned long long appended = *p.gq_n;
   const long long n = (long long)min(appended, (unsigned long long)p.gq_cap);
-  for (long long c = gw; 32 * c < n; c += GW)
-    flush_queue<D, TIn, N, B, MODE>(&p, p.gq + 64 * c, (int)min(32LL, n - 32 * c), scratch[warp], lane);
+  for (long long c = gw; kFixChunk * c < n; c += GW)
+    flush_queue<D, TIn, N, B, MODE>(p.job, p.gq + 2 * kFixChunk * c, (int)min((long long)kFixChunk, n - kFixChunk * c),
+                                    scratch[warp], lane);
   if (appended <= (unsigned long long)p.gq_cap) return;
   const long long nwords = ((long long)p.ntiles * RW + 31) / 32;
   for (long long w0 = gw * 32; w0 < nwords; w0 += GW * 32) {
@@ -1520,7 +1517,7 @@ __global__ void __launch_bounds__(32 * kFixWarps) encode_fixup_kernel(const __gr
           whole[warp][1] = make_uint4(0u, 0u, 0u, 0u);
         }
         __syncwarp();
-        flush_queue<D, TIn, N, B, MODE>(&p, whole[warp], 1, scratch[warp], lane);
+        flush_queue<D, TIn, N, B, MODE>(p.job, whole[warp], 1, scratch[warp], lane);
       }
     }
   }
@@ -1541,10 +1538,23 @@ static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_
     if (e != cudaSuccess) return e;
     configured[dev].store(1, std::memory_order_release);
   }
-  int per_sm = 0;
-  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kEncThreads, C::SMEM);
-  if (e != cudaSuccess) return e;
-  if (per_sm < 1) per_sm = 1;
+  // resident CTAs per SM of both kernels, found once per device
+  static std::atomic<int> occ[64][2];
+  int per_sm = dev >= 0 && dev < 64 ? occ[dev][0].load(std::memory_order_acquire) : 0;
+  int fix_sm = dev >= 0 && dev < 64 ? occ[dev][1].load(std::memory_order_acquire) : 0;
+  auto fix = encode_fixup_kernel<D, TIn, N, B, MODE>;
+  if (per_sm == 0 || fix_sm == 0) {
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kEncThreads, C::SMEM);
+    if (e != cudaSuccess) return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&fix_sm, fix, 32 * kFixWarps, 0);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+    if (fix_sm < 1) fix_sm = 1;
+    if (dev >= 0 && dev < 64) {
+      occ[dev][0].store(per_sm, std::memory_order_release);
+      occ[dev][1].store(fix_sm, std::memory_order_release);
+    }
+  }
   int grid = grid_cap * per_sm;
   const int need = (p.ntiles + kEncWarps - 1) / kEncWarps;
   if (grid > need) grid = need;
@@ -1553,15 +1563,19 @@ static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_
   cudaError_t le = cudaGetLastError();
   if (le != cudaSuccess) return le;
   // the fix-up: enough warps for the queue's capacity, up to a full GPU
-  auto fix = encode_fixup_kernel<D, TIn, N, B, MODE>;
-  int fix_sm = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&fix_sm, fix, 32 * kFixWarps, 0);
-  if (e != cudaSuccess) return e;
-  const int64_t chunks = (p.gq_cap + 31) / 32;
-  int64_t fgrid = (int64_t)grid_cap * (fix_sm < 1 ? 1 : fix_sm);
+  FixParams f;
+  f.job = p.gjobs;
+  f.gq = p.gq;
+  f.gq_n = p.gq_n;
+  f.ovf = p.ovf;
+  f.gq_cap = p.gq_cap;
+  f.njobs = p.njobs;
+  f.ntiles = p.ntiles;
+  const int64_t chunks = (p.gq_cap + kFixChunk - 1) / kFixChunk;
+  int64_t fgrid = (int64_t)grid_cap * fix_sm;
   fgrid = std::min<int64_t>(fgrid, (chunks + kFixWarps - 1) / kFixWarps);
   if (fgrid < 1) fgrid = 1;
-  fix<<<(int)fgrid, 32 * kFixWarps, 0, st>>>(p);
+  fix<<<(int)fgrid, 32 * kFixWarps, 0, st>>>(f);
   return cudaGetLastError();
 }
 

@@ -169,11 +169,12 @@ def test_invalid_arguments_rejected_before_launch(tac_host):
 
 
 def test_encode_workspace_size_and_checks(tac_host):
-    """tac_encode_workspace_bytes: per launch group a 64-byte counter block and
-    one bit per warp-tile row (rounded up to 16 bytes) are the minimum; the
-    recommended size adds a queue of one 32-byte entry per 512 angle pairs plus
-    1024.  tac_encode_multi_ws rejects a NULL, misaligned or too small
-    workspace before any device work."""
+    """tac_encode_workspace_bytes: per launch group a 64-byte counter block,
+    one bit per warp-tile row (rounded up to 16 bytes) and a copy of its job
+    table (104 bytes a job, rounded up to 16) are the minimum; the recommended
+    size adds a queue of one 32-byte entry per 512 angle pairs plus 1024.
+    tac_encode_multi_ws rejects a NULL, misaligned or too small workspace
+    before any device work."""
     lib = tac_host.load()
     rows = tac_host._Rows()
     rows.data, rows.dtype, rows.rows, rows.row_stride = 16, 0, 1000, 128
@@ -185,7 +186,7 @@ def test_encode_workspace_size_and_checks(tac_host):
         jobs[i].codes, jobs[i].norms, jobs[i].capacity, jobs[i].slot = buf, buf, 1000, None
     mn = ctypes.c_int64(0)
     rec = lib.tac_encode_workspace_bytes(jobs, 2, ctypes.byref(mn))
-    per_min = 64 + ((250 * 4 + 127) // 128) * 16          # d = 128: 4-row warp tiles
+    per_min = 64 + ((250 * 4 + 127) // 128) * 16 + 112    # d = 128: 4-row warp tiles; one job
     assert mn.value == 2 * per_min
     assert rec == 2 * (per_min + 32 * (1000 * 64 // 512 + 1024))
     assert lib.tac_encode_workspace_bytes(jobs, 2, None) == rec
