@@ -15,21 +15,21 @@
 
 namespace tac {
 cudaError_t launch_encode_16_bf16(const EncParams& p, int n, int b, int mode, int sms,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int phase);
 cudaError_t launch_encode_32_bf16(const EncParams& p, int n, int b, int mode, int sms,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int phase);
 cudaError_t launch_encode_64_bf16(const EncParams& p, int n, int b, int mode, int sms,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int phase);
 cudaError_t launch_encode_128_bf16(const EncParams& p, int n, int b, int mode, int sms,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int phase);
 cudaError_t launch_encode_16_f32(const EncParams& p, int n, int b, int mode, int sms,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int phase);
 cudaError_t launch_encode_32_f32(const EncParams& p, int n, int b, int mode, int sms,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int phase);
 cudaError_t launch_encode_64_f32(const EncParams& p, int n, int b, int mode, int sms,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int phase);
 cudaError_t launch_encode_128_f32(const EncParams& p, int n, int b, int mode, int sms,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int phase);
 cudaError_t launch_decode_16_bf16(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
 cudaError_t launch_decode_32_bf16(const DecParams& p, int n, int b, int mode, int sms,
@@ -47,14 +47,15 @@ cudaError_t launch_decode_64_f32(const DecParams& p, int n, int b, int mode, int
 cudaError_t launch_decode_128_f32(const DecParams& p, int n, int b, int mode, int sms,
                                  cudaStream_t st);
 
+// phase: 1 the encode kernel, 2 its fix-up, 3 both in order (one stream).
 static cudaError_t launch_encode(int d, int dtype, int n, int b, int mode, const EncParams& p, int sms,
-                                 cudaStream_t st) {
+                                 cudaStream_t st, int phase) {
   const bool bf = dtype == TAC_BF16;
   switch (d) {
-    case 16: return bf ? launch_encode_16_bf16(p, n, b, mode, sms, st) : launch_encode_16_f32(p, n, b, mode, sms, st);
-    case 32: return bf ? launch_encode_32_bf16(p, n, b, mode, sms, st) : launch_encode_32_f32(p, n, b, mode, sms, st);
-    case 64: return bf ? launch_encode_64_bf16(p, n, b, mode, sms, st) : launch_encode_64_f32(p, n, b, mode, sms, st);
-    case 128: return bf ? launch_encode_128_bf16(p, n, b, mode, sms, st) : launch_encode_128_f32(p, n, b, mode, sms, st);
+    case 16: return bf ? launch_encode_16_bf16(p, n, b, mode, sms, st, phase) : launch_encode_16_f32(p, n, b, mode, sms, st, phase);
+    case 32: return bf ? launch_encode_32_bf16(p, n, b, mode, sms, st, phase) : launch_encode_32_f32(p, n, b, mode, sms, st, phase);
+    case 64: return bf ? launch_encode_64_bf16(p, n, b, mode, sms, st, phase) : launch_encode_64_f32(p, n, b, mode, sms, st, phase);
+    case 128: return bf ? launch_encode_128_bf16(p, n, b, mode, sms, st, phase) : launch_encode_128_f32(p, n, b, mode, sms, st, phase);
   }
   return cudaErrorInvalidValue;
 }
@@ -531,18 +532,30 @@ int run_encode(std::vector<EncGroup>& groups, uint8_t* ws, int64_t ws_bytes, cud
   caps.resize(groups.size());
   for (size_t g = 0; g < groups.size(); ++g) gtiles[g] = groups[g].p.ntiles;
   sm_shares(gtiles.data(), (int)groups.size(), sms, caps.data());
-  GroupFork fork(st, (int)groups.size());
-  if (fork.error() != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(fork.error()));
-  for (size_t g = 0; g < groups.size(); ++g) {
-    const EncGroup& G = groups[g];
-    e = tac::launch_encode(G.d, G.dt, G.na, G.nb, G.mode, G.p, caps[g], fork.stream((int)g));
-    if (e != cudaSuccess) {
-      fork.join();
-      return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+  // A call that gives every launch the whole GPU runs its encode launches
+  // first and then all fix-ups side by side: an encode launch fills every SM,
+  // so a fix-up queued behind it on its stream would not overlap the next
+  // group's encode and the fix-ups would run one after another.  A small call
+  // (launches on shares of the SMs, side by side) chains each group's fix-up
+  // to its encode.
+  bool whole = true;
+  for (size_t g = 0; g < groups.size(); ++g) whole = whole && caps[g] == sms;
+  const int rounds = whole && groups.size() > 1 ? 2 : 1;
+  for (int r = 0; r < rounds; ++r) {
+    const int phase = rounds == 1 ? 3 : r + 1;
+    GroupFork fork(st, (int)groups.size());
+    if (fork.error() != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(fork.error()));
+    for (size_t g = 0; g < groups.size(); ++g) {
+      const EncGroup& G = groups[g];
+      e = tac::launch_encode(G.d, G.dt, G.na, G.nb, G.mode, G.p, caps[g], fork.stream((int)g), phase);
+      if (e != cudaSuccess) {
+        fork.join();
+        return fail(TAC_E_CUDA, "%s: launch failed: %s", who, cudaGetErrorString(e));
+      }
     }
+    e = fork.join();
+    if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(e));
   }
-  e = fork.join();
-  if (e != cudaSuccess) return fail(TAC_E_CUDA, "%s: %s", who, cudaGetErrorString(e));
   return 0;
 }
 

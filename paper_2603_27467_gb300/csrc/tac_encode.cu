@@ -1526,8 +1526,9 @@ __global__ void __launch_bounds__(32 * kFixWarps) encode_fixup_kernel(const __gr
 // ---------------------------------------------------------------------------
 // Host-side launch helpers (called from tac_api.cu).
 // ---------------------------------------------------------------------------
+// phase: bit 0 launches the encode kernel, bit 1 its fix-up (3: both, in order).
 template <int D, typename TIn, int N, int B, int MODE>
-static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_t st) {
+static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_t st, int phase) {
   using C = Enc<D, TIn, N, B, MODE>;
   auto kern = encode_kernel<D, TIn, N, B, MODE>;
   static std::atomic<int> configured[64];   // per device; concurrent first calls set the same
@@ -1558,10 +1559,13 @@ static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_
   int grid = grid_cap * per_sm;
   const int need = (p.ntiles + kEncWarps - 1) / kEncWarps;
   if (grid > need) grid = need;
-  if (grid < 1) return cudaSuccess;
-  kern<<<grid, kEncThreads, C::SMEM, st>>>(p);
-  cudaError_t le = cudaGetLastError();
-  if (le != cudaSuccess) return le;
+  if (grid < 1) return cudaSuccess;   // no rows: neither kernel runs
+  if (phase & 1) {
+    kern<<<grid, kEncThreads, C::SMEM, st>>>(p);
+    const cudaError_t le = cudaGetLastError();
+    if (le != cudaSuccess) return le;
+  }
+  if (!(phase & 2)) return cudaSuccess;
   // the fix-up: enough warps for the queue's capacity, up to a full GPU
   FixParams f;
   f.job = p.gjobs;
@@ -1582,15 +1586,15 @@ static cudaError_t launch_encode_v(const EncParams& p, int grid_cap, cudaStream_
 // One kernel per supported (n, norm bits, mode): n in {2, 4, ..., 256, 48, 56},
 // (B, mode) in {(4, linear), (4, log), (8, linear), (8, log), (32, fp32)}.
 template <int D, typename TIn>
-static cudaError_t launch_encode_t(const EncParams& p, int n, int b, int mode, int sms, cudaStream_t st) {
+static cudaError_t launch_encode_t(const EncParams& p, int n, int b, int mode, int sms, cudaStream_t st, int phase) {
 #define TAC_ENC_N(NN)                                                                                   \
   if (n == NN) {                                                                                        \
-    if (mode == TAC_NORM_FP32) return b == 32 ? launch_encode_v<D, TIn, NN, 32, TAC_NORM_FP32>(p, sms, st) \
+    if (mode == TAC_NORM_FP32) return b == 32 ? launch_encode_v<D, TIn, NN, 32, TAC_NORM_FP32>(p, sms, st, phase) \
                                               : cudaErrorInvalidValue;                                  \
-    if (b == 4) return mode == TAC_NORM_LOG ? launch_encode_v<D, TIn, NN, 4, TAC_NORM_LOG>(p, sms, st)     \
-                                            : launch_encode_v<D, TIn, NN, 4, TAC_NORM_LINEAR>(p, sms, st); \
-    if (b == 8) return mode == TAC_NORM_LOG ? launch_encode_v<D, TIn, NN, 8, TAC_NORM_LOG>(p, sms, st)     \
-                                            : launch_encode_v<D, TIn, NN, 8, TAC_NORM_LINEAR>(p, sms, st); \
+    if (b == 4) return mode == TAC_NORM_LOG ? launch_encode_v<D, TIn, NN, 4, TAC_NORM_LOG>(p, sms, st, phase)     \
+                                            : launch_encode_v<D, TIn, NN, 4, TAC_NORM_LINEAR>(p, sms, st, phase); \
+    if (b == 8) return mode == TAC_NORM_LOG ? launch_encode_v<D, TIn, NN, 8, TAC_NORM_LOG>(p, sms, st, phase)     \
+                                            : launch_encode_v<D, TIn, NN, 8, TAC_NORM_LINEAR>(p, sms, st, phase); \
     return cudaErrorInvalidValue;                                                                       \
   }
   TAC_ENC_N(2) TAC_ENC_N(4) TAC_ENC_N(8) TAC_ENC_N(16) TAC_ENC_N(32) TAC_ENC_N(64) TAC_ENC_N(128)
@@ -1614,8 +1618,8 @@ static cudaError_t launch_encode_t(const EncParams& p, int n, int b, int mode, i
 #endif
 #define TAC_ENC_INSTANCE(DD, NAME, T)                                                                 \
   cudaError_t launch_encode_##DD##_##NAME(const EncParams& p, int n, int b, int mode, int sms,       \
-                                          cudaStream_t st) {                                         \
-    return launch_encode_t<DD, T>(p, n, b, mode, sms, st);                                           \
+                                          cudaStream_t st, int phase) {                              \
+    return launch_encode_t<DD, T>(p, n, b, mode, sms, st, phase);                                    \
   }
 #if defined(TAC_ALL_INSTANCES) || (TAC_INST_D == 16 && TAC_INST_BF16)
 TAC_ENC_INSTANCE(16, bf16, __nv_bfloat16)
