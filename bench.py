@@ -397,11 +397,11 @@ def run_e2e(tac, ws, world, dev, steps, chunk_blocks, step_bytes, barrier):
     for _ in range(2):                                # warm-up
         one_step()
     barrier()
-    # Five timed rounds of `steps` steps; the median round is reported (rounds
-    # on the shared host show intermittent halvings of the link rate, listed
-    # in round_ms_per_step).
+    # Nine timed rounds of `steps` steps; the median round is reported (rounds
+    # on the shared host alternate between two link rates, about 2.5x apart,
+    # listed in round_ms_per_step).
     rounds = []
-    for _ in range(5):
+    for _ in range(9):
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(s_in)
