@@ -47,8 +47,8 @@ MEASURED_TRAFFIC = {
                "bytes_per_row": 338.776},
     "decode": {"sources": ("tac_common.cuh", "tac_decode.cu"), "sha256_16": "af89c8435cfc002c",
                "bytes_per_row": 305.386},
-    "attend": {"sources": ("tac_common.cuh", "tac_attend.cuh", "tac_attend.cu"), "sha256_16": "2ca20d9ce47a635b",
-               "bytes_per_row": 216.889},
+    "attend": {"sources": ("tac_common.cuh", "tac_attend.cuh", "tac_attend.cu"), "sha256_16": "4e341a7176bc2a95",
+               "bytes_per_row": 221.787},
 }
 
 
@@ -492,8 +492,9 @@ def run_attend(args):
         "roofline": {"bound": "hbm", "kernel": "attend_partial + attend_combine", "achieved": gbs, "peak": hbm,
                      "unit": "GB/s", "frac": gbs / hbm, "peak_source": f"{peak_kind} hbm_gbs",
                      "traffic": measured_traffic("attend", w.layers * w.heads * T),
-                     "traffic_note": "attend_partial DRAM bytes per token-head (all launches of a step) from ncu "
-                                     "at 4096 tokens, scaled by token-heads; null once the kernel source changes"},
+                     "traffic_note": "attend_partial + attend_combine DRAM bytes per token-head (all launches of "
+                                     "a step) from ncu at 4096 tokens, scaled by token-heads; null once the kernel "
+                                     "source changes"},
         "gpu_launches": 2 * args.steps * (1 + (len(jobs) - 1) // tac.ATTEND_MAX_JOBS), "clocks": clocks}), flush=True)
 
 
