@@ -21,17 +21,19 @@
 //      test: a candidate edge from an arctangent approximation (the angle of
 //      (|E|, |O|) is pi/4 + atan((|O| - |E|) / (|O| + |E|)), with an odd cubic
 //      for atan on [-1, 1], max error 0.00496 rad), then the sign of the cross
-//      product of (E, O) with the edge direction.  The test is
-//      certified by a rigorous bound on the fp32 error; the pairs it does not
-//      certify (about 1e-4 of them) are re-decided by the warp from exact
-//      sums of the staged input;
+//      product of (E, O) with the edge direction.  The test is certified by a
+//      bound on the fp32 error;
 //   4. Eq. 2 norm codes (linear, or on log2 r) against the row's minimum and
-//      maximum pair norms; a code whose fp32 Eq. 2 value lies within a band
-//      of a rounding midpoint is re-decided from exact sums as well, and the
-//      fp32 extremes are stored as the header (r_min, r_max);
+//      maximum pair norms, certified the same way against a band around each
+//      rounding midpoint; the fp32 extremes are stored as the header
+//      (r_min, r_max);
 //   5. each lane packs its 8 codes LSB-first; the warp stages its records in
 //      shared memory and writes them with one 16-byte store per lane (contiguous
-//      slots) or per row (scatter-append slots).
+//      slots) or per row (scatter-append slots);
+//   6. the codes not certified (about 4e-4 of them) go to a per-warp queue in
+//      shared memory, moved to a queue in the call's workspace when it fills;
+//      a fix-up kernel after the encode re-decides them (a double-float second
+//      look, then exact integer sums of the row) and patches the records.
 #include <algorithm>
 #include <atomic>
 
