@@ -349,7 +349,9 @@ def decode(cache: Cache, cfg: LayerCfg, rows: int | None = None, dtype=None, y=N
 class Prepared:
     """A batched call with its job array marshalled once: calling it makes only
     the C call.  The jobs' tensors must stay allocated (their addresses are in
-    the array) and the jobs unchanged while it is used."""
+    the array) and the jobs unchanged while it is used.  A prepared encode or
+    attention call reuses one workspace on every call, so its calls must not
+    overlap in time: make them on one stream, or order the streams."""
 
     def __init__(self, fn, arr, n, extra, keep):
         self._fn, self._arr, self._n, self._extra, self._keep = fn, arr, n, extra, keep
