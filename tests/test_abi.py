@@ -260,3 +260,23 @@ def test_binding_constants_match_header(tac_host):
     assert define("TAC_MAX_JOBS") == tac_host.MAX_JOBS
     assert define("TAC_ATTEND_MAX_JOBS") == tac_host.ATTEND_MAX_JOBS
     assert define("TAC_ATTEND_SPLIT") == 256
+
+
+def test_launch_count_matches_the_grouping(tac_host):
+    """launch_count (the bench's gpu_launches): jobs with rows grouped by kernel
+    shape (d, dtype, n, norm bits, norm mode), at most MAX_JOBS to a group; an
+    encode group launches the encode kernel and its fix-up, a decode group one
+    kernel."""
+    import torch
+    tac = tac_host
+    k_cfg, v_cfg = tac.LayerCfg(128, 64, 8, 0), tac.LayerCfg(128, 256, 4, 1)
+    x = torch.zeros((4, 128), dtype=torch.bfloat16)
+    empty = torch.zeros((0, 128), dtype=torch.bfloat16)
+    enc = [tac.EncodeJob(k_cfg, x, None), tac.EncodeJob(k_cfg, x, None), tac.EncodeJob(v_cfg, x, None),
+           tac.EncodeJob(v_cfg, empty, None), tac.EncodeJob(k_cfg, x.float(), None)]
+    assert tac.launch_count(enc) == 2 * 3            # (k, bf16), (v, bf16), (k, fp32); the empty job adds none
+    many = [tac.EncodeJob(k_cfg, x, None)] * (tac.MAX_JOBS + 1)
+    assert tac.launch_count(many) == 2 * 2
+    dec = [tac.DecodeJob(k_cfg, None, x), tac.DecodeJob(v_cfg, None, x), tac.DecodeJob(v_cfg, None, empty)]
+    assert tac.launch_count(dec) == 2
+    assert tac.launch_count([]) == 0
