@@ -217,10 +217,14 @@ int tac_decode(const void* codes, const void* norms, const tac_layer_cfg* cfg, t
  * CUDA graph.  A call with fewer than 640 warp tiles (4-row d = 128 tiles,
  * 8-row d = 64 tiles, ...) per SM in all gives each launch a share of the SMs
  * in proportion to its tiles, so that its launches run side by side; larger
- * calls give every launch the whole GPU.  The first call with several launches
- * on a device creates three streams and four events (kept for the process);
- * make it outside stream capture.  With `slot` the rows of a decode step land at per-sequence record
- * slots (streaming append).  Jobs must not write overlapping slots.
+ * calls give every launch the whole GPU.  Each launch is followed by its
+ * fix-up kernel (see tac_encode_multi_ws): in a small call on the launch's
+ * stream right after it, in a larger one after all of the call's encode
+ * launches (a second fork / join), the fix-ups side by side.  The first call
+ * with several launches on a device creates three streams and four events
+ * (kept for the process); make it outside stream capture.  With `slot` the
+ * rows of a decode step land at per-sequence record slots (streaming append).
+ * Jobs must not write overlapping slots.
  */
 int tac_encode_multi(const tac_encode_job* jobs, int njobs, tac_stream_t stream);
 
